@@ -1,0 +1,352 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix, not against itself.
+
+Each test names the passage it pins.  None of these needs a GPU.
+"""
+import itertools
+import math
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+from scipy.spatial import distance
+
+from oracle import rift_oracle as O
+from synth import workloads as W
+
+F32 = np.float32
+
+
+# ---------------------------------------------------------------- Eq. 1 (Section 2.3 Stage 1)
+
+def test_eq1_hand_case():
+    # V = (1, 0), t = (0.6, 0.8), B = {(1, 0), (0, 1)}: s = 0.6 - (1 + 0)/2 = 0.1
+    V = torch.tensor([[1.0, 0.0]], dtype=torch.float64)
+    t = torch.tensor([0.6, 0.8], dtype=torch.float64)
+    B = torch.tensor([[1.0, 0.0], [0.0, 1.0]], dtype=torch.float64)
+    assert float(O.margin(V, t, B)[0]) == pytest.approx(0.1, abs=1e-15)
+
+
+def test_eq1_tile_equal_to_query():
+    # V = t gives s = 1 - mean_j B_j . t
+    g = torch.Generator().manual_seed(1)
+    t = O.l2norm(torch.randn(16, generator=g, dtype=torch.float64))
+    B = O.l2norm(torch.randn(5, 16, generator=g, dtype=torch.float64))
+    s = O.margin(t[None, :], t, B)
+    assert float(s[0]) == pytest.approx(1.0 - float((B @ t).mean()), abs=1e-14)
+
+
+def test_eq1_without_background_is_cosine():
+    # M = 0: s_i = cos(V_i, t) (scipy's cosine distance is 1 - cos)
+    rng = np.random.default_rng(2)
+    X = rng.standard_normal((7, 33))
+    t = rng.standard_normal(33)
+    s = O.margin(O.l2norm(torch.tensor(X)), O.l2norm(torch.tensor(t)), torch.zeros(0, 33, dtype=torch.float64))
+    ref = [1.0 - distance.cosine(x, t) for x in X]
+    np.testing.assert_allclose(s.numpy(), ref, rtol=0, atol=1e-13)
+
+
+def test_token_relevance_matches_scipy_cosines():
+    rng = np.random.default_rng(3)
+    X = rng.standard_normal((11, 24))
+    t = rng.standard_normal(24)
+    B = rng.standard_normal((4, 24))
+    r = O.token_relevance(torch.tensor(X), O.l2norm(torch.tensor(t)), O.l2norm(torch.tensor(B)))
+    ref = [(1 - distance.cosine(x, t)) - np.mean([1 - distance.cosine(x, b) for b in B]) for x in X]
+    np.testing.assert_allclose(r.numpy(), ref, rtol=0, atol=1e-13)
+
+
+def test_tile_embedding_is_direction_of_the_pooled_tokens():
+    rng = np.random.default_rng(4)
+    X = torch.tensor(rng.standard_normal((9, 12)))
+    V = O.tile_embedding(X)
+    s = X.sum(0)
+    np.testing.assert_allclose(V.numpy(), (s / s.norm()).numpy(), atol=1e-15)
+    np.testing.assert_allclose(O.tile_embedding(3.5 * X).numpy(), V.numpy(), atol=1e-15)
+    assert float(V.norm()) == pytest.approx(1.0, abs=1e-15)
+
+
+def test_query_embedding_templates():
+    E = torch.tensor([[3.0, 4.0, 0.0], [0.0, 0.0, 2.0], [1.0, 0.0, 0.0]], dtype=torch.float64)
+    # one template, one id: t = E[id] / ||E[id]||
+    np.testing.assert_allclose(O.query_embedding(E, [0]).numpy(), [0.6, 0.8, 0.0], atol=1e-15)
+    # two templates [0] and [1]: l2norm((0.6, 0.8, 0) + (0, 0, 1)) = (0.6, 0.8, 1)/sqrt(2)
+    np.testing.assert_allclose(O.query_embedding(E, [[0], [1]]).numpy(),
+                               np.array([0.6, 0.8, 1.0]) / math.sqrt(2), atol=1e-15)
+    # one template [0, 2]: mean (2, 2, 0) -> (1, 1, 0)/sqrt(2)
+    np.testing.assert_allclose(O.query_embedding(E, [0, 2]).numpy(), np.array([1, 1, 0]) / math.sqrt(2), atol=1e-15)
+    B = O.background_embeddings(E, [1, 0])
+    np.testing.assert_allclose(B.numpy(), [[0, 0, 1], [0.6, 0.8, 0]], atol=1e-15)
+
+
+# ---------------------------------------------------------------- kNN smoothing (Appendix B Step 2)
+
+def _beats(G, i, a, b):
+    """a ranks before b as a neighbour of i: larger similarity, then the lower index."""
+    return G[i, a] > G[i, b] or (G[i, a] == G[i, b] and a < b)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_knn_neighbours_brute_force(seed):
+    rng = np.random.default_rng(seed)
+    N = 7
+    G = rng.integers(-3, 4, size=(N, N)).astype(F32)  # small integers force many ties
+    for m in range(0, N):
+        nbr = O.knn_neighbours(G, m)
+        for i in range(N):
+            others = [j for j in range(N) if j != i]
+            # the unique m-subset whose every member beats every non-member
+            sets = [set(S) for S in itertools.combinations(others, m)
+                    if all(_beats(G, i, a, b) for a in S for b in others if b not in S)]
+            assert len(sets) == 1
+            assert set(nbr[i].tolist()) == sets[0]
+            # rank order
+            assert all(_beats(G, i, nbr[i][k], nbr[i][k + 1]) for k in range(m - 1))
+
+
+def test_knn_m_capped_at_n_minus_one():
+    G = np.eye(3, dtype=F32)
+    assert O.knn_neighbours(G, 6).shape == (3, 2)
+
+
+def test_smooth_hand_case_and_special_cases():
+    s = np.array([0.0, 1.0, 2.0, 3.0], dtype=F32)
+    nbr = np.array([[1], [0], [3], [2]])
+    np.testing.assert_array_equal(O.smooth(s, nbr), np.array([0.5, 0.5, 2.5, 2.5], dtype=F32))
+    # m = 0: no smoothing, bit-exact
+    np.testing.assert_array_equal(O.smooth(s, np.zeros((4, 0), dtype=np.int64)), s)
+    # m = N - 1: every tile averages the whole scene; sums run in index order, so the results
+    # are bit-equal and min-max gives u = 1 everywhere
+    rng = np.random.default_rng(0)
+    s = rng.standard_normal(5).astype(F32)
+    nbr = np.array([[j for j in range(5) if j != i] for i in range(5)])[:, ::-1].copy()
+    st = O.smooth(s, nbr)
+    assert len(set(st.tolist())) == 1
+    assert np.all(O.minmax_normalize(st) == 1.0)
+
+
+# ---------------------------------------------------------------- min-max and tau (Stage 1; App. B Step 3)
+
+def test_minmax_invariants_and_top_tile_kept():
+    rng = np.random.default_rng(5)
+    for _ in range(20):
+        s = rng.standard_normal(rng.integers(2, 50)).astype(F32)
+        u = O.minmax_normalize(s)
+        assert u.dtype == F32
+        assert u[np.argmax(s)] == 1.0 and u[np.argmin(s)] == 0.0
+        assert np.all((u >= 0) & (u <= 1))
+        kept = O.retained(u, 0.37)
+        assert int(np.argmax(s)) in kept  # "no query can be left with zero tiles"
+
+
+def test_minmax_two_tiles_and_all_equal():
+    assert O.minmax_normalize(np.array([0.3, -0.2], dtype=F32)).tolist() == [1.0, 0.0]
+    assert O.minmax_normalize(np.array([0.25] * 4, dtype=F32)).tolist() == [1.0] * 4
+    assert O.minmax_normalize(np.array([7.0], dtype=F32)).tolist() == [1.0]
+
+
+def test_threshold_is_greater_or_equal():
+    # u = 0.37f exactly must be kept (Appendix B: u_i >= 0.37; Listing 1: >=)
+    s = np.array([0.0, F32(0.37), 1.0], dtype=F32)
+    u = O.minmax_normalize(s)
+    assert u[1] == F32(0.37)
+    assert O.retained(u, 0.37) == [1, 2]
+    assert O.retained(np.array([np.nextafter(F32(0.37), F32(0))], dtype=F32), 0.37) == []
+
+
+def test_nonfinite_scores_raise():
+    with pytest.raises(O.OracleError):
+        O.minmax_normalize(np.array([0.0, np.nan], dtype=F32))
+    with pytest.raises(O.OracleError):
+        O.top_b(np.array([0.0, np.inf], dtype=F32), 1)
+
+
+# ---------------------------------------------------------------- Eq. 2 budget rule (Stage 2)
+
+def _exact_argmax(p: Fraction, pol):
+    """Eq. 2 in exact rational arithmetic; returns (budget, margin to the runner-up)."""
+    lam = Fraction(str(pol.lam))
+    U = [p * Fraction(str(a)) + (1 - p) * Fraction(str(b)) - lam * Fraction(str(e))
+         for a, b, e in zip(pol.alpha_pos, pol.alpha_neg, pol.energy)]
+    order = sorted(range(len(U)), key=lambda k: (-U[k], k))
+    margin = U[order[0]] - U[order[1]] if len(U) > 1 else Fraction(1)
+    return pol.C[order[0]], margin
+
+
+@pytest.mark.parametrize("pol", [W.RIFT_POLICY, W.RIFT_POLICY_SKEW])
+def test_budget_truth_table_against_exact_arithmetic(pol):
+    for k in range(0, 101):
+        p32 = F32(k / 100)
+        b_exact, margin = _exact_argmax(Fraction(float(p32)), pol)
+        if margin > Fraction(1, 10 ** 5):  # fp32 rounding (~1e-7) cannot flip it
+            assert O.budget(float(p32), pol) == b_exact, (k, b_exact)
+
+
+def test_budget_walkthrough_inversion():
+    # Appendix B Step 4: confident (object) tiles get 72 tokens, low-p clutter tiles 288
+    pol = W.RIFT_POLICY
+    assert O.budget(1.0, pol) == 72
+    for p in (0.0, 0.2, 0.37, 0.5, 0.7):
+        assert O.budget(p, pol) == 288
+    # the skewed policy reaches every budget of C as p grows
+    got = {O.budget(k / 100, W.RIFT_POLICY_SKEW) for k in range(101)}
+    assert got == set(W.RIFT_POLICY_SKEW.C)
+
+
+def test_budget_ties_go_to_the_cheaper_budget():
+    pol = W.Policy(tau=0.37, C=(72, 144, 288), alpha_pos=(0.5, 0.5, 0.5), alpha_neg=(0.5, 0.5, 0.5),
+                   energy=(0.0, 0.0, 0.0), lam=0.0)
+    assert O.budget(0.3, pol) == 72
+
+
+# ---------------------------------------------------------------- top-b (Stage 2: dominant tokens)
+
+@pytest.mark.parametrize("seed", range(8))
+def test_top_b_brute_force_with_ties(seed):
+    rng = np.random.default_rng(100 + seed)
+    n = 9
+    r = (rng.integers(-2, 3, size=n) * 0.25).astype(F32)
+    r[rng.integers(0, n)] = F32(-0.0)
+    r[rng.integers(0, n)] = F32(0.0)
+    for b in range(1, n + 1):
+        got = O.top_b(r, b)
+        assert got == sorted(got) and len(got) == b
+        chosen = set(got)
+        rest = [k for k in range(n) if k not in chosen]
+        for a in chosen:
+            for c in rest:  # every selected token beats every unselected one
+                assert r[a] > r[c] or (r[a] == r[c] and a < c)
+
+
+def test_top_b_full_budget_keeps_everything():
+    r = np.random.default_rng(0).standard_normal(576).astype(F32)
+    assert O.top_b(r, 576) == list(range(576))
+
+
+# ---------------------------------------------------------------- packing accounting
+
+def test_pack_accounting_and_full_budget_equals_exhaustive():
+    wl = W.TINY
+    sc = W.make_scene(wl.scene, wl.decoder.vocab)
+    # full budget on all tiles: tau = 0 keeps every tile, C = {576} keeps every token
+    sel = O.select(sc.X, sc.embed, sc.query_ids, sc.bg_ids, wl.knn_m, W.KEEP_ALL)
+    assert sel.kept == list(range(wl.scene.N))
+    assert all(s == list(range(576)) for s in sel.sel)
+    H0, cu, pos = O.pack(sc.X, sc.embed, sel.kept, sel.sel, sc.sys_ids, sc.query_ids)
+    S, Q = wl.scene.S, wl.scene.Q
+    L = S + 576 + Q
+    assert cu == [L * i for i in range(wl.scene.N + 1)]
+    assert pos == list(range(L)) * wl.scene.N
+    for i in range(wl.scene.N):
+        exhaustive = torch.cat([sc.embed[sc.sys_ids], sc.X[i].to(torch.bfloat16), sc.embed[sc.query_ids]])
+        assert torch.equal(H0[cu[i]:cu[i + 1]], exhaustive)
+
+
+def test_pack_ragged_accounting():
+    wl = W.TINY
+    sc = W.make_scene(wl.scene, wl.decoder.vocab)
+    sel = O.select(sc.X, sc.embed, sc.query_ids, sc.bg_ids, wl.knn_m, wl.policy)
+    H0, cu, pos = O.pack(sc.X, sc.embed, sel.kept, sel.sel, sc.sys_ids, sc.query_ids)
+    S, Q = wl.scene.S, wl.scene.Q
+    assert cu[-1] == H0.shape[0] == sum(S + b + Q for b in sel.budgets)
+    assert all(b in wl.policy.C for b in sel.budgets)
+    assert [len(s) for s in sel.sel] == sel.budgets
+    for j, (i, idx) in enumerate(zip(sel.kept, sel.sel)):
+        rows = H0[cu[j]:cu[j + 1]]
+        assert torch.equal(rows[S:S + len(idx)], sc.X[i][idx].to(torch.bfloat16))
+        assert pos[cu[j]:cu[j + 1]] == list(range(cu[j + 1] - cu[j]))
+
+
+# ---------------------------------------------------------------- decoder prefill (Section 2.1)
+
+def _tiny_layers(dec, seed=0):
+    return [W.make_layer(dec, l, "cpu", seed) for l in range(dec.n_layers)], W.make_final_norm(dec, "cpu", seed)
+
+
+def _textbook_prefill(H0, layers, g_final, dec):
+    """Second, independent formulation: torch SDPA (is_causal), complex-number RoPE,
+    F.rms_norm and F.silu, all in fp64."""
+    h = H0.to(torch.float64)
+    L = h.shape[0]
+    hd, H = dec.head_dim, dec.n_heads
+    half = hd // 2
+    freqs = 1.0 / (dec.rope_theta ** (torch.arange(0, hd, 2, dtype=torch.float64) / hd))
+    rot = torch.polar(torch.ones(L, half, dtype=torch.float64), torch.outer(torch.arange(L, dtype=torch.float64), freqs))
+
+    def rope(x):  # x [L, H, hd]; pairs (j, j + hd/2) as one complex number
+        z = torch.complex(x[..., :half], x[..., half:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], dim=-1)
+
+    for Wl in layers:
+        f = {k: v.to(torch.float64) for k, v in Wl.items()}
+        x = F.rms_norm(h, (dec.d,), f["g_attn"], dec.eps)
+        q = rope((x @ f["wq"].T).view(L, H, hd)).transpose(0, 1)
+        k = rope((x @ f["wk"].T).view(L, H, hd)).transpose(0, 1)
+        v = (x @ f["wv"].T).view(L, H, hd).transpose(0, 1)
+        a = F.scaled_dot_product_attention(q, k, v, is_causal=True).transpose(0, 1).reshape(L, dec.d)
+        h = h + a @ f["wo"].T
+        x = F.rms_norm(h, (dec.d,), f["g_ffn"], dec.eps)
+        h = h + (F.silu(x @ f["wg"].T) * (x @ f["wu"].T)) @ f["wd"].T
+    return F.rms_norm(h, (dec.d,), g_final.to(torch.float64), dec.eps)
+
+
+def test_prefill_matches_textbook_formulation():
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    H0 = (torch.randn(37, dec.d, generator=torch.Generator().manual_seed(0))).to(torch.bfloat16)
+    out = O.prefill_sequence(H0, lambda l: layers[l], gf, dec)
+    ref = _textbook_prefill(H0, layers, gf, dec)
+    assert torch.allclose(out, ref, rtol=0, atol=1e-10)
+
+
+def test_prefill_single_token_closed_form():
+    # L = 1: softmax over one key is 1 and RoPE at position 0 is the identity, so each layer is
+    # h += W_o W_v x then the SwiGLU FFN.
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    h = torch.randn(1, dec.d, generator=torch.Generator().manual_seed(1), dtype=torch.float64)
+    ref = h.clone()
+    for Wl in layers:
+        f = {k: v.to(torch.float64) for k, v in Wl.items()}
+        x = ref / torch.sqrt((ref ** 2).mean() + dec.eps) * f["g_attn"]
+        ref = ref + (x @ f["wv"].T) @ f["wo"].T
+        x = ref / torch.sqrt((ref ** 2).mean() + dec.eps) * f["g_ffn"]
+        g = x @ f["wg"].T
+        ref = ref + ((g / (1 + torch.exp(-g))) * (x @ f["wu"].T)) @ f["wd"].T
+    ref = ref / torch.sqrt((ref ** 2).mean() + dec.eps) * gf.to(torch.float64)
+    out = O.prefill_sequence(h, lambda l: layers[l], gf, dec)
+    assert torch.allclose(out, ref, rtol=0, atol=1e-12)
+
+
+def test_prefill_is_causal():
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    H0 = torch.randn(20, dec.d, generator=torch.Generator().manual_seed(2), dtype=torch.float64)
+    full = O.prefill_sequence(H0, lambda l: layers[l], gf, dec)
+    prefix = O.prefill_sequence(H0[:12], lambda l: layers[l], gf, dec)
+    assert torch.allclose(full[:12], prefix, rtol=0, atol=1e-12)
+    H1 = H0.clone()
+    H1[15] += 1.0
+    changed = O.prefill_sequence(H1, lambda l: layers[l], gf, dec)
+    assert torch.allclose(changed[:15], full[:15], rtol=0, atol=1e-12)
+    assert not torch.allclose(changed[15:], full[15:])
+
+
+def test_rope_rotation_preserves_norm_and_relative_position():
+    x = torch.randn(5, 2, 64, generator=torch.Generator().manual_seed(3), dtype=torch.float64)
+    y = O.rope(x, torch.arange(5), 1e4)
+    assert torch.allclose(x.norm(dim=-1), y.norm(dim=-1), atol=1e-12)
+    assert torch.allclose(O.rope(x, torch.zeros(5, dtype=torch.long), 1e4), x, atol=0)
+    # <R(p) a, R(q) b> depends on q - p only
+    a, b = x[0, 0], x[1, 0]
+    d1 = O.rope(a.view(1, 1, 64), torch.tensor([3]), 1e4).flatten() @ O.rope(b.view(1, 1, 64), torch.tensor([7]), 1e4).flatten()
+    d2 = O.rope(a.view(1, 1, 64), torch.tensor([10]), 1e4).flatten() @ O.rope(b.view(1, 1, 64), torch.tensor([14]), 1e4).flatten()
+    assert float(d1) == pytest.approx(float(d2), abs=1e-12)
+
+
+def test_attention_matches_sdpa():
+    q, k, v = (torch.randn(13, 3, 16, generator=torch.Generator().manual_seed(s), dtype=torch.float64) for s in (4, 5, 6))
+    ref = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1),
+                                         is_causal=True).transpose(0, 1)
+    assert torch.allclose(O.causal_attention(q, k, v), ref, atol=1e-13)
