@@ -1,0 +1,347 @@
+"""Benchmark of Rift's hot path on GB300: one step = one scene query through every stage
+(query prep, Eq. 1 scoring, kNN smoothing, min-max + tau pruning, Eq. 2 budgets, top-b
+selection, ragged packing, 32-layer prefill of the retained sequences).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload rift400_7b] [--impl reference]
+
+Prints one JSON line.  value = retained prefill tokens/s over all ranks (each rank runs its
+own replica of the scene query: the queries are independent, there is no collective on the
+data path).  Inputs (X: 1.9 GB, weights: 13 GB) are larger than L2, so no flush is needed.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+import torch  # noqa: E402
+
+from synth import workloads as W  # noqa: E402
+
+METRIC = "retained prefill tokens/s"
+UNIT = "tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="rift400_7b", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--impl", default="rift", choices=["rift", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------------------------------ dist
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max(x: float, ws: int) -> float:
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def reduce_sum(x: float, ws: int) -> float:
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            uuid = "GPU-" + str(torch.cuda.get_device_properties(self.idx).uuid)
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", uuid, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------ oracle arm
+
+def oracle_sample(wl, sc, n_tiles: int, n_layers: int, budget: int, device):
+    """Time the CPU oracle on a bounded sample of the workload: Eq. 1 scoring + selection of
+    n_tiles tiles, and the prefill of one sequence with `budget` vision tokens through n_layers
+    layers.  Returns (seconds per tile, seconds per prefill token per layer, cores, sample text)."""
+    from oracle import rift_oracle as O
+    torch.set_num_threads(len(os.sched_getaffinity(0)))
+    cores = torch.get_num_threads()
+    dec = wl.decoder
+    Xs = sc.X[:n_tiles].cpu()
+    embed = sc.embed.cpu()
+    t0 = time.perf_counter()
+    t = O.query_embedding(embed, [sc.query_ids])
+    B = O.background_embeddings(embed, sc.bg_ids)
+    r64, V, s64 = O.score_scene(Xs, t, B)
+    r32 = O.to_f32(r64)
+    for i in range(n_tiles):
+        O.top_b(r32[i], budget)
+    t_tile = (time.perf_counter() - t0) / n_tiles
+    sel = O.top_b(r32[0], budget)
+    H0, cu, _ = O.pack(Xs, embed, [0], [sel], sc.sys_ids, sc.query_ids)
+    L = H0.shape[0]
+    layers = [W.make_layer(dec, l, device) for l in range(n_layers)]
+    gf = W.make_final_norm(dec, device).cpu()
+    t0 = time.perf_counter()
+    h = H0.to(torch.float64)
+    pos = torch.arange(L)
+    for l in range(n_layers):
+        h = O.decoder_layer(h, {k: v.cpu() for k, v in layers[l].items()}, dec, pos)
+    O.rmsnorm(h, gf, dec.eps)
+    t_tok_layer = (time.perf_counter() - t0) / (L * n_layers)
+    text = (f"oracle on {n_tiles} of {wl.scene.N} tiles (scoring + top-b) and one {L}-token sequence through "
+            f"{n_layers} of {dec.n_layers} layers (fp64), extrapolated linearly to the full query")
+    return t_tile, t_tok_layer, cores, text
+
+
+def oracle_tokens_per_s(wl, T, t_tile, t_tok_layer):
+    step_s = wl.scene.N * t_tile + T * t_tok_layer * wl.decoder.n_layers
+    return T / step_s, step_s
+
+
+def expected_T(wl, sc, device):
+    """Retained tokens of the query (from the oracle's own selection on the full scene)."""
+    from oracle import rift_oracle as O
+    if wl.policy.tau == 0.0 and wl.policy.C == (wl.scene.n_v,):
+        return wl.scene.N * (wl.scene.S + wl.scene.n_v + wl.scene.Q)
+    sel = O.select(sc.X.cpu(), sc.embed.cpu(), sc.query_ids, sc.bg_ids, wl.knn_m, wl.policy)
+    return sum(wl.scene.S + b + wl.scene.Q for b in sel.budgets)
+
+
+def run_reference(args, wl, ws, rank):
+    if rank != 0:
+        return
+    dev = torch.device("cuda", 0) if torch.cuda.is_available() else torch.device("cpu")
+    sc = W.make_scene(wl.scene, wl.decoder.vocab, dev)
+    T = expected_T(wl, sc, dev)
+    budget = min(wl.policy.C)
+    times, vals = [], []
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        t_tile, t_tok, cores, text = oracle_sample(wl, sc, 2, 2, budget, dev)
+        v, _ = oracle_tokens_per_s(wl, T, t_tile, t_tok)
+        if k >= args.warmup:
+            times.append(time.perf_counter() - t0)
+            vals.append(v)
+    value = statistics.median(vals)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "tiles": wl.scene.N, "retained_tokens_T": T},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": "per step: " + text},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------------ main arm
+
+def main():
+    args = parse()
+    ws, rank, local = dist_setup()
+    wl = W.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl, ws, rank)
+        return
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_29029_gb300 import DeviceModel, ScenePipeline, abi
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    s, dec = wl.scene, wl.decoder
+    sc = W.make_scene(s, dec.vocab, dev)
+    layers = [W.make_layer(dec, l, dev) for l in range(dec.n_layers)]
+    dm = DeviceModel(dec, layers, W.make_final_norm(dec, dev), dev)
+    del layers
+    pipe = ScenePipeline(s.N, s.n_v, s.d, s.x_dtype, s.M, s.S, s.Q, wl.knn_m, wl.policy, model=dm, device=dev)
+    i32 = dict(dtype=torch.int32, device=dev)
+    q = torch.tensor(sc.query_ids, **i32)
+    bg = torch.tensor(sc.bg_ids, **i32)
+    sy = torch.tensor(sc.sys_ids, **i32)
+    stream = torch.cuda.current_stream()
+
+    def step(X):
+        return pipe.run(X, sc.embed, q, bg, sy, q, stream=stream)
+
+    for _ in range(max(args.warmup, 1)):
+        n_kept, T = step(sc.X)
+    torch.cuda.synchronize()
+
+    # ---- timed region: inputs resident in HBM
+    barrier(ws)
+    torch.cuda.synchronize()
+    abi.profile_enable(True)
+    l0 = abi.launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            n_kept, T = step(sc.X)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    launches = abi.launch_count() - l0
+    abi.profile_enable(False)
+    prof = abi.profile_read()
+    barrier(ws)
+    ms = e0.elapsed_time(e1)
+    ms_max = reduce_max(ms, ws)
+    tokens_all = reduce_sum(float(T * args.steps), ws)
+    value = tokens_all / (ms_max / 1e3)
+
+    # ---- end to end: host buffers, H2D of the step's inputs and D2H of its result inside the region
+    X_host = sc.X.cpu().pin_memory()
+    embed_host = sc.embed.cpu().pin_memory()
+    ids_host = [torch.tensor(v, dtype=torch.int32).pin_memory() for v in (sc.query_ids, sc.bg_ids, sc.sys_ids)]
+    X_dev = torch.empty_like(sc.X)
+    emb_dev = torch.empty_like(sc.embed)
+    ids_dev = [torch.empty_like(h, device=dev) for h in ids_host]
+    out_host = torch.empty(T, s.d, dtype=torch.bfloat16).pin_memory()
+    barrier(ws)
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    Te = 0
+    for _ in range(args.e2e_steps):
+        X_dev.copy_(X_host, non_blocking=True)
+        emb_dev.copy_(embed_host, non_blocking=True)
+        for hdst, hsrc in zip(ids_dev, ids_host):
+            hdst.copy_(hsrc, non_blocking=True)
+        nk, Te = pipe.run(X_dev, emb_dev, ids_dev[0], ids_dev[1], ids_dev[2], ids_dev[0], stream=stream)
+        out_host[:Te].copy_(pipe.packed[:Te], non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = reduce_max(f0.elapsed_time(f1), ws)
+    e2e_val = reduce_sum(float(Te * args.e2e_steps), ws) / (e2e_ms / 1e3)
+    h2d = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
+    d2h = Te * s.d * 2 + 8
+
+    if rank != 0:
+        return
+    # ---- roofline of the dominant kernel (the prefill GEMM) from the live event timing
+    peaks = json.loads((ROOT / "MEASURED_PEAKS.json").read_text()) if (ROOT / "MEASURED_PEAKS.json").exists() else {}
+    peak = peaks.get("bf16_tflops_sustained", 1700.0)
+    gemm_ms, gemm_n = prof["gemm"]
+    gemm_flops = args.steps * T * dec.linear_flops_per_token
+    achieved = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
+    traffic = None
+    per_step = {k: round(v[0] / args.steps, 3) for k, v in prof.items()}
+    sel_ms = (prof["score"][0] + prof["select"][0] + prof["pack"][0]) / args.steps
+
+    cpu = None
+    if not args.no_cpu_baseline and ws == 1:
+        t_tile, t_tok, cores, text = oracle_sample(wl, sc, 8, 4, int(round((T / max(n_kept, 1)) - s.S - s.Q)), dev)
+        v, step_s = oracle_tokens_per_s(wl, T, t_tile, t_tok)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": text,
+               "extrapolated_step_s": step_s}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "tiles": s.N, "tokens_per_tile": s.n_v, "d": s.d,
+                   "decoder": f"{dec.n_layers}x{dec.d} LLaMA/Vicuna-7B shape, random init",
+                   "kept_tiles": n_kept, "retained_tokens_T": T,
+                   "mean_budget_frac": round((T / max(n_kept, 1) - s.S - s.Q) / s.n_v, 4),
+                   "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
+                   "l2": "inputs larger than L2 (X %.2f GB, weights %.1f GB)" % (
+                       sc.X.numel() * sc.X.element_size() / 1e9, dec.n_layers * dec.params_per_layer * 2 / 1e9)},
+        "scene_queries_per_s": 1e3 * args.steps / ms_max,
+        "select_latency_ms": sel_ms,
+        "kernels_ms_per_step": per_step,
+        "roofline": {"bound": "tensor", "kernel": "prefill GEMM", "achieved": achieved, "peak": peak,
+                     "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                     "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (of measured)",
+                     "launches": gemm_n},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,232 @@
+/*
+ * rift.h -- C ABI of the GB300 (sm_103a) hot path of Rift: query-conditioned tile
+ * pruning and elastic, per-tile token-budgeted prefill over a tiled scene.
+ *
+ * Calls, in the order the method runs them:
+ *   rift_query_prep              Section 2.3 Stage 1: the query embedding t and the
+ *                                background embeddings B_j that Eq. 1 compares against
+ *   rift_score_tiles             Eq. 1 on every vision token and every tile, then the
+ *                                kNN smoothing of Appendix B Step 2
+ *   rift_select_budgeted_tokens  per-scene min-max and the tau threshold (Section 2.3
+ *                                Stage 1, Appendix B Step 3), the budget argmax of Eq. 2
+ *                                (Section 2.3 Stage 2), and each kept tile's top-b tokens
+ *   rift_pack_ragged             one sequence per kept tile, [system | tokens | query],
+ *                                packed back to back with varlen offsets
+ *   rift_prefill_layers          the decoder prefill over the packed batch (Section 2.1)
+ *
+ * Conventions shared by every call
+ *   - Every array argument is a DEVICE pointer owned by the caller, unless marked
+ *     "host".  The library never allocates device memory: scratch comes from the
+ *     caller's workspace `ws` (size from the matching *_workspace_bytes query; pass
+ *     at least that many bytes, 256-byte aligned).
+ *   - Sizes are host ints.  Counts that only the device knows (n_kept, T) are written
+ *     to device ints and can be read after rift_sync_status.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; 0 = the legacy default stream)
+ *     and return RIFT_OK once the work is enqueued.  Argument errors that the host can
+ *     see are returned at once and nothing is launched.  Errors that only the device can
+ *     see (a non-finite score, a packed batch larger than its capacity, an id outside
+ *     the vocabulary, a bounded wait that ran out) set a per-process device flag; the
+ *     next rift_sync_status returns and clears it.
+ *   - Nothing throws across this boundary; no call keeps a pointer after it returns.
+ *   - Matrices are row-major.  bf16 is IEEE binary16-brain (1-8-7) stored in uint16.
+ *   - Every fp32 value that decides an integer (a neighbour, a kept tile, a budget, a
+ *     selected token) is computed in fp32 with the operation order documented below,
+ *     and ties go to the lower index.
+ */
+#ifndef RIFT_H
+#define RIFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RIFT_OK = 0,
+  RIFT_ERR_INVALID = 1,     /* bad argument: null pointer, size out of range, misalignment */
+  RIFT_ERR_CAPACITY = 2,    /* an output did not fit its capacity (e.g. T > max_T) */
+  RIFT_ERR_NONFINITE = 3,   /* a NaN or Inf score reached a decision */
+  RIFT_ERR_CUDA = 4,        /* a CUDA runtime call failed */
+  RIFT_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+  RIFT_ERR_UNSUPPORTED = 6, /* a valid request this build does not implement */
+  RIFT_ERR_BAD_ID = 7       /* a token or tile id outside its range */
+} rift_status;
+
+typedef enum { RIFT_F32 = 0, RIFT_BF16 = 1 } rift_dtype;
+
+typedef void* rift_stream_t; /* cudaStream_t */
+
+#define RIFT_MAX_BUDGETS 8
+#define RIFT_MAX_NV 1024      /* vision tokens per tile */
+#define RIFT_MAX_TILES 65536
+#define RIFT_MAX_KNN 16
+
+/* Stage-1 threshold and Stage-2 budget table (Section 2.3, Eq. 2).
+ *   tau        keep tile i iff u_i >= tau, 0 <= tau <= 1 (Appendix B: tau = 0.37)
+ *   n_c, C     candidate budgets, strictly ascending, each in [1, n_v]
+ *              (the paper: {72, 144, 288, 432, 576})
+ *   alpha_pos  profiled accuracy on tiles that contain the object, per c
+ *   alpha_neg  profiled accuracy on tiles that do not, per c
+ *   energy     profiled energy per c;  lambda  the accuracy-energy trade-off
+ * U_i(c) = ((p_i * alpha_pos[c]) + ((1 - p_i) * alpha_neg[c])) - (lambda * energy[c]),
+ * each operation a correctly rounded fp32 op; b_i = C[argmax_c U_i(c)], ties to the
+ * lower index (the cheaper budget). */
+typedef struct {
+  float tau;
+  int n_c;
+  int C[RIFT_MAX_BUDGETS];
+  float alpha_pos[RIFT_MAX_BUDGETS];
+  float alpha_neg[RIFT_MAX_BUDGETS];
+  float energy[RIFT_MAX_BUDGETS];
+  float lambda;
+} rift_policy;
+
+/* A LLaMA/Vicuna-shaped decoder (Section 2.1; LLaVA-1.5-7B: 32 layers, d 4096, 32 heads
+ * x 128, FFN 11008, eps 1e-6, rope_theta 1e4).  The per-layer fields are HOST arrays of
+ * n_layers DEVICE pointers to bf16 weights:
+ *   w_qkv      [3d, d]   rows 0..d-1 = W_q, d..2d-1 = W_k, 2d..3d-1 = W_v (out x in)
+ *   w_o        [d, d]
+ *   w_gate_up  [2 ffn, d] W_gate and W_up interleaved in groups of 16 rows:
+ *              rows 32g..32g+15 = W_gate rows 16g..16g+15, rows 32g+16..32g+31 = W_up
+ *              rows 16g..16g+15 (ffn must be a multiple of 16)
+ *   w_down     [d, ffn]
+ *   g_attn, g_ffn [d]    RMSNorm gains;  g_final [d] (one device pointer)
+ * Requirements: d % 64 == 0, head_dim in {64, 128}, n_heads * head_dim == d. */
+typedef struct {
+  int n_layers, d, n_heads, head_dim, ffn;
+  float eps, rope_theta;
+  const void* const* w_qkv;
+  const void* const* w_o;
+  const void* const* w_gate_up;
+  const void* const* w_down;
+  const void* const* g_attn;
+  const void* const* g_ffn;
+  const void* g_final;
+} rift_model;
+
+/* Version of this ABI (bumped on any signature change). */
+int rift_abi_version(void);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* rift_status_string(rift_status s);
+
+/* Waits for all work on `stream`, then returns and clears the device error flags set
+ * by earlier calls (RIFT_OK if none).  If several flags are set, the most specific one
+ * is returned (BAD_ID, NONFINITE, CAPACITY, TIMEOUT, in that order). */
+rift_status rift_sync_status(rift_stream_t stream);
+
+/* ---- a1. Query preparation (Section 2.3 Stage 1; Listing 1's E(phrase), E(terms)) ----
+ * The paper embeds the query's object phrase and M background terms with RemoteCLIP.
+ * Stand-in here: the decoder's own token embedding.
+ *   embed       bf16 [vocab, d]
+ *   phrase_ids  int32 [n_templates * n_phrase]: template k's ids at k*n_phrase
+ *   bg_ids      int32 [M] (M may be 0; bg_ids may then be NULL)
+ *   t           out fp32 [d]:   t = l2norm(mean_k l2norm(mean_q embed[phrase_ids[k][q]]))
+ *   B           out fp32 [M,d]: B_j = l2norm(embed[bg_ids[j]]) (NULL allowed if M == 0)
+ * Ids outside [0, vocab) set RIFT_ERR_BAD_ID. */
+rift_status rift_query_prep(const void* embed, int vocab, int d,
+                            const int* phrase_ids, int n_templates, int n_phrase,
+                            const int* bg_ids, int M, float* t, float* B,
+                            rift_stream_t stream);
+
+/* ---- a2-a4. Relevance scores (Eq. 1) and kNN smoothing (Appendix B Step 2) ----
+ *   X             [N, n_v, d] vision tokens, fp32 or bf16 (xdt)
+ *   t, B          from rift_query_prep (B may be NULL if M == 0)
+ *   knn_m         neighbours per tile; the call uses m = min(knn_m, N - 1), 0 <= knn_m <= 16
+ *   token_scores  out fp32 [N, n_v]: r_ik = x_ik . w / ||x_ik||, w = t - (1/M) sum_j B_j
+ *                 (Eq. 1 applied to each token)
+ *   tile_s_raw    out fp32 [N]: s_i = V_i . w, V_i = P_i / ||P_i||, P_i = sum_k x_ik (Eq. 1)
+ *   tile_s        out fp32 [N]: s~_i = (sum over {i} + NN(i) in ascending index of s_j)
+ *                 / (m + 1), NN(i) = the m tiles j != i of largest fp32 V_i . V_j, ties to
+ *                 the lower j
+ *   nbr           out int32 [N, m] (nullable): NN(i) in rank order
+ * Limits: 1 <= N <= RIFT_MAX_TILES, 1 <= n_v <= RIFT_MAX_NV, 64 <= d <= 8192, d % 64 == 0,
+ * 0 <= M <= 64; X 16-byte aligned. */
+size_t rift_score_workspace_bytes(int N, int n_v, int d, int M);
+rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int d,
+                             const float* t, const float* B, int M, int knn_m,
+                             float* token_scores, float* tile_s_raw, float* tile_s, int* nbr,
+                             void* ws, size_t ws_bytes, rift_stream_t stream);
+
+/* ---- a5-a7. Prune, budget and select (Section 2.3; Appendix B Steps 3-4) ----
+ *   token_scores, tile_s  from rift_score_tiles (tile_s = the smoothed scores)
+ *   p          fp32 [N] (nullable): p_i, the probability that tile i holds the object;
+ *              NULL uses p_i = u_i (stand-in for the paper's learned predictor)
+ *   policy     host pointer, see rift_policy
+ *   u          out fp32 [N]: (s~_i - min) / (max - min), or 1 for all if max == min
+ *   kept       out int32 [N]: the kept tiles (u_i >= tau) in ascending order, first n_kept
+ *   n_kept     out int32 [1]
+ *   budgets    out int32 [N]: b_j for kept slot j (first n_kept entries)
+ *   sel        out int32 [N * n_v]: kept slot j's selected token indices at sel_off[j],
+ *              the b_j largest token scores (ties to the lower index), ascending
+ *   sel_off    out int32 [N + 1]: exclusive prefix sum of budgets; entries j > n_kept
+ *              are set to the total
+ * A NaN or Inf among the scores that are read sets RIFT_ERR_NONFINITE. */
+size_t rift_select_workspace_bytes(int N, int n_v);
+rift_status rift_select_budgeted_tokens(const float* token_scores, const float* tile_s,
+                                        int N, int n_v, const float* p,
+                                        const rift_policy* policy,
+                                        float* u, int* kept, int* n_kept, int* budgets,
+                                        int* sel, int* sel_off,
+                                        void* ws, size_t ws_bytes, rift_stream_t stream);
+
+/* ---- a8. Ragged packing (the per-tile VLM prompt of Appendix B Step 5) ----
+ *   X, xdt, N, n_v, d     as for rift_score_tiles (fp32 tokens are rounded to bf16)
+ *   kept, n_kept, sel, sel_off   from rift_select_budgeted_tokens
+ *   sys_ids    int32 [S] system-prompt ids;  query_ids int32 [Q] query ids
+ *   embed      bf16 [vocab, d]
+ *   packed     out bf16 [max_T, d]: sequence j = [embed[sys_ids] | X[kept[j], sel_j] |
+ *              embed[query_ids]], sequences back to back in kept order
+ *   cu_seqlens out int32 [N + 1]: cu_seqlens[j] = j (S + Q) + sel_off[j]; entries
+ *              j > n_kept are set to T
+ *   positions  out int32 [max_T]: position of each packed row in its sequence (0..L_j-1)
+ *   T          out int32 [1]: total packed rows
+ * T > max_T sets RIFT_ERR_CAPACITY (rows beyond max_T are not written). */
+rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int d,
+                             const int* kept, const int* n_kept,
+                             const int* sel, const int* sel_off,
+                             const int* sys_ids, int S, const int* query_ids, int Q,
+                             const void* embed, int vocab,
+                             void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
+                             rift_stream_t stream);
+
+/* ---- a9. Decoder prefill (Section 2.1) ----
+ *   hidden     bf16 [T, d]: in, the packed batch; out, the final hidden states (after the
+ *              final RMSNorm).  The residual stream is kept in fp32 in the workspace.
+ *   T          packed rows (host int, e.g. read back after rift_sync_status)
+ *   cu_seqlens int32 [n_seq + 1], positions int32 [T] from rift_pack_ragged
+ *   max_len    an upper bound on every sequence length (host int)
+ * Each layer: h += W_o Attn(RoPE(q), RoPE(k), v) with x = RMSNorm(h) g_attn, causal within
+ * each sequence only; h += W_down(SiLU(W_gate x) * (W_up x)) with x = RMSNorm(h) g_ffn.
+ * GEMMs take bf16 operands and accumulate in fp32. */
+size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len);
+rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
+                                const int* cu_seqlens, int n_seq, int max_len,
+                                const int* positions,
+                                void* ws, size_t ws_bytes, rift_stream_t stream);
+
+/* ---- Instrumentation for benchmarks (does not change any result) ----
+ * Kernel classes timed by the profiler: */
+#define RIFT_PROF_GEMM 0      /* the prefill GEMMs (QKV, O, gate/up, down) */
+#define RIFT_PROF_ATTN 1      /* varlen causal attention (with its q-block schedule) */
+#define RIFT_PROF_NORM 2      /* RMSNorm kernels */
+#define RIFT_PROF_ROPE 3      /* RoPE table and rotation */
+#define RIFT_PROF_SCORE 4     /* query prep, token/tile scores, kNN */
+#define RIFT_PROF_SELECT 5    /* prune, budgets, top-b */
+#define RIFT_PROF_PACK 6      /* ragged packing */
+#define RIFT_PROF_CLASSES 7
+/* rift_profile_enable(1) starts recording a pair of CUDA events on the launch stream around
+ * every kernel launch of the classes above (0 stops).  rift_profile_read waits for the recorded
+ * events, writes per-class totals (ms[c] in milliseconds, launches[c]) for n_classes classes and
+ * clears the record.  Returns RIFT_ERR_CUDA if an event query fails. */
+void rift_profile_enable(int on);
+rift_status rift_profile_read(double* ms, long long* launches, int n_classes);
+/* Number of kernels this library has launched since it was loaded (always counted). */
+long long rift_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RIFT_H */

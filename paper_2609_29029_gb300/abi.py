@@ -1,0 +1,187 @@
+"""ctypes binding of include/rift.h: the same call names, argument marshalling only.
+
+Tensors are passed as raw device pointers (``tensor.data_ptr()``) and streams as raw
+``cudaStream_t`` handles.  Every computation happens inside libriftgb.so; if the library is
+missing this module raises at import time, there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from pathlib import Path
+
+import torch
+
+LIB_PATH = Path(__file__).resolve().parent / "libriftgb.so"
+
+RIFT_OK, RIFT_ERR_INVALID, RIFT_ERR_CAPACITY, RIFT_ERR_NONFINITE, RIFT_ERR_CUDA, RIFT_ERR_TIMEOUT, \
+    RIFT_ERR_UNSUPPORTED, RIFT_ERR_BAD_ID = range(8)
+RIFT_F32, RIFT_BF16 = 0, 1
+MAX_BUDGETS = 8
+
+
+class RiftError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+class Policy(C.Structure):
+    _fields_ = [("tau", C.c_float), ("n_c", C.c_int), ("C", C.c_int * MAX_BUDGETS),
+                ("alpha_pos", C.c_float * MAX_BUDGETS), ("alpha_neg", C.c_float * MAX_BUDGETS),
+                ("energy", C.c_float * MAX_BUDGETS), ("lam", C.c_float)]
+
+
+class Model(C.Structure):
+    _fields_ = [("n_layers", C.c_int), ("d", C.c_int), ("n_heads", C.c_int), ("head_dim", C.c_int),
+                ("ffn", C.c_int), ("eps", C.c_float), ("rope_theta", C.c_float),
+                ("w_qkv", C.POINTER(C.c_void_p)), ("w_o", C.POINTER(C.c_void_p)),
+                ("w_gate_up", C.POINTER(C.c_void_p)), ("w_down", C.POINTER(C.c_void_p)),
+                ("g_attn", C.POINTER(C.c_void_p)), ("g_ffn", C.POINTER(C.c_void_p)),
+                ("g_final", C.c_void_p)]
+
+
+_vp, _i, _f, _sz = C.c_void_p, C.c_int, C.c_float, C.c_size_t
+
+SIGNATURES = {
+    "rift_abi_version": (_i, []),
+    "rift_status_string": (C.c_char_p, [_i]),
+    "rift_sync_status": (_i, [_vp]),
+    "rift_query_prep": (_i, [_vp, _i, _i, _vp, _i, _i, _vp, _i, _vp, _vp, _vp]),
+    "rift_score_workspace_bytes": (_sz, [_i, _i, _i, _i]),
+    "rift_score_tiles": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "rift_select_workspace_bytes": (_sz, [_i, _i]),
+    "rift_select_budgeted_tokens": (_i, [_vp, _vp, _i, _i, _vp, C.POINTER(Policy), _vp, _vp, _vp, _vp, _vp,
+                                         _vp, _vp, _sz, _vp]),
+    "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _i,
+                              _vp, _vp, _vp, _vp]),
+    "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
+    "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _sz, _vp]),
+    "rift_profile_enable": (None, [_i]),
+    "rift_profile_read": (_i, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), _i]),
+    "rift_launch_count": (C.c_longlong, []),
+}
+
+PROF_CLASSES = ("gemm", "attention", "rmsnorm", "rope", "score", "select", "pack")
+
+
+def _load():
+    if not LIB_PATH.exists():
+        raise ImportError(f"{LIB_PATH} is missing: build it first (python -m paper_2609_29029_gb300.build); "
+                          "the Rift hot path has no CPU fallback")
+    lib = C.CDLL(str(LIB_PATH))
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+lib = _load()
+
+
+def status_string(s: int) -> str:
+    return lib.rift_status_string(int(s)).decode()
+
+
+def _check(status: int, where: str):
+    if status != RIFT_OK:
+        raise RiftError(status, where)
+
+
+def ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def stream_handle(stream=None) -> int:
+    if isinstance(stream, int):
+        return stream
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def make_policy(policy) -> Policy:
+    p = Policy()
+    p.tau = policy.tau
+    p.n_c = len(policy.C)
+    for k, c in enumerate(policy.C):
+        p.C[k] = c
+        p.alpha_pos[k] = policy.alpha_pos[k]
+        p.alpha_neg[k] = policy.alpha_neg[k]
+        p.energy[k] = policy.energy[k]
+    p.lam = policy.lam
+    return p
+
+
+def abi_version() -> int:
+    return lib.rift_abi_version()
+
+
+def sync_status(stream=None):
+    _check(lib.rift_sync_status(stream_handle(stream)), "rift_sync_status")
+
+
+def query_prep(embed, vocab, d, phrase_ids, n_templates, n_phrase, bg_ids, M, t, B, stream=None):
+    _check(lib.rift_query_prep(ptr(embed), vocab, d, ptr(phrase_ids), n_templates, n_phrase, ptr(bg_ids), M,
+                               ptr(t), ptr(B), stream_handle(stream)), "rift_query_prep")
+
+
+def score_workspace_bytes(N, n_v, d, M) -> int:
+    return lib.rift_score_workspace_bytes(N, n_v, d, M)
+
+
+def score_tiles(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_raw, tile_s, nbr, ws, ws_bytes,
+                stream=None):
+    _check(lib.rift_score_tiles(ptr(X), xdt, N, n_v, d, ptr(t), ptr(B), M, knn_m, ptr(token_scores),
+                                ptr(tile_s_raw), ptr(tile_s), ptr(nbr), ptr(ws), ws_bytes, stream_handle(stream)),
+           "rift_score_tiles")
+
+
+def select_workspace_bytes(N, n_v) -> int:
+    return lib.rift_select_workspace_bytes(N, n_v)
+
+
+def select_budgeted_tokens(token_scores, tile_s, N, n_v, p, policy: Policy, u, kept, n_kept, budgets, sel,
+                           sel_off, ws, ws_bytes, stream=None):
+    _check(lib.rift_select_budgeted_tokens(ptr(token_scores), ptr(tile_s), N, n_v, ptr(p), C.byref(policy),
+                                           ptr(u), ptr(kept), ptr(n_kept), ptr(budgets), ptr(sel), ptr(sel_off),
+                                           ptr(ws), ws_bytes, stream_handle(stream)),
+           "rift_select_budgeted_tokens")
+
+
+def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, packed,
+                max_T, cu_seqlens, positions, T, stream=None):
+    _check(lib.rift_pack_ragged(ptr(X), xdt, N, n_v, d, ptr(kept), ptr(n_kept), ptr(sel), ptr(sel_off),
+                                ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(packed), max_T,
+                                ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),
+           "rift_pack_ragged")
+
+
+def prefill_workspace_bytes(model: Model, max_T, max_seqs, max_len) -> int:
+    return lib.rift_prefill_workspace_bytes(C.byref(model), max_T, max_seqs, max_len)
+
+
+def prefill_layers(model: Model, hidden, T, cu_seqlens, n_seq, max_len, positions, ws, ws_bytes, stream=None):
+    _check(lib.rift_prefill_layers(C.byref(model), ptr(hidden), T, ptr(cu_seqlens), n_seq, max_len,
+                                   ptr(positions), ptr(ws), ws_bytes, stream_handle(stream)),
+           "rift_prefill_layers")
+
+
+def profile_enable(on: bool):
+    lib.rift_profile_enable(1 if on else 0)
+
+
+def profile_read() -> dict:
+    """Per kernel class: (total ms, launches) recorded since profiling was enabled."""
+    n = len(PROF_CLASSES)
+    ms = (C.c_double * n)()
+    cnt = (C.c_longlong * n)()
+    _check(lib.rift_profile_read(ms, cnt, n), "rift_profile_read")
+    return {k: (ms[i], cnt[i]) for i, k in enumerate(PROF_CLASSES)}
+
+
+def launch_count() -> int:
+    return lib.rift_launch_count()

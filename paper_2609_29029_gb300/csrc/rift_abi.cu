@@ -1,0 +1,257 @@
+// The C ABI of include/rift.h: argument validation, workspace carving and launches on the
+// caller's stream.  Nothing here allocates device memory.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <mutex>
+#include <vector>
+
+#include "rift_internal.h"
+
+using namespace rift;
+
+namespace {
+
+constexpr size_t WS_ALIGN = 256;
+
+bool ws_ok(const void* ws, size_t have, size_t need) {
+  if (need == 0) return true;
+  return ws != nullptr && have >= need && (reinterpret_cast<uintptr_t>(ws) % WS_ALIGN) == 0;
+}
+
+bool dims_ok(int N, int n_v, int d) {
+  return N >= 1 && N <= RIFT_MAX_TILES && n_v >= 1 && n_v <= RIFT_MAX_NV && d >= 64 && d <= 8192 &&
+         d % 64 == 0;
+}
+
+struct ProfRec {
+  int cls, n;
+  cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<cudaEvent_t> g_pool;
+std::vector<ProfRec> g_recs;
+cudaEvent_t g_open[RIFT_PROF_CLASSES] = {};
+std::atomic<long long> g_launches{0};
+
+cudaEvent_t pool_get() {
+  if (!g_pool.empty()) {
+    cudaEvent_t e = g_pool.back();
+    g_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+}  // namespace
+
+namespace rift {
+
+void prof_begin(int cls, cudaStream_t st) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (!g_prof_on) return;
+  cudaEvent_t e = pool_get();
+  if (e && cudaEventRecord(e, st) == cudaSuccess) g_open[cls] = e;
+}
+
+void prof_end(int cls, cudaStream_t st, int n) {
+  g_launches += n;
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (!g_prof_on || !g_open[cls]) return;
+  cudaEvent_t e = pool_get();
+  if (e && cudaEventRecord(e, st) == cudaSuccess) g_recs.push_back({cls, n, g_open[cls], e});
+  g_open[cls] = nullptr;
+}
+
+}  // namespace rift
+
+extern "C" {
+
+void rift_profile_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof_on = on != 0;
+}
+
+rift_status rift_profile_read(double* ms, long long* launches, int n_classes) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  rift_status st = RIFT_OK;
+  for (int c = 0; c < n_classes; ++c) {
+    if (ms) ms[c] = 0.0;
+    if (launches) launches[c] = 0;
+  }
+  for (const ProfRec& r : g_recs) {
+    float t = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) st = RIFT_ERR_CUDA;
+    if (r.cls < n_classes) {
+      if (ms) ms[r.cls] += t;
+      if (launches) launches[r.cls] += r.n;
+    }
+    g_pool.push_back(r.a);
+    g_pool.push_back(r.b);
+  }
+  g_recs.clear();
+  return st;
+}
+
+long long rift_launch_count(void) { return g_launches.load(); }
+
+int rift_abi_version(void) { return 1; }
+
+const char* rift_status_string(rift_status s) {
+  switch (s) {
+    case RIFT_OK: return "ok";
+    case RIFT_ERR_INVALID: return "invalid argument";
+    case RIFT_ERR_CAPACITY: return "output capacity exceeded";
+    case RIFT_ERR_NONFINITE: return "non-finite score";
+    case RIFT_ERR_CUDA: return "CUDA runtime error";
+    case RIFT_ERR_TIMEOUT: return "device wait timed out";
+    case RIFT_ERR_UNSUPPORTED: return "unsupported";
+    case RIFT_ERR_BAD_ID: return "id out of range";
+  }
+  return "unknown status";
+}
+
+rift_status rift_sync_status(rift_stream_t stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return RIFT_ERR_CUDA;
+  unsigned int f = read_clear_err_score() | read_clear_err_select() | read_clear_err_pack() |
+                   read_clear_err_prefill();
+  if (cudaGetLastError() != cudaSuccess) return RIFT_ERR_CUDA;
+  if (f & RIFT_EBIT_BADID) return RIFT_ERR_BAD_ID;
+  if (f & RIFT_EBIT_NONFINITE) return RIFT_ERR_NONFINITE;
+  if (f & RIFT_EBIT_CAPACITY) return RIFT_ERR_CAPACITY;
+  if (f & RIFT_EBIT_TIMEOUT) return RIFT_ERR_TIMEOUT;
+  return RIFT_OK;
+}
+
+rift_status rift_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_templates,
+                            int n_phrase, const int* bg_ids, int M, float* t, float* B,
+                            rift_stream_t stream) {
+  if (!embed || !phrase_ids || !t || vocab < 1 || d < 64 || d > 8192 || d % 64 != 0 || n_templates < 1 ||
+      n_phrase < 1 || M < 0 || M > 64 || (M > 0 && (!bg_ids || !B)))
+    return RIFT_ERR_INVALID;
+  prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
+  launch_query_prep(embed, vocab, d, phrase_ids, n_templates, n_phrase, bg_ids, M, t, B,
+                    static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), 1);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_score_workspace_bytes(int N, int n_v, int d, int M) {
+  if (!dims_ok(N, n_v, d)) return 0;
+  return score_layout(N, n_v, d, M).total;
+}
+
+rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t,
+                             const float* B, int M, int knn_m, float* token_scores, float* tile_s_raw,
+                             float* tile_s, int* nbr, void* ws, size_t ws_bytes, rift_stream_t stream) {
+  if (!dims_ok(N, n_v, d) || !X || !t || !token_scores || !tile_s_raw || !tile_s) return RIFT_ERR_INVALID;
+  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
+  if (xdt == RIFT_F32 && d > 4096) return RIFT_ERR_UNSUPPORTED;
+  if (M < 0 || M > 64 || (M > 0 && !B) || knn_m < 0 || knn_m > RIFT_MAX_KNN) return RIFT_ERR_INVALID;
+  if (!aligned16(X)) return RIFT_ERR_INVALID;
+  const size_t need = rift_score_workspace_bytes(N, n_v, d, M);
+  if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
+  const int m = std::min(knn_m, N - 1);
+  prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
+  const int nk = launch_score(X, xdt, N, n_v, d, t, B, M, m, token_scores, tile_s_raw, tile_s, nbr,
+                              static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_select_workspace_bytes(int N, int n_v) {
+  (void)N;
+  (void)n_v;
+  return 0;
+}
+
+rift_status rift_select_budgeted_tokens(const float* token_scores, const float* tile_s, int N, int n_v,
+                                        const float* p, const rift_policy* policy, float* u, int* kept,
+                                        int* n_kept, int* budgets, int* sel, int* sel_off, void* ws,
+                                        size_t ws_bytes, rift_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (!token_scores || !tile_s || !policy || !u || !kept || !n_kept || !budgets || !sel || !sel_off)
+    return RIFT_ERR_INVALID;
+  if (N < 1 || N > RIFT_MAX_TILES || n_v < 1 || n_v > RIFT_MAX_NV) return RIFT_ERR_INVALID;
+  const rift_policy& pol = *policy;
+  if (!(pol.tau >= 0.f && pol.tau <= 1.f)) return RIFT_ERR_INVALID;
+  if (pol.n_c < 1 || pol.n_c > RIFT_MAX_BUDGETS) return RIFT_ERR_INVALID;
+  for (int c = 0; c < pol.n_c; ++c) {
+    if (pol.C[c] < 1 || pol.C[c] > n_v) return RIFT_ERR_INVALID;
+    if (c > 0 && pol.C[c] <= pol.C[c - 1]) return RIFT_ERR_INVALID;
+    if (!std::isfinite(pol.alpha_pos[c]) || !std::isfinite(pol.alpha_neg[c]) || !std::isfinite(pol.energy[c]))
+      return RIFT_ERR_INVALID;
+  }
+  if (!std::isfinite(pol.lambda)) return RIFT_ERR_INVALID;
+  prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
+  launch_select(token_scores, tile_s, N, n_v, p, pol, u, kept, n_kept, budgets, sel, sel_off,
+                static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream), 2);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
+                             const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
+                             const int* query_ids, int Q, const void* embed, int vocab, void* packed, int max_T,
+                             int* cu_seqlens, int* positions, int* T, rift_stream_t stream) {
+  if (!dims_ok(N, n_v, d) || !X || !kept || !n_kept || !sel || !sel_off || !embed || !packed || !cu_seqlens ||
+      !positions || !T)
+    return RIFT_ERR_INVALID;
+  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
+  if (S < 0 || Q < 0 || (S > 0 && !sys_ids) || (Q > 0 && !query_ids) || vocab < 1 || max_T < 0)
+    return RIFT_ERR_INVALID;
+  if (!aligned16(X) || !aligned16(embed) || !aligned16(packed)) return RIFT_ERR_INVALID;
+  prof_begin(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream));
+  launch_pack(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, packed,
+              max_T, cu_seqlens, positions, T, static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream), 2);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+static bool model_ok(const rift_model* m) {
+  if (!m) return false;
+  if (m->n_layers < 1 || m->d < 64 || m->d > 8192 || m->d % 64 != 0) return false;
+  if (m->head_dim != 64 && m->head_dim != 128) return false;
+  if (m->n_heads < 1 || m->n_heads * m->head_dim != m->d) return false;
+  if (m->ffn < 16 || m->ffn % 16 != 0) return false;
+  if (!(m->eps > 0.f) || !(m->rope_theta > 0.f)) return false;
+  if (!m->w_qkv || !m->w_o || !m->w_gate_up || !m->w_down || !m->g_attn || !m->g_ffn || !m->g_final)
+    return false;
+  for (int l = 0; l < m->n_layers; ++l) {
+    const void* p[6] = {m->w_qkv[l], m->w_o[l], m->w_gate_up[l], m->w_down[l], m->g_attn[l], m->g_ffn[l]};
+    for (const void* q : p)
+      if (!q || !aligned16(q)) return false;
+  }
+  return aligned16(m->g_final);
+}
+
+size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len) {
+  if (!model_ok(m) || max_T < 0 || max_seqs < 0 || max_len < 1) return 0;
+  return prefill_layout(*m, max_T, max_seqs, max_len).total;
+}
+
+rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const int* cu_seqlens, int n_seq,
+                                int max_len, const int* positions, void* ws, size_t ws_bytes,
+                                rift_stream_t stream) {
+  if (!model_ok(m) || !hidden || !cu_seqlens || !positions || T < 0 || n_seq < 0 || max_len < 1)
+    return RIFT_ERR_INVALID;
+  if (T > 0 && n_seq < 1) return RIFT_ERR_INVALID;
+  if (!aligned16(hidden)) return RIFT_ERR_INVALID;
+  const size_t need = prefill_layout(*m, T, n_seq, max_len).total;
+  if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
+  if (launch_prefill(*m, hidden, T, cu_seqlens, n_seq, max_len, positions, static_cast<char*>(ws),
+                     static_cast<cudaStream_t>(stream)))
+    return RIFT_ERR_INVALID;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,63 @@
+// Internal launcher declarations shared by the translation units of the Rift library.
+#pragma once
+
+#include "rift_common.cuh"
+
+namespace rift {
+
+// Benchmark instrumentation: events around launches of a class (when enabled) and a launch
+// counter.  prof_begin/prof_end bracket the launches; n is the number of kernels inside.
+void prof_begin(int cls, cudaStream_t st);
+void prof_end(int cls, cudaStream_t st, int n);
+
+// Per-translation-unit device error flags (read and cleared by rift_sync_status).
+unsigned int read_clear_err_score();
+unsigned int read_clear_err_select();
+unsigned int read_clear_err_pack();
+unsigned int read_clear_err_prefill();
+
+// ---- score.cu ----
+struct ScoreLayout {
+  int chunk_tokens, n_chunks, n_jblk;
+  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, total;
+};
+ScoreLayout score_layout(int N, int n_v, int d, int M);
+void launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
+                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st);
+int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                 int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
+                 cudaStream_t st);
+
+// ---- select.cu ----
+void launch_select(const float* token_scores, const float* tile_s, int N, int n_v, const float* p,
+                   const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
+                   int* sel_off, cudaStream_t st);
+
+// ---- pack.cu ----
+void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
+                 const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
+                 const int* query_ids, int Q, const void* embed, int vocab, void* packed, int max_T,
+                 int* cu_seqlens, int* positions, int* T, cudaStream_t st);
+
+// ---- prefill (prefill.cu, gemm.cu, attention.cu) ----
+struct PrefillLayout {
+  size_t h32_off, xn_off, qkv_off, attn_off, act_off, rope_off, sched_off, total;
+  int max_qblocks;
+};
+PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len);
+int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
+                   int max_len, const int* positions, char* ws, cudaStream_t st);
+
+// GEMM: C[M, N] = A[M, K] . B[N, K]^T (bf16 operands, fp32 accumulation) + epilogue.
+enum GemmEpilogue {
+  EPI_STORE_BF16 = 0,  // C bf16 [M, N]
+  EPI_RESID_F32 = 1,   // R fp32 [M, N] += acc
+  EPI_SWIGLU = 2       // N = 2F interleaved in 16-column groups; C bf16 [M, F] = silu(g) * u
+};
+int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
+                cudaStream_t st);
+
+void launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
+                      int head_dim, const int2* sched, int n_sched_max, void* out, cudaStream_t st);
+
+}  // namespace rift

@@ -1,0 +1,162 @@
+"""Device buffers and the call sequence of one scene query through the C ABI.
+
+This module owns memory (torch tensors) and issues the five ABI calls in order; every
+computation is a kernel of libriftgb.so.  One host read-back per query (n_kept and T, after
+packing) sizes the prefill launch.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass
+
+import torch
+
+from . import abi
+
+
+def interleave_gate_up(wg: torch.Tensor, wu: torch.Tensor) -> torch.Tensor:
+    """[2F, d] with W_gate and W_up interleaved in 16-row groups (the layout rift_model wants)."""
+    F, d = wg.shape
+    assert F % 16 == 0 and wu.shape == wg.shape
+    return torch.stack([wg.view(F // 16, 16, d), wu.view(F // 16, 16, d)], dim=1).reshape(2 * F, d).contiguous()
+
+
+class DeviceModel:
+    """Decoder weights in the library's layout plus the rift_model struct that points at them."""
+
+    def __init__(self, dec, layers: list, g_final: torch.Tensor, device="cuda"):
+        self.dec = dec
+        self.layers = []
+        for W in layers:
+            self.layers.append({
+                "qkv": torch.cat([W["wq"], W["wk"], W["wv"]], 0).to(device, torch.bfloat16).contiguous(),
+                "o": W["wo"].to(device, torch.bfloat16).contiguous(),
+                "gate_up": interleave_gate_up(W["wg"].to(device), W["wu"].to(device)).to(torch.bfloat16),
+                "down": W["wd"].to(device, torch.bfloat16).contiguous(),
+                "g_attn": W["g_attn"].to(device, torch.bfloat16).contiguous(),
+                "g_ffn": W["g_ffn"].to(device, torch.bfloat16).contiguous(),
+            })
+        self.g_final = g_final.to(device, torch.bfloat16).contiguous()
+        n = len(self.layers)
+        arr = C.c_void_p * n
+        self._ptrs = {k: arr(*[L[k].data_ptr() for L in self.layers])
+                      for k in ("qkv", "o", "gate_up", "down", "g_attn", "g_ffn")}
+        m = abi.Model()
+        m.n_layers, m.d, m.n_heads, m.head_dim, m.ffn = n, dec.d, dec.n_heads, dec.head_dim, dec.ffn
+        m.eps, m.rope_theta = dec.eps, dec.rope_theta
+        m.w_qkv, m.w_o = self._ptrs["qkv"], self._ptrs["o"]
+        m.w_gate_up, m.w_down = self._ptrs["gate_up"], self._ptrs["down"]
+        m.g_attn, m.g_ffn = self._ptrs["g_attn"], self._ptrs["g_ffn"]
+        m.g_final = self.g_final.data_ptr()
+        self.struct = m
+
+
+@dataclass
+class QueryResult:
+    n_kept: int
+    T: int
+    t: torch.Tensor
+    token_scores: torch.Tensor
+    tile_s_raw: torch.Tensor
+    tile_s: torch.Tensor
+    nbr: torch.Tensor
+    u: torch.Tensor
+    kept: torch.Tensor
+    budgets: torch.Tensor
+    sel: torch.Tensor
+    sel_off: torch.Tensor
+    cu_seqlens: torch.Tensor
+    positions: torch.Tensor
+    hidden: torch.Tensor      # [T, d] bf16: packed input, then (after prefill) final hidden states
+
+
+class ScenePipeline:
+    """Buffers for scenes of N tiles x n_v tokens x d, and the run of one query."""
+
+    def __init__(self, N, n_v, d, xdt, M, S, Q, knn_m, policy, model: DeviceModel | None = None,
+                 max_T: int | None = None, device="cuda"):
+        self.N, self.n_v, self.d, self.M, self.S, self.Q = N, n_v, d, M, S, Q
+        self.xdt = abi.RIFT_BF16 if xdt in ("bf16", torch.bfloat16) else abi.RIFT_F32
+        self.knn_m = knn_m
+        self.m = min(knn_m, N - 1)
+        self.policy = abi.make_policy(policy)
+        self.model = model
+        self.max_T = max_T if max_T is not None else N * (S + n_v + Q)
+        self.max_len = S + n_v + Q
+        dev = torch.device(device)
+        f32, i32 = dict(dtype=torch.float32, device=dev), dict(dtype=torch.int32, device=dev)
+        self.t = torch.empty(d, **f32)
+        self.B = torch.empty(max(M, 1), d, **f32)
+        self.token_scores = torch.empty(N, n_v, **f32)
+        self.tile_s_raw = torch.empty(N, **f32)
+        self.tile_s = torch.empty(N, **f32)
+        self.nbr = torch.empty(max(N * self.m, 1), **i32)
+        self.u = torch.empty(N, **f32)
+        self.kept = torch.empty(N, **i32)
+        self.n_kept = torch.zeros(1, **i32)
+        self.budgets = torch.empty(N, **i32)
+        self.sel = torch.empty(N * n_v, **i32)
+        self.sel_off = torch.empty(N + 1, **i32)
+        self.packed = torch.empty(self.max_T, d, dtype=torch.bfloat16, device=dev)
+        self.cu = torch.empty(N + 1, **i32)
+        self.positions = torch.empty(max(self.max_T, 1), **i32)
+        self.T = torch.zeros(1, **i32)
+        self.counts_host = torch.zeros(2, dtype=torch.int32, pin_memory=True)
+        self.ws_score_bytes = abi.score_workspace_bytes(N, n_v, d, M)
+        self.ws_score = torch.empty(self.ws_score_bytes, dtype=torch.uint8, device=dev)
+        self.ws_prefill = None
+        self.ws_prefill_bytes = 0
+        self.device = dev
+
+    def _prefill_ws(self, T, n_seq):
+        need = abi.prefill_workspace_bytes(self.model.struct, T, n_seq, self.max_len)
+        if need > self.ws_prefill_bytes:
+            self.ws_prefill = torch.empty(need, dtype=torch.uint8, device=self.device)
+            self.ws_prefill_bytes = need
+        return self.ws_prefill, need
+
+    def select(self, X, embed, phrase_ids, bg_ids, p=None, n_templates=1, stream=None):
+        """a1-a7: query prep, scoring, smoothing, pruning, budgets and token selection."""
+        vocab = embed.shape[0]
+        n_phrase = phrase_ids.numel() // n_templates
+        abi.query_prep(embed, vocab, self.d, phrase_ids, n_templates, n_phrase, bg_ids if self.M else None,
+                       self.M, self.t, self.B if self.M else None, stream)
+        abi.score_tiles(X, self.xdt, self.N, self.n_v, self.d, self.t, self.B if self.M else None, self.M,
+                        self.knn_m, self.token_scores, self.tile_s_raw, self.tile_s,
+                        self.nbr if self.m > 0 else None, self.ws_score, self.ws_score_bytes, stream)
+        abi.select_budgeted_tokens(self.token_scores, self.tile_s, self.N, self.n_v, p, self.policy, self.u,
+                                   self.kept, self.n_kept, self.budgets, self.sel, self.sel_off, None, 0, stream)
+
+    def pack(self, X, embed, sys_ids, query_ids, stream=None):
+        """a8: the packed batch, cu_seqlens and positions."""
+        abi.pack_ragged(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.sel, self.sel_off,
+                        sys_ids, self.S, query_ids, self.Q, embed, embed.shape[0], self.packed, self.max_T,
+                        self.cu, self.positions, self.T, stream)
+
+    def read_counts(self, stream=None):
+        """Sync, check device error flags and read (n_kept, T) back to the host."""
+        s = stream if stream is not None else torch.cuda.current_stream()
+        self.counts_host[0:1].copy_(self.n_kept, non_blocking=True)
+        self.counts_host[1:2].copy_(self.T, non_blocking=True)
+        abi.sync_status(s)
+        return int(self.counts_host[0]), int(self.counts_host[1])
+
+    def prefill(self, T, n_seq, stream=None):
+        """a9: decoder prefill over the packed batch, in place."""
+        ws, need = self._prefill_ws(T, n_seq)
+        abi.prefill_layers(self.model.struct, self.packed, T, self.cu, n_seq, self.max_len, self.positions, ws,
+                           need, stream)
+
+    def run(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, prefill=True, stream=None):
+        self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)
+        self.pack(X, embed, sys_ids, query_ids, stream)
+        n_kept, T = self.read_counts(stream)
+        if prefill and self.model is not None and T > 0:
+            self.prefill(T, n_kept, stream)
+        return n_kept, T
+
+    def result(self, n_kept, T) -> QueryResult:
+        return QueryResult(n_kept, T, self.t, self.token_scores, self.tile_s_raw, self.tile_s,
+                           self.nbr[:self.N * self.m].view(self.N, self.m), self.u, self.kept[:n_kept],
+                           self.budgets[:n_kept], self.sel, self.sel_off[:n_kept + 1], self.cu[:n_kept + 1],
+                           self.positions[:T], self.packed[:T])

@@ -1,0 +1,121 @@
+"""The C-ABI library builds, loads and exports every entry point of include/rift.h; host-side
+argument validation rejects bad calls before anything reaches a GPU.  No GPU needed."""
+import ctypes as C
+import re
+from pathlib import Path
+
+import pytest
+
+HEADER = Path(__file__).resolve().parent.parent / "include" / "rift.h"
+
+
+def declared_functions():
+    text = re.sub(r"/\*.*?\*/", "", HEADER.read_text(), flags=re.S)
+    names = re.findall(r"^[A-Za-z_][\w\s\*]*?\b(rift_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_hot_path_calls():
+    names = declared_functions()
+    for n in ("rift_query_prep", "rift_score_tiles", "rift_select_budgeted_tokens", "rift_pack_ragged",
+              "rift_prefill_layers", "rift_sync_status"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(riftlib):
+    lib = C.CDLL(str(riftlib.LIB_PATH))
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_status_strings(riftlib):
+    assert riftlib.status_string(0) == "ok"
+    assert riftlib.status_string(riftlib.RIFT_ERR_CAPACITY) == "output capacity exceeded"
+    assert riftlib.abi_version() == 1
+
+
+FAKE = 0x10000  # a 16-byte aligned non-null address; validation rejects before using it
+
+
+def test_score_tiles_rejects_bad_shapes(riftlib):
+    lib = riftlib.lib
+    ws = riftlib.score_workspace_bytes(4, 576, 256, 8)
+    assert ws > 0
+    args = dict(X=FAKE, xdt=1, N=4, n_v=576, d=256, t=FAKE, B=FAKE, M=8, knn_m=6, r=FAKE, s0=FAKE, s1=FAKE,
+                nbr=None, ws=FAKE, wsb=ws, st=0)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return lib.rift_score_tiles(a["X"], a["xdt"], a["N"], a["n_v"], a["d"], a["t"], a["B"], a["M"], a["knn_m"],
+                                    a["r"], a["s0"], a["s1"], a["nbr"], a["ws"], a["wsb"], a["st"])
+
+    INV = riftlib.RIFT_ERR_INVALID
+    assert call(N=0) == INV
+    assert call(n_v=0) == INV and call(n_v=1025) == INV
+    assert call(d=100) == INV and call(d=8256) == INV
+    assert call(knn_m=-1) == INV and call(knn_m=17) == INV
+    assert call(X=None) == INV and call(r=None) == INV
+    assert call(X=FAKE + 4) == INV            # misaligned tokens
+    assert call(wsb=ws - 1) == INV            # workspace too small
+    assert call(ws=FAKE + 8) == INV           # workspace misaligned
+    assert call(xdt=7) == INV
+    assert call(M=1, B=None) == INV
+    assert call(xdt=0, d=8192) == riftlib.RIFT_ERR_UNSUPPORTED
+
+
+def _policy(riftlib, **kw):
+    from synth import workloads as W
+    p = riftlib.make_policy(W.RIFT_POLICY)
+    for k, v in kw.items():
+        setattr(p, k, v)
+    return p
+
+
+def test_select_rejects_bad_policies(riftlib):
+    lib = riftlib.lib
+
+    def call(pol, N=4, n_v=576):
+        return lib.rift_select_budgeted_tokens(FAKE, FAKE, N, n_v, None, C.byref(pol), FAKE, FAKE, FAKE, FAKE,
+                                               FAKE, FAKE, None, 0, 0)
+
+    INV = riftlib.RIFT_ERR_INVALID
+    assert call(_policy(riftlib, tau=1.5)) == INV
+    assert call(_policy(riftlib, tau=float("nan"))) == INV
+    assert call(_policy(riftlib, n_c=0)) == INV and call(_policy(riftlib, n_c=9)) == INV
+    p = _policy(riftlib)
+    p.C[1], p.C[2] = p.C[2], p.C[1]          # not ascending
+    assert call(p) == INV
+    assert call(_policy(riftlib), n_v=288) == INV   # C holds 576 > n_v
+    p = _policy(riftlib)
+    p.alpha_pos[0] = float("inf")
+    assert call(p) == INV
+    assert call(_policy(riftlib), N=0) == INV
+
+
+def test_pack_and_prefill_reject_bad_arguments(riftlib):
+    lib = riftlib.lib
+    INV = riftlib.RIFT_ERR_INVALID
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, None, 8, FAKE, 16, FAKE, 1000, FAKE,
+                                100, FAKE, FAKE, FAKE, 0) == INV  # S > 0 without ids
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000,
+                                FAKE + 2, 100, FAKE, FAKE, FAKE, 0) == INV  # misaligned output
+    m = riftlib.Model()
+    m.n_layers, m.d, m.n_heads, m.head_dim, m.ffn, m.eps, m.rope_theta = 2, 256, 4, 64, 688, 1e-6, 1e4
+    assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0  # null weight arrays
+    arr = (C.c_void_p * 2)(FAKE, FAKE)
+    for f in ("w_qkv", "w_o", "w_gate_up", "w_down", "g_attn", "g_ffn"):
+        setattr(m, f, arr)
+    m.g_final = FAKE
+    assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) > 0
+    m.head_dim = 96
+    assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0
+    m.head_dim, m.ffn = 64, 690
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, FAKE, 1 << 30, 0) == INV
+
+
+def test_query_prep_rejects_bad_arguments(riftlib):
+    lib = riftlib.lib
+    INV = riftlib.RIFT_ERR_INVALID
+    assert lib.rift_query_prep(FAKE, 1000, 256, FAKE, 0, 16, FAKE, 8, FAKE, FAKE, 0) == INV
+    assert lib.rift_query_prep(FAKE, 1000, 256, FAKE, 1, 16, None, 8, FAKE, FAKE, 0) == INV
+    assert lib.rift_query_prep(FAKE, 1000, 200, FAKE, 1, 16, FAKE, 8, FAKE, FAKE, 0) == INV
