@@ -40,7 +40,30 @@ def parse():
     ap.add_argument("--impl", default="rift", choices=["rift", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     return ap.parse_args()
+
+
+def ncu_summary(path: str) -> str:
+    """Per kernel: launches, total device time and share of an ncu --csv launch list."""
+    import csv
+    with open(path) as f:
+        rows = list(csv.DictReader([ln for ln in f if ln.startswith('"')]))
+    agg = {}
+    for r in rows:
+        if r.get("Metric Name") != "gpu__time_duration.sum":
+            continue
+        name = r["Kernel Name"].split("(")[0]
+        scale = {"ns": 1e-6, "us": 1e-3, "usecond": 1e-3, "ms": 1.0, "msecond": 1.0}.get(r["Metric Unit"], 1e-6)
+        t = float(r["Metric Value"].replace(",", "")) * scale
+        n, tot = agg.get(name, (0, 0.0))
+        agg[name] = (n + 1, tot + t)
+    total = sum(v[1] for v in agg.values())
+    out = [f"{'kernel':<44} {'launches':>8} {'total ms':>11} {'share':>7}"]
+    for name, (n, t) in sorted(agg.items(), key=lambda kv: -kv[1][1]):
+        out.append(f"{name:<44} {n:>8} {t:>11.3f} {100 * t / total:>6.2f}%")
+    out.append(f"{'all':<44} {sum(v[0] for v in agg.values()):>8} {total:>11.3f} 100.00%")
+    return "\n".join(out)
 
 
 # ------------------------------------------------------------------------------------------ dist
@@ -220,6 +243,9 @@ def run_reference(args, wl, ws, rank):
 
 def main():
     args = parse()
+    if args.ncu_summary:
+        print(ncu_summary(args.ncu_summary))
+        return
     ws, rank, local = dist_setup()
     wl = W.WORKLOADS[args.workload]
     if args.impl == "reference":

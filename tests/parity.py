@@ -27,9 +27,10 @@ HIDDEN_TOL = 2e-2    # final hidden states, max |g - o| / max |o| per sequence
 SMALL24 = W.Workload("small24_f32", W.SceneSpec(N=24, d=256, x_dtype="f32", planted_frac=0.1,
                                                 distractor_frac=0.15, S=8, Q=16),
                      W.TINY_DECODER, W.RIFT_POLICY, knn_m=6)
+# n_v = 200: the budget set C scaled from {72, ..., 576} of 576 tokens to 200 tokens
 RAGGED = W.Workload("ragged40_bf16", W.SceneSpec(N=40, d=256, x_dtype="bf16", n_v=200, grid=14,
                                                  planted_frac=0.1, distractor_frac=0.2, S=5, Q=7, M=3),
-                    W.TINY_DECODER, W.RIFT_POLICY_SKEW, knn_m=4)
+                    W.TINY_DECODER, replace(W.RIFT_POLICY_SKEW, C=(25, 50, 100, 150, 200)), knn_m=4)
 
 
 def to_dev(sc, device):
