@@ -150,6 +150,25 @@ rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int 
                              float* token_scores, float* tile_s_raw, float* tile_s, int* nbr,
                              void* ws, size_t ws_bytes, rift_stream_t stream);
 
+/* ---- rift_score_tiles without a workspace (no counterpart in the paper) ----
+ * For callers that cannot allocate device memory at all -- e.g. an edge or flight program
+ * whose device memory is planned once before launch, or a plug-in inside another runtime's
+ * memory pool -- this variant of rift_score_tiles takes its scratch from a fixed array
+ * compiled into the library (RIFT_NOALLOC_SCORE_SCRATCH_BYTES on every GPU that loads the
+ * library, held until the process exits) and allocates nothing.  Arguments and outputs are
+ * those of rift_score_tiles without ws/ws_bytes; results are the same.
+ *   - A scene whose scratch (rift_score_workspace_bytes(N, n_v, d, M)) exceeds the array
+ *     returns RIFT_ERR_CAPACITY and launches nothing (64 MiB holds N = 400 tiles at d = 4096).
+ *   - The first call on each device looks up the array's device address while that device is
+ *     current; make that first call before any stream capture.
+ *   - All calls share the array and it keeps the last call's contents (nothing needs to start
+ *     at zero).  Calls whose work overlaps on the GPU race on it: order them. */
+#define RIFT_NOALLOC_SCORE_SCRATCH_BYTES (64u << 20)
+rift_status rift_score_tiles_noalloc(const void* X, rift_dtype xdt, int N, int n_v, int d,
+                                     const float* t, const float* B, int M, int knn_m,
+                                     float* token_scores, float* tile_s_raw, float* tile_s, int* nbr,
+                                     rift_stream_t stream);
+
 /* ---- a5-a7. Prune, budget and select (Section 2.3; Appendix B Steps 3-4) ----
  *   token_scores, tile_s  from rift_score_tiles (tile_s = the smoothed scores)
  *   p          fp32 [N] (nullable): p_i, the probability that tile i holds the object;

@@ -56,6 +56,7 @@ SIGNATURES = {
                               _vp, _vp, _vp, _vp]),
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
     "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _sz, _vp]),
+    "rift_score_tiles_noalloc": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp]),
     "rift_profile_enable": (None, [_i]),
     "rift_profile_read": (_i, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), _i]),
     "rift_launch_count": (C.c_longlong, []),
@@ -138,6 +139,16 @@ def score_tiles(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_raw, til
     _check(lib.rift_score_tiles(ptr(X), xdt, N, n_v, d, ptr(t), ptr(B), M, knn_m, ptr(token_scores),
                                 ptr(tile_s_raw), ptr(tile_s), ptr(nbr), ptr(ws), ws_bytes, stream_handle(stream)),
            "rift_score_tiles")
+
+
+def score_tiles_noalloc(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_raw, tile_s, nbr, stream=None):
+    """rift_score_tiles for callers without an allocator: scratch from the library's fixed array."""
+    _check(lib.rift_score_tiles_noalloc(ptr(X), xdt, N, n_v, d, ptr(t), ptr(B), M, knn_m, ptr(token_scores),
+                                        ptr(tile_s_raw), ptr(tile_s), ptr(nbr), stream_handle(stream)),
+           "rift_score_tiles_noalloc")
+
+
+NOALLOC_SCORE_SCRATCH_BYTES = 64 << 20
 
 
 def select_workspace_bytes(N, n_v) -> int:
