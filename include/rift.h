@@ -226,6 +226,20 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 const int* positions,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
 
+/* ---- The linear layer of a9 on its own (the GEMM every prefill layer runs four times) ----
+ * out = A W^T with A bf16 [M, K], W bf16 [N, K] (both row-major, K contiguous), products
+ * accumulated in fp32 on the tensor cores, then:
+ *   RIFT_EPI_STORE_BF16  out bf16 [M, N] = A W^T
+ *   RIFT_EPI_RESID_F32   out fp32 [M, N] += A W^T      (the residual adds after W_o and W_down)
+ *   RIFT_EPI_SWIGLU      W holds gate and up rows interleaved in groups of 16 (as w_gate_up);
+ *                        out bf16 [M, N/2] = SiLU(x W_gate^T) * (x W_up^T), N % 32 == 0
+ * K % 8 == 0 and N % 8 == 0; A, W, out 16-byte aligned.  M == 0 is a no-op. */
+#define RIFT_EPI_STORE_BF16 0
+#define RIFT_EPI_RESID_F32 1
+#define RIFT_EPI_SWIGLU 2
+rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int epilogue, void* out,
+                        rift_stream_t stream);
+
 /* ---- Instrumentation for benchmarks (does not change any result) ----
  * Kernel classes timed by the profiler: */
 #define RIFT_PROF_GEMM 0      /* the prefill GEMMs (QKV, O, gate/up, down) */

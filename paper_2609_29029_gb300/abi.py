@@ -16,6 +16,7 @@ LIB_PATH = Path(__file__).resolve().parent / "libriftgb.so"
 RIFT_OK, RIFT_ERR_INVALID, RIFT_ERR_CAPACITY, RIFT_ERR_NONFINITE, RIFT_ERR_CUDA, RIFT_ERR_TIMEOUT, \
     RIFT_ERR_UNSUPPORTED, RIFT_ERR_BAD_ID = range(8)
 RIFT_F32, RIFT_BF16 = 0, 1
+RIFT_EPI_STORE_BF16, RIFT_EPI_RESID_F32, RIFT_EPI_SWIGLU = 0, 1, 2
 MAX_BUDGETS = 8
 
 
@@ -57,6 +58,7 @@ SIGNATURES = {
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
     "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _sz, _vp]),
     "rift_score_tiles_noalloc": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp]),
+    "rift_linear": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
     "rift_profile_enable": (None, [_i]),
     "rift_profile_read": (_i, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), _i]),
     "rift_launch_count": (C.c_longlong, []),
@@ -169,6 +171,10 @@ def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query
                                 ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(packed), max_T,
                                 ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),
            "rift_pack_ragged")
+
+
+def linear(A, W, M, N, K, epilogue, out, stream=None):
+    _check(lib.rift_linear(ptr(A), ptr(W), M, N, K, epilogue, ptr(out), stream_handle(stream)), "rift_linear")
 
 
 def prefill_workspace_bytes(model: Model, max_T, max_seqs, max_len) -> int:

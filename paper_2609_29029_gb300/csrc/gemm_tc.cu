@@ -1,0 +1,406 @@
+// The prefill GEMMs on Blackwell's fifth-generation tensor cores (tcgen05, sm_103a).
+//
+// C[M, N] = A[M, K] . B[N, K]^T with bf16 operands (both K-major) and fp32 accumulation in
+// tensor memory, plus the fused epilogues of the decoder layer (bf16 store, fp32 residual add,
+// SwiGLU over 16-column gate/up groups).
+//
+// Persistent, warp-specialised kernel, one CTA per SM (192 threads):
+//   warp 0      one thread issues TMA tile loads (128B-swizzled) into a 4-stage shared-memory ring
+//   warp 1      allocates 512 TMEM columns; one thread issues tcgen05.mma (M = 128, N = 256, K = 16)
+//               into one of two 256-column fp32 accumulators and commits to mbarriers
+//   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes (one row per thread), fused op, store
+// Two accumulators let the epilogue of one tile overlap the main loop of the next.  Tiles are
+// visited in bands of 8 M-tiles so a band's A rows and the current B tiles stay in L2.
+// Every mbarrier wait is bounded (RIFT_SPIN_LIMIT iterations, ~4 s of globaltimer): on timeout
+// the kernel sets RIFT_EBIT_TIMEOUT, lets every role fall through, waits for its issued copies
+// and frees its tensor memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "rift_internal.h"
+
+namespace rift {
+
+__device__ unsigned int g_err_gemm;
+
+unsigned int read_clear_err_gemm() {
+  unsigned int v = 0, z = 0;
+  cudaMemcpyFromSymbol(&v, g_err_gemm, sizeof(v));
+  cudaMemcpyToSymbol(g_err_gemm, &z, sizeof(z));
+  return v;
+}
+
+namespace tc {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;  // 16 KB
+constexpr int B_BYTES = BN * BK * 2;  // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int THREADS = 192;
+constexpr int ACC_COLS = BN;        // fp32 accumulator columns per buffer
+constexpr int TMEM_COLS = 2 * ACC_COLS;
+constexpr int GROUP_M = 8;
+constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+
+// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1), B bf16 (10-12 = 1),
+// both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                           ((uint32_t)(BM >> 4) << 24);
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Shared-memory matrix descriptor for a K-major tile written by TMA with 128-byte swizzling:
+// start address >> 4 (bits 0-13), leading byte offset 16 B (unused for this layout), stride
+// byte offset 1024 B between 8-row groups (bits 32-45), descriptor version 1 (bit 46),
+// swizzle mode 2 = 128B (bits 61-63).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.b32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded wait for the phase of parity `parity`.  Returns false if the kernel is aborting or
+// the wait ran out (which starts the abort).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 0; i < RIFT_SPIN_LIMIT; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 255u) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > 4000000000ull) break;
+    }
+  }
+  atomicOr(&g_err_gemm, RIFT_EBIT_TIMEOUT);
+  *abort_flag = 1;
+  return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accum));
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
+
+// 32 consecutive fp32 accumulator columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int& m_blk, int& n_blk) {
+  const int per_group = GROUP_M * nt;
+  const int grp = tile / per_group;
+  const int first_m = grp * GROUP_M;
+  const int gsz = min(mt - first_m, GROUP_M);
+  const int r = tile - grp * per_group;
+  m_blk = first_m + r % gsz;
+  n_blk = r / gsz;
+}
+
+__device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
+
+// Epilogue for one row of one 32-column chunk (columns n0 .. n0 + 31 of the tile).
+template <int EPI>
+__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row, int col, int N, void* C) {
+  if constexpr (EPI == EPI_STORE_BF16) {
+    uint16_t* out = static_cast<uint16_t*>(C) + (size_t)row * N + col;
+    if (col + 32 <= N) {
+      uint4* o4 = reinterpret_cast<uint4*>(out);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        o4[q] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
+                           pack_bf16x2(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
+                           pack_bf16x2(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
+                           pack_bf16x2(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; j += 2)
+        if (col + j < N)
+          *reinterpret_cast<uint32_t*>(out + j) = pack_bf16x2(__uint_as_float(r[j]), __uint_as_float(r[j + 1]));
+    }
+  } else if constexpr (EPI == EPI_RESID_F32) {
+    float* out = static_cast<float*>(C) + (size_t)row * N + col;
+    if (col + 32 <= N) {
+      float4* o4 = reinterpret_cast<float4*>(out);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 v = o4[q];
+        v.x += __uint_as_float(r[4 * q + 0]);
+        v.y += __uint_as_float(r[4 * q + 1]);
+        v.z += __uint_as_float(r[4 * q + 2]);
+        v.w += __uint_as_float(r[4 * q + 3]);
+        o4[q] = v;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col + j < N) out[j] += __uint_as_float(r[j]);
+    }
+  } else {  // EPI_SWIGLU: columns col..col+15 are gate, col+16..col+31 the matching up rows
+    if (col >= N) return;
+    const int F = N / 2;
+    uint16_t* out = static_cast<uint16_t*>(C) + (size_t)row * F + col / 2;
+    uint32_t p[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float g0 = __uint_as_float(r[2 * j]), g1 = __uint_as_float(r[2 * j + 1]);
+      const float u0 = __uint_as_float(r[16 + 2 * j]), u1 = __uint_as_float(r[16 + 2 * j + 1]);
+      p[j] = pack_bf16x2(silu(g0) * u0, silu(g1) * u1);
+    }
+    uint4* o4 = reinterpret_cast<uint4*>(out);
+    o4[0] = make_uint4(p[0], p[1], p[2], p[3]);
+    o4[1] = make_uint4(p[4], p[5], p[6], p[7]);
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
+                   int K, void* C) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull_bar(b), 1);
+      mbar_init(tempty_bar(b), 128);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int mt = (M + BM - 1) / BM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
+  const int n_tiles = mt * nt;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        int m_blk, n_blk;
+        tile_coords(tile, mt, nt, m_blk, n_blk);
+        for (int k = 0; k < kt; ++k, ++it) {
+          const int s = it % STAGES;
+          const uint32_t round = it / STAGES;
+          if (!mbar_wait(empty_bar(s), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+          mbar_expect_tx(full_bar(s), STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * BM, full_bar(s));
+          tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+        }
+      }
+      // Before leaving, make sure no copy this thread issued is still in flight (bounded).
+      for (int j = 1; j <= STAGES && it - j >= 0; ++j) {
+        const int i2 = it - j;
+        const int s = i2 % STAGES;
+        const uint32_t round = i2 / STAGES;
+        for (uint32_t w = 0; w < (1u << 22) && !mbar_try_wait(full_bar(s), round & 1u); ++w) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tl) {
+        const int b = tl & 1;
+        const uint32_t use = tl >> 1;
+        if (!mbar_wait(tempty_bar(b), (use & 1u) ^ 1u, abort_flag)) break;
+        fence_after();
+        const uint32_t tmem_d = tmem_base + (uint32_t)(b * ACC_COLS);
+        for (int k = 0; k < kt; ++k, ++it) {
+          const int s = it % STAGES;
+          const uint32_t round = it / STAGES;
+          if (!mbar_wait(full_bar(s), round & 1u, abort_flag)) { ok = false; break; }
+          fence_after();
+          const uint64_t ad = smem_desc(smem_u32(sA + s * A_BYTES));
+          const uint64_t bd = smem_desc(smem_u32(sB + s * B_BYTES));
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along K per step (encoded >> 4)
+            umma_bf16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k | kk) != 0 ? 1u : 0u);
+          umma_commit(empty_bar(s));
+        }
+        if (ok) umma_commit(tfull_bar(b));
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 -> TMEM lane quarters 2, 3, 0, 1)
+    const int quarter = warp & 3;
+    int tl = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++tl) {
+      int m_blk, n_blk;
+      tile_coords(tile, mt, nt, m_blk, n_blk);
+      const int b = tl & 1;
+      const uint32_t use = tl >> 1;
+      if (!mbar_wait(tfull_bar(b), use & 1u, abort_flag)) break;
+      fence_after();
+      const int row = m_blk * BM + quarter * 32 + lane;
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * ACC_COLS);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C);
+      }
+      fence_before();
+      mbar_arrive(tempty_bar(b));
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------------------------------------ host
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [rows, inner] (row-major, inner contiguous), box [box_rows, 64], 128B swizzle,
+// out-of-bounds elements read as zero.
+static bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+static int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int EPI>
+static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
+    attr = true;
+  }
+  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+  const int grid = tiles < sm_count() ? tiles : sm_count();
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C);
+  return 0;
+}
+
+}  // namespace tc
+
+// Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU), A, B and C
+// 16-byte aligned.
+int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st) {
+  using namespace tc;
+  if (M <= 0 || N <= 0 || K <= 0) return 0;
+  if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
+  switch (epi) {
+    case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, st);
+    case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, st);
+    case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, st);
+    default: return 1;
+  }
+}
+
+}  // namespace rift

@@ -126,12 +126,11 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   return L;
 }
 
-int launch_gemm_mma(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st);
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st);
 
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st) {
   prof_begin(RIFT_PROF_GEMM, st);
-  const int r = launch_gemm_mma(A, B, M, N, K, epi, C, st);
+  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, st);
   prof_end(RIFT_PROF_GEMM, st, 1);
   return r;
 }

@@ -117,7 +117,7 @@ const char* rift_status_string(rift_status s) {
 rift_status rift_sync_status(rift_stream_t stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return RIFT_ERR_CUDA;
   unsigned int f = read_clear_err_score() | read_clear_err_select() | read_clear_err_pack() |
-                   read_clear_err_prefill();
+                   read_clear_err_prefill() | read_clear_err_gemm();
   if (cudaGetLastError() != cudaSuccess) return RIFT_ERR_CUDA;
   if (f & RIFT_EBIT_BADID) return RIFT_ERR_BAD_ID;
   if (f & RIFT_EBIT_NONFINITE) return RIFT_ERR_NONFINITE;
@@ -250,6 +250,18 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const 
   if (launch_prefill(*m, hidden, T, cu_seqlens, n_seq, max_len, positions, static_cast<char*>(ws),
                      static_cast<cudaStream_t>(stream)))
     return RIFT_ERR_INVALID;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int epilogue, void* out,
+                        rift_stream_t stream) {
+  if (!A || !W || !out || M < 0 || N < 1 || K < 1) return RIFT_ERR_INVALID;
+  if (epilogue < RIFT_EPI_STORE_BF16 || epilogue > RIFT_EPI_SWIGLU) return RIFT_ERR_INVALID;
+  if (K % 8 != 0 || N % 8 != 0 || (epilogue == RIFT_EPI_SWIGLU && N % 32 != 0)) return RIFT_ERR_INVALID;
+  if (!aligned16(A) || !aligned16(W) || !aligned16(out)) return RIFT_ERR_INVALID;
+  if (M == 0) return RIFT_OK;
+  if (launch_gemm(A, W, M, N, K, epilogue, out, static_cast<cudaStream_t>(stream))) return RIFT_ERR_CUDA;
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }

@@ -15,6 +15,7 @@ unsigned int read_clear_err_score();
 unsigned int read_clear_err_select();
 unsigned int read_clear_err_pack();
 unsigned int read_clear_err_prefill();
+unsigned int read_clear_err_gemm();
 
 // ---- score.cu ----
 struct ScoreLayout {
