@@ -41,6 +41,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
+    ap.add_argument("--kernel-case", choices=["prefill", "score"],
+                    help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
+                         "'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); each runs 3 times")
     return ap.parse_args()
 
 
@@ -241,10 +244,46 @@ def run_reference(args, wl, ws, rank):
 
 # ------------------------------------------------------------------------------------------ main arm
 
+def kernel_case(name: str):
+    """Small cases for ncu captures: inputs larger than L2, about 1 GB on the device."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_29029_gb300 import DeviceModel, ScenePipeline, abi
+    dev = torch.device("cuda", 0)
+    if name == "prefill":
+        dec = W.DecoderShape(n_layers=1, d=4096, n_heads=32, head_dim=128, ffn=11008, vocab=32000)
+        dm = DeviceModel(dec, [W.make_layer(dec, 0, dev)], W.make_final_norm(dec, dev), dev)
+        lens = [341] * 12
+        T = sum(lens)
+        from synth import rng
+        H0 = rng.normal_f32(0, rng.stream_id("case"), T * dec.d, dev).view(T, dec.d).to(torch.bfloat16)
+        cu = torch.tensor([0] + [sum(lens[:i + 1]) for i in range(len(lens))], dtype=torch.int32, device=dev)
+        pos = torch.cat([torch.arange(L, dtype=torch.int32, device=dev) for L in lens])
+        need = abi.prefill_workspace_bytes(dm.struct, T, len(lens), 635)
+        ws = torch.empty(need, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            hid = H0.clone()
+            abi.prefill_layers(dm.struct, hid, T, cu, len(lens), 635, pos, ws, need)
+        abi.sync_status()
+    else:
+        wl = W.sweep_workload(64)
+        s = wl.scene
+        sc = W.make_scene(s, wl.decoder.vocab, dev)
+        pipe = ScenePipeline(s.N, s.n_v, s.d, s.x_dtype, s.M, s.S, s.Q, wl.knn_m, wl.policy, device=dev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        for _ in range(3):
+            pipe.select(sc.X, sc.embed, torch.tensor(sc.query_ids, **i32), torch.tensor(sc.bg_ids, **i32))
+        abi.sync_status()
+    print(f"kernel case {name}: ok")
+
+
 def main():
     args = parse()
     if args.ncu_summary:
         print(ncu_summary(args.ncu_summary))
+        return
+    if args.kernel_case:
+        kernel_case(args.kernel_case)
         return
     ws, rank, local = dist_setup()
     wl = W.WORKLOADS[args.workload]

@@ -85,7 +85,8 @@ typedef struct {
 
 /* A LLaMA/Vicuna-shaped decoder (Section 2.1; LLaVA-1.5-7B: 32 layers, d 4096, 32 heads
  * x 128, FFN 11008, eps 1e-6, rope_theta 1e4).  The per-layer fields are HOST arrays of
- * n_layers DEVICE pointers to bf16 weights:
+ * n_layers DEVICE pointers; projection weights are fp16 (the tensor-core operand type, and the
+ * dtype of the LLaVA-1.5-7B checkpoint), norm gains bf16:
  *   w_qkv      [3d, d]   rows 0..d-1 = W_q, d..2d-1 = W_k, 2d..3d-1 = W_v (out x in)
  *   w_o        [d, d]
  *   w_gate_up  [2 ffn, d] W_gate and W_up interleaved in groups of 16 rows:
@@ -139,8 +140,8 @@ rift_status rift_query_prep(const void* embed, int vocab, int d,
  *                 (Eq. 1 applied to each token)
  *   tile_s_raw    out fp32 [N]: s_i = V_i . w, V_i = P_i / ||P_i||, P_i = sum_k x_ik (Eq. 1)
  *   tile_s        out fp32 [N]: s~_i = (sum over {i} + NN(i) in ascending index of s_j)
- *                 / (m + 1), NN(i) = the m tiles j != i of largest fp32 V_i . V_j, ties to
- *                 the lower j
+ *                 / (m + 1), NN(i) = the m tiles j != i of largest V_i . V_j, ties to the lower
+ *                 j (candidates found in fp32, ranked by their fp64-accumulated similarity)
  *   nbr           out int32 [N, m] (nullable): NN(i) in rank order
  * Limits: 1 <= N <= RIFT_MAX_TILES, 1 <= n_v <= RIFT_MAX_NV, 64 <= d <= 8192, d % 64 == 0,
  * 0 <= M <= 64; X 16-byte aligned. */
@@ -219,7 +220,8 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
  *   max_len    an upper bound on every sequence length (host int)
  * Each layer: h += W_o Attn(RoPE(q), RoPE(k), v) with x = RMSNorm(h) g_attn, causal within
  * each sequence only; h += W_down(SiLU(W_gate x) * (W_up x)) with x = RMSNorm(h) g_ffn.
- * GEMMs take bf16 operands and accumulate in fp32. */
+ * GEMM and attention operands are fp16 (normalised activations, q/k/v, softmax weights,
+ * attention output, SwiGLU output), accumulation fp32, residual stream fp32. */
 size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len);
 rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 const int* cu_seqlens, int n_seq, int max_len,
@@ -227,14 +229,14 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
 
 /* ---- The linear layer of a9 on its own (the GEMM every prefill layer runs four times) ----
- * out = A W^T with A bf16 [M, K], W bf16 [N, K] (both row-major, K contiguous), products
+ * out = A W^T with A fp16 [M, K], W fp16 [N, K] (both row-major, K contiguous), products
  * accumulated in fp32 on the tensor cores, then:
- *   RIFT_EPI_STORE_BF16  out bf16 [M, N] = A W^T
+ *   RIFT_EPI_STORE_F16   out fp16 [M, N] = A W^T
  *   RIFT_EPI_RESID_F32   out fp32 [M, N] += A W^T      (the residual adds after W_o and W_down)
  *   RIFT_EPI_SWIGLU      W holds gate and up rows interleaved in groups of 16 (as w_gate_up);
- *                        out bf16 [M, N/2] = SiLU(x W_gate^T) * (x W_up^T), N % 32 == 0
+ *                        out fp16 [M, N/2] = SiLU(x W_gate^T) * (x W_up^T), N % 32 == 0
  * K % 8 == 0 and N % 8 == 0; A, W, out 16-byte aligned.  M == 0 is a no-op. */
-#define RIFT_EPI_STORE_BF16 0
+#define RIFT_EPI_STORE_F16 0
 #define RIFT_EPI_RESID_F32 1
 #define RIFT_EPI_SWIGLU 2
 rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int epilogue, void* out,

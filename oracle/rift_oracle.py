@@ -15,10 +15,13 @@ Each function restates one step of the paper in the paper's order:
   Section 2.1 ......................... decoder prefill over [system | vision | query]
 
 Precision.  Scores are computed in fp64 and rounded once to fp32; every
-decision (neighbour choice, min-max, threshold, utility argmax, top-b order) is
-then taken in fp32, with each fp32 operation written out one at a time in the
-order given below, so the result is fixed by IEEE round-to-nearest.  The
-prefill is fp64 throughout, on weights and inputs that are bf16 values.
+decision (min-max, threshold, utility argmax, top-b order) is then taken in
+fp32, with each fp32 operation written out one at a time in the order given
+below, so the result is fixed by IEEE round-to-nearest.  The one exception is
+the neighbour choice of the smoothing step: tile similarities are compared in
+fp64, because nearly parallel tiles have similarities closer to 1 than fp32's
+spacing there (6e-8), which would turn their order into a rounding accident.
+The prefill is fp64 throughout, on weights and inputs that are bf16 values.
 
 Readings of points the paper leaves open (each also used by the CUDA path):
   * Stand-in embeddings (the paper uses RemoteCLIP): V_i = l2norm(mean_k x_ik)
@@ -128,18 +131,18 @@ def to_f32(x) -> np.ndarray:
 # a4  kNN smoothing (Appendix B Step 2; Listing 1 comment: smoothed with the 6 most similar tiles)
 # ------------------------------------------------------------------------------------------
 
-def similarity_f32(V: torch.Tensor) -> np.ndarray:
-    """Cosine similarities G = V V^T in fp64, rounded to fp32 for the neighbour decision."""
-    return to_f32(V @ V.T)
+def similarity(V: torch.Tensor) -> np.ndarray:
+    """Cosine similarities G = V V^T in fp64 (the neighbour decision compares these)."""
+    return (V @ V.T).numpy()
 
 
-def knn_neighbours(G32: np.ndarray, m: int) -> np.ndarray:
+def knn_neighbours(G: np.ndarray, m: int) -> np.ndarray:
     """For each i: the m tiles j != i of largest G_ij, ties to the lower j, in rank order."""
-    N = G32.shape[0]
+    N = G.shape[0]
     m = min(m, N - 1)
     nbr = np.zeros((N, max(m, 0)), dtype=np.int64)
     for i in range(N):
-        cand = [(-float(G32[i, j]), j) for j in range(N) if j != i]
+        cand = [(-float(G[i, j]), j) for j in range(N) if j != i]
         cand.sort()
         nbr[i] = [j for _, j in cand[:m]]
     return nbr
@@ -314,7 +317,7 @@ class Selection:
     s64: torch.Tensor          # [N] fp64 Eq. 1 tile scores
     r32: np.ndarray
     s32: np.ndarray
-    G32: np.ndarray
+    G: np.ndarray              # [N, N] fp64 similarities
     nbr: np.ndarray            # [N, m]
     s_tilde: np.ndarray        # [N] fp32
     u: np.ndarray              # [N] fp32
@@ -324,9 +327,9 @@ class Selection:
     sel: list                  # per kept tile, ascending token indices
 
 
-def decide(r32, s32, G32, m, policy, p_ext=None):
-    """Every decision of a5-a7 from fp32 scores."""
-    nbr = knn_neighbours(G32, m)
+def decide(r32, s32, G, m, policy, p_ext=None):
+    """Every decision of a4-a7 from the fp32 scores and the fp64 similarities."""
+    nbr = knn_neighbours(G, m)
     st = smooth(s32, nbr)
     u = minmax_normalize(st)
     kept = retained(u, policy.tau)
@@ -344,6 +347,6 @@ def select(X, embed, query_ids, bg_ids, m, policy, p_ext=None, templates=None) -
     B = background_embeddings(embed, bg_ids)
     r64, V, s64 = score_scene(X, t, B)
     r32, s32 = to_f32(r64), to_f32(s64)
-    G32 = similarity_f32(V)
-    nbr, st, u, kept, p, bud, sel = decide(r32, s32, G32, m, policy, p_ext)
-    return Selection(t, B, r64, V, s64, r32, s32, G32, nbr, st, u, kept, p, bud, sel)
+    G = similarity(V)
+    nbr, st, u, kept, p, bud, sel = decide(r32, s32, G, m, policy, p_ext)
+    return Selection(t, B, r64, V, s64, r32, s32, G, nbr, st, u, kept, p, bud, sel)

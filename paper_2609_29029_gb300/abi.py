@@ -16,7 +16,7 @@ LIB_PATH = Path(__file__).resolve().parent / "libriftgb.so"
 RIFT_OK, RIFT_ERR_INVALID, RIFT_ERR_CAPACITY, RIFT_ERR_NONFINITE, RIFT_ERR_CUDA, RIFT_ERR_TIMEOUT, \
     RIFT_ERR_UNSUPPORTED, RIFT_ERR_BAD_ID = range(8)
 RIFT_F32, RIFT_BF16 = 0, 1
-RIFT_EPI_STORE_BF16, RIFT_EPI_RESID_F32, RIFT_EPI_SWIGLU = 0, 1, 2
+RIFT_EPI_STORE_F16, RIFT_EPI_RESID_F32, RIFT_EPI_SWIGLU = 0, 1, 2
 MAX_BUDGETS = 8
 
 

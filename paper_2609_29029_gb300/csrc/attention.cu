@@ -4,8 +4,8 @@
 //
 // CTA = (q-block of 64 rows of one sequence, one head), 4 warps x 16 query rows.  K/V tiles
 // of 64 keys are double-buffered through shared memory with cp.async; S = Q K^T and O = P V
-// run on mma.sync m16n8k16 (bf16 in, fp32 accumulate) with an online softmax in fp32 (exp2,
-// scale folded with log2 e).  P is re-used from the S accumulators as the A operand.
+// run on mma.sync m16n8k16 (fp16 in, fp32 accumulate) with an online softmax in fp32 (exp2,
+// scale folded with log2 e).  P is re-used from the S accumulators as the A operand (fp16).
 #include "rift_internal.h"
 
 namespace rift {
@@ -31,9 +31,9 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
 }
-__device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+__device__ __forceinline__ void mma_f16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
   asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};\n"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
@@ -135,8 +135,8 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const uint16_t* __restric
         const int col = kk * 16 + ((lane >> 3) & 1) * 8;
         uint32_t r0, r1, r2, r3;
         ldsm_x4(smem_u32(Ks + (buf * BKV + row) * LD + col), r0, r1, r2, r3);
-        mma_bf16(s[2 * jp], qf[kk], r0, r1);
-        mma_bf16(s[2 * jp + 1], qf[kk], r2, r3);
+        mma_f16(s[2 * jp], qf[kk], r0, r1);
+        mma_f16(s[2 * jp + 1], qf[kk], r2, r3);
       }
     }
     // mask (causal + sequence end), online softmax
@@ -174,8 +174,8 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const uint16_t* __restric
       const float p2 = exp2f(s[j][2] - mx[1]), p3 = exp2f(s[j][3] - mx[1]);
       rsum[0] += p0 + p1;
       rsum[1] += p2 + p3;
-      pf[j >> 1][(j & 1) * 2 + 0] = pack_bf16x2(p0, p1);
-      pf[j >> 1][(j & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+      pf[j >> 1][(j & 1) * 2 + 0] = pack_half2(p0, p1);
+      pf[j >> 1][(j & 1) * 2 + 1] = pack_half2(p2, p3);
     }
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
@@ -199,8 +199,8 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const uint16_t* __restric
         const int col = jp * 16 + (lane >> 4) * 8;
         uint32_t r0, r1, r2, r3;
         ldsm_x4_t(smem_u32(Vs + (buf * BKV + row) * LD + col), r0, r1, r2, r3);
-        mma_bf16(o[2 * jp], a, r0, r1);
-        mma_bf16(o[2 * jp + 1], a, r2, r3);
+        mma_f16(o[2 * jp], a, r0, r1);
+        mma_f16(o[2 * jp + 1], a, r2, r3);
       }
     }
     __syncthreads();  // the buffer is refilled two iterations later
@@ -215,7 +215,7 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const uint16_t* __restric
     uint16_t* dst = out + (size_t)(seq0 + qr) * d + h * HD;
 #pragma unroll
     for (int j = 0; j < HD / 8; ++j)
-      *reinterpret_cast<uint32_t*>(dst + j * 8 + c2) = pack_bf16x2(o[j][2 * r] * inv, o[j][2 * r + 1] * inv);
+      *reinterpret_cast<uint32_t*>(dst + j * 8 + c2) = pack_half2(o[j][2 * r] * inv, o[j][2 * r + 1] * inv);
   }
 }
 

@@ -1,8 +1,8 @@
 // The prefill GEMMs on Blackwell's fifth-generation tensor cores (tcgen05, sm_103a).
 //
-// C[M, N] = A[M, K] . B[N, K]^T with bf16 operands (both K-major) and fp32 accumulation in
-// tensor memory, plus the fused epilogues of the decoder layer (bf16 store, fp32 residual add,
-// SwiGLU over 16-column gate/up groups).
+// C[M, N] = A[M, K] . B[N, K]^T with fp16 operands (both K-major) and fp32 accumulation in
+// tensor memory, plus the fused epilogues of the decoder layer (fp16 store with RoPE on q and
+// k, fp32 residual add, SwiGLU over 16-column gate/up groups).
 //
 // Persistent, warp-specialised kernel, one CTA per SM (192 threads):
 //   warp 0      one thread issues TMA tile loads (128B-swizzled) into a 4-stage shared-memory ring
@@ -10,7 +10,7 @@
 //               into one of two 256-column fp32 accumulators and commits to mbarriers
 //   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes (one row per thread), fused op, store
 // Two accumulators let the epilogue of one tile overlap the main loop of the next.  Tiles are
-// visited in bands of 8 M-tiles so a band's A rows and the current B tiles stay in L2.
+// visited in bands of 16 M-tiles so a band's A rows and the current B tiles stay in L2.
 // Every mbarrier wait is bounded (RIFT_SPIN_LIMIT iterations, ~4 s of globaltimer): on timeout
 // the kernel sets RIFT_EBIT_TIMEOUT, lets every role fall through, waits for its issued copies
 // and frees its tensor memory.
@@ -41,13 +41,12 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 192;
 constexpr int ACC_COLS = BN;        // fp32 accumulator columns per buffer
 constexpr int TMEM_COLS = 2 * ACC_COLS;
-constexpr int GROUP_M = 8;
+constexpr int GROUP_M = 16;
 constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
 
-// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1), B bf16 (10-12 = 1),
-// both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                           ((uint32_t)(BM >> 4) << 24);
+// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A fp16 (bits 7-9 = 0), B fp16
+// (bits 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -111,7 +110,7 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accum) {
+__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accum) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
@@ -158,15 +157,15 @@ __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row,
       uint4* o4 = reinterpret_cast<uint4*>(out);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        o4[q] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
-                           pack_bf16x2(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
-                           pack_bf16x2(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
-                           pack_bf16x2(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
+        o4[q] = make_uint4(pack_half2(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
+                           pack_half2(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
+                           pack_half2(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
+                           pack_half2(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
     } else {
 #pragma unroll
       for (int j = 0; j < 32; j += 2)
         if (col + j < N)
-          *reinterpret_cast<uint32_t*>(out + j) = pack_bf16x2(__uint_as_float(r[j]), __uint_as_float(r[j + 1]));
+          *reinterpret_cast<uint32_t*>(out + j) = pack_half2(__uint_as_float(r[j]), __uint_as_float(r[j + 1]));
     }
   } else if constexpr (EPI == EPI_RESID_F32) {
     float* out = static_cast<float*>(C) + (size_t)row * N + col;
@@ -195,7 +194,7 @@ __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row,
     for (int j = 0; j < 8; ++j) {
       const float g0 = __uint_as_float(r[2 * j]), g1 = __uint_as_float(r[2 * j + 1]);
       const float u0 = __uint_as_float(r[16 + 2 * j]), u1 = __uint_as_float(r[16 + 2 * j + 1]);
-      p[j] = pack_bf16x2(silu(g0) * u0, silu(g1) * u1);
+      p[j] = pack_half2(silu(g0) * u0, silu(g1) * u1);
     }
     uint4* o4 = reinterpret_cast<uint4*>(out);
     o4[0] = make_uint4(p[0], p[1], p[2], p[3]);
@@ -203,10 +202,36 @@ __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row,
   }
 }
 
+// Rotate-half RoPE on fp32 accumulators: r1 holds dims j0..j0+31 of a head, r2 the partner
+// dims j0+half..; y1 = x1 cos - x2 sin, y2 = x2 cos + x1 sin, rounded once to fp16.
+__device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint32_t (&r2)[32], int row, int col,
+                                           int half, int N, int pos, const float2* __restrict__ tab, void* C) {
+  uint16_t* out = static_cast<uint16_t*>(C) + (size_t)row * N + col;
+  const int head_dim = 2 * half;
+  const int j0 = col % head_dim;
+  const float2* cs = tab + (size_t)pos * half + j0;
+  uint32_t p1[16], p2[16];
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    const float2 c0 = cs[e], c1 = cs[e + 1];
+    const float a0 = __uint_as_float(r1[e]), a1 = __uint_as_float(r1[e + 1]);
+    const float b0 = __uint_as_float(r2[e]), b1 = __uint_as_float(r2[e + 1]);
+    p1[e / 2] = pack_half2(a0 * c0.x - b0 * c0.y, a1 * c1.x - b1 * c1.y);
+    p2[e / 2] = pack_half2(b0 * c0.x + a0 * c0.y, b1 * c1.x + a1 * c1.y);
+  }
+  uint4* o1 = reinterpret_cast<uint4*>(out);
+  uint4* o2 = reinterpret_cast<uint4*>(out + half);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    o1[q] = make_uint4(p1[4 * q], p1[4 * q + 1], p1[4 * q + 2], p1[4 * q + 3]);
+    o2[q] = make_uint4(p2[4 * q], p2[4 * q + 1], p2[4 * q + 2], p2[4 * q + 3]);
+  }
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, void* C) {
+                   int K, void* C, const EpiParams ep) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -294,7 +319,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t bd = smem_desc(smem_u32(sB + s * B_BYTES));
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along K per step (encoded >> 4)
-            umma_bf16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k | kk) != 0 ? 1u : 0u);
+            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k | kk) != 0 ? 1u : 0u);
           umma_commit(empty_bar(s));
         }
         if (ok) umma_commit(tfull_bar(b));
@@ -313,11 +338,34 @@ __global__ void __launch_bounds__(THREADS, 1)
       fence_after();
       const int row = m_blk * BM + quarter * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * ACC_COLS);
+      if constexpr (EPI == EPI_QKV_ROPE) {
+        const int half = ep.head_dim >> 1;
+        const int pos = (row < M) ? ep.positions[row] : 0;
+        const bool pos_ok = pos >= 0 && pos < ep.max_len;
+        if (row < M && !pos_ok) atomicOr(&g_err_gemm, RIFT_EBIT_BADID);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c, r);
-        if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C);
+        for (int c = 0; c < BN; c += 32) {
+          const int col = n_blk * BN + c;
+          if (col >= N) break;
+          if (col < ep.rope_cols) {
+            if ((c % ep.head_dim) >= half) continue;  // done with its partner c - half
+            uint32_t r1[32], r2[32];
+            tmem_ld32(taddr + c, r1);
+            tmem_ld32(taddr + c + half, r2);
+            if (row < M && pos_ok) rope_chunk(r1, r2, row, col, half, N, pos, ep.rope, C);
+          } else {
+            uint32_t r[32];
+            tmem_ld32(taddr + c, r);
+            if (row < M) epilogue_chunk<EPI_STORE_BF16>(r, row, col, N, C);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c, r);
+          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C);
+        }
       }
       fence_before();
       mbar_arrive(tempty_bar(b));
@@ -347,7 +395,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 2-D bf16 tensor [rows, inner] (row-major, inner contiguous), box [box_rows, 64], 128B swizzle,
+// 2-D fp16 tensor [rows, inner] (row-major, inner contiguous), box [box_rows, 64], 128B swizzle,
 // out-of-bounds elements read as zero.
 static bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
   auto fn = encode_fn();
@@ -356,7 +404,7 @@ static bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_
   cuuint64_t strides[1] = {inner * 2};
   cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -373,7 +421,8 @@ static int sm_count() {
 }
 
 template <int EPI>
-static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, cudaStream_t st) {
+static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
+                  cudaStream_t st) {
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
@@ -381,24 +430,28 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   }
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = tiles < sm_count() ? tiles : sm_count();
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C);
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep);
   return 0;
 }
 
 }  // namespace tc
 
-// Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU), A, B and C
-// 16-byte aligned.
-int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st) {
+// Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
+// the RoPE epilogue), A, B and C 16-byte aligned.
+int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
+                   cudaStream_t st) {
   using namespace tc;
   if (M <= 0 || N <= 0 || K <= 0) return 0;
   if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
+  if (epi == EPI_QKV_ROPE && (N % 64 != 0 || (ep.head_dim != 64 && ep.head_dim != 128) || !ep.positions || !ep.rope))
+    return 1;
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
   switch (epi) {
-    case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, st);
-    case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, st);
-    case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, st);
+    case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, ep, st);
+    case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, ep, st);
+    case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, ep, st);
+    case EPI_QKV_ROPE: return launch<EPI_QKV_ROPE>(ma, mb, M, N, K, C, ep, st);
     default: return 1;
   }
 }

@@ -1,16 +1,18 @@
 // Decoder prefill over the packed batch (Section 2.1): the per-layer kernel sequence, the
 // fused RMSNorm kernels and RoPE.
 //
-// Per layer, with the residual stream h kept in fp32:
-//   xn  = RMSNorm(h) g_attn                      rmsnorm_kernel            (bf16 out)
-//   qkv = xn W_qkv^T                             GEMM, bf16 store
-//   q,k = RoPE(q,k)                              rope_kernel (in place)
+// Per layer, with the residual stream h kept in fp32 and every GEMM operand in fp16:
+//   xn  = RMSNorm(h) g_attn                      rmsnorm_kernel            (fp16 out)
+//   qkv = xn W_qkv^T, RoPE on q and k            GEMM, RoPE epilogue on the fp32 accumulators
 //   a   = causal varlen attention(q, k, v)       attention
 //   h  += a W_o^T                                GEMM, fp32 residual epilogue
 //   xn  = RMSNorm(h) g_ffn
 //   act = SiLU(xn W_g^T) * (xn W_u^T)            GEMM, SwiGLU epilogue (interleaved gate/up)
 //   h  += act W_down^T                           GEMM, fp32 residual epilogue
 // and finally hidden = RMSNorm(h) g_final in bf16.
+// fp16 rather than bf16 operands: after 32 layers the bf16 rounding of the GEMM inputs alone
+// moves the final hidden states by about 3% of their largest magnitude; fp16 (3 more mantissa
+// bits, same tensor-core rate, LLaVA-1.5-7B's checkpoint dtype) keeps the whole path near 0.5%.
 #include "rift_internal.h"
 
 namespace rift {
@@ -28,8 +30,9 @@ constexpr int NORM_THREADS = 256;
 constexpr int NORM_MAXV = 8;  // float4 per thread: d <= 8192
 
 // y = h / sqrt(mean(h^2) + eps) * g, one CTA per row.  IN_BF16: h is the bf16 packed input,
-// which is also widened into the fp32 residual stream h32.
-template <bool IN_BF16>
+// which is also widened into the fp32 residual stream h32.  OUT_F16: y in fp16 (the GEMM
+// operand); otherwise bf16 (the final hidden states).
+template <bool IN_BF16, bool OUT_F16>
 __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __restrict__ in,
                                                                float* __restrict__ h32,
                                                                const uint16_t* __restrict__ gain,
@@ -64,8 +67,13 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __res
       const float g0 = __uint_as_float(gr.x << 16), g1 = __uint_as_float(gr.x & 0xffff0000u);
       const float g2 = __uint_as_float(gr.y << 16), g3 = __uint_as_float(gr.y & 0xffff0000u);
       uint2 o;
-      o.x = pack_bf16x2(v[q].x * inv * g0, v[q].y * inv * g1);
-      o.y = pack_bf16x2(v[q].z * inv * g2, v[q].w * inv * g3);
+      if constexpr (OUT_F16) {
+        o.x = pack_half2(v[q].x * inv * g0, v[q].y * inv * g1);
+        o.y = pack_half2(v[q].z * inv * g2, v[q].w * inv * g3);
+      } else {
+        o.x = pack_bf16x2(v[q].x * inv * g0, v[q].y * inv * g1);
+        o.y = pack_bf16x2(v[q].z * inv * g2, v[q].w * inv * g3);
+      }
       reinterpret_cast<uint2*>(out + row * d)[c] = o;
     }
   }
@@ -80,33 +88,6 @@ __global__ void rope_table_kernel(float2* __restrict__ tab, int max_len, int hal
   double s, c;
   sincos((double)p * inv, &s, &c);
   tab[i] = make_float2((float)c, (float)s);
-}
-
-// Rotate-half RoPE on q and k in place: dims j and j + hd/2 of each head form a pair.
-// One thread per (row, head, pair) of q and the same of k.
-__global__ void rope_kernel(uint16_t* __restrict__ qkv, const int* __restrict__ positions, int T, int H,
-                            int hd, const float2* __restrict__ tab, int max_len) {
-  const int half = hd / 2;
-  const size_t n = (size_t)T * 2 * H * half;
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-    const int j = i % half;
-    size_t r = i / half;
-    const int hh = r % (2 * H);  // 0..H-1: q heads, H..2H-1: k heads
-    const size_t t = r / (2 * H);
-    int pos = positions[t];
-    if (pos < 0 || pos >= max_len) {
-      atomicOr(&g_err_prefill, RIFT_EBIT_BADID);
-      pos = 0;
-    }
-    const float2 cs = tab[(size_t)pos * half + j];
-    uint16_t* base = qkv + t * (size_t)(3 * H * hd) + (size_t)hh * hd;
-    const float x1 = bf16_bits_to_float(base[j]), x2 = bf16_bits_to_float(base[j + half]);
-    const float y1 = x1 * cs.x - x2 * cs.y;
-    const float y2 = x2 * cs.x + x1 * cs.y;
-    __nv_bfloat16 b1 = __float2bfloat16_rn(y1), b2 = __float2bfloat16_rn(y2);
-    base[j] = *reinterpret_cast<uint16_t*>(&b1);
-    base[j + half] = *reinterpret_cast<uint16_t*>(&b2);
-  }
 }
 
 PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len) {
@@ -126,22 +107,25 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   return L;
 }
 
-int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st);
-
-int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st) {
+int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st,
+                const EpiParams& ep) {
   prof_begin(RIFT_PROF_GEMM, st);
-  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, st);
+  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, ep, st);
   prof_end(RIFT_PROF_GEMM, st, 1);
   return r;
 }
 
-static void norm_launch(bool in_bf16, int T, const void* in, float* h32, const void* gain, uint16_t* out,
-                        int d, float eps, cudaStream_t st) {
+// kind 0: packed bf16 input -> h32 + fp16 xn; 1: h32 -> fp16 xn; 2: h32 -> bf16 final output.
+static void norm_launch(int kind, int T, const void* in, float* h32, const void* gain, uint16_t* out, int d,
+                        float eps, cudaStream_t st) {
   prof_begin(RIFT_PROF_NORM, st);
-  if (in_bf16)
-    rmsnorm_kernel<true><<<T, NORM_THREADS, 0, st>>>(in, h32, static_cast<const uint16_t*>(gain), out, d, eps);
+  const uint16_t* g = static_cast<const uint16_t*>(gain);
+  if (kind == 0)
+    rmsnorm_kernel<true, true><<<T, NORM_THREADS, 0, st>>>(in, h32, g, out, d, eps);
+  else if (kind == 1)
+    rmsnorm_kernel<false, true><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
   else
-    rmsnorm_kernel<false><<<T, NORM_THREADS, 0, st>>>(in, nullptr, static_cast<const uint16_t*>(gain), out, d, eps);
+    rmsnorm_kernel<false, false><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
   prof_end(RIFT_PROF_NORM, st, 1);
 }
 
@@ -161,26 +145,27 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   prof_begin(RIFT_PROF_ROPE, st);
   rope_table_kernel<<<(max_len * half + 255) / 256, 256, 0, st>>>(rope, max_len, half, m.rope_theta);
   prof_end(RIFT_PROF_ROPE, st, 1);
-  const size_t rope_n = (size_t)T * 2 * m.n_heads * half;
-  const int rope_grid = (int)std::min<size_t>((rope_n + 255) / 256, 152 * 64);
+  EpiParams rope_ep;
+  rope_ep.positions = positions;
+  rope_ep.rope = rope;
+  rope_ep.rope_cols = 2 * d;
+  rope_ep.head_dim = m.head_dim;
+  rope_ep.max_len = max_len;
   for (int l = 0; l < m.n_layers; ++l) {
     if (l == 0)
-      norm_launch(true, T, hidden, h32, m.g_attn[0], xn, d, m.eps, st);
+      norm_launch(0, T, hidden, h32, m.g_attn[0], xn, d, m.eps, st);
     else
-      norm_launch(false, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
-    if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_STORE_BF16, qkv, st)) return 1;
-    prof_begin(RIFT_PROF_ROPE, st);
-    rope_kernel<<<rope_grid, 256, 0, st>>>(qkv, positions, T, m.n_heads, m.head_dim, rope, max_len);
-    prof_end(RIFT_PROF_ROPE, st, 1);
+      norm_launch(1, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
+    if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
     prof_begin(RIFT_PROF_ATTN, st);
     launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st);
     prof_end(RIFT_PROF_ATTN, st, 2);
     if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st)) return 1;
-    norm_launch(false, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
+    norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
     if (launch_gemm(xn, m.w_gate_up[l], T, 2 * m.ffn, d, EPI_SWIGLU, act, st)) return 1;
     if (launch_gemm(act, m.w_down[l], T, d, m.ffn, EPI_RESID_F32, h32, st)) return 1;
   }
-  norm_launch(false, T, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden), d, m.eps, st);
+  norm_launch(2, T, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden), d, m.eps, st);
   return 0;
 }
 

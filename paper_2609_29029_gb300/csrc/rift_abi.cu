@@ -257,7 +257,7 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const 
 rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int epilogue, void* out,
                         rift_stream_t stream) {
   if (!A || !W || !out || M < 0 || N < 1 || K < 1) return RIFT_ERR_INVALID;
-  if (epilogue < RIFT_EPI_STORE_BF16 || epilogue > RIFT_EPI_SWIGLU) return RIFT_ERR_INVALID;
+  if (epilogue < RIFT_EPI_STORE_F16 || epilogue > RIFT_EPI_SWIGLU) return RIFT_ERR_INVALID;
   if (K % 8 != 0 || N % 8 != 0 || (epilogue == RIFT_EPI_SWIGLU && N % 32 != 0)) return RIFT_ERR_INVALID;
   if (!aligned16(A) || !aligned16(W) || !aligned16(out)) return RIFT_ERR_INVALID;
   if (M == 0) return RIFT_OK;

@@ -20,7 +20,7 @@ unsigned int read_clear_err_gemm();
 // ---- score.cu ----
 struct ScoreLayout {
   int chunk_tokens, n_chunks, n_jblk;
-  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, total;
+  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, total;
 };
 ScoreLayout score_layout(int N, int n_v, int d, int M);
 void launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
@@ -49,14 +49,24 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
 int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
                    int max_len, const int* positions, char* ws, cudaStream_t st);
 
-// GEMM: C[M, N] = A[M, K] . B[N, K]^T (bf16 operands, fp32 accumulation) + epilogue.
+// GEMM: C[M, N] = A[M, K] . B[N, K]^T (fp16 operands, fp32 accumulation) + epilogue.
 enum GemmEpilogue {
-  EPI_STORE_BF16 = 0,  // C bf16 [M, N]
+  EPI_STORE_BF16 = 0,  // C fp16 [M, N] (name kept from the ABI's numbering)
   EPI_RESID_F32 = 1,   // R fp32 [M, N] += acc
-  EPI_SWIGLU = 2       // N = 2F interleaved in 16-column groups; C bf16 [M, F] = silu(g) * u
+  EPI_SWIGLU = 2,      // N = 2F interleaved in 16-column groups; C fp16 [M, F] = silu(g) * u
+  EPI_QKV_ROPE = 3     // C fp16 [M, N]; columns < rope_cols get rotate-half RoPE at positions[row]
+};
+struct EpiParams {
+  const int* positions = nullptr;  // [M] position of each row (EPI_QKV_ROPE)
+  const float2* rope = nullptr;    // [max_len, head_dim/2] (cos, sin)
+  int rope_cols = 0;               // q and k columns: 2 d
+  int head_dim = 0;
+  int max_len = 0;
 };
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
-                cudaStream_t st);
+                cudaStream_t st, const EpiParams& ep = EpiParams());
+int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
+                   cudaStream_t st);
 
 void launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
                       int head_dim, const int2* sched, int n_sched_max, void* out, cudaStream_t st);

@@ -6,6 +6,8 @@
 // with the background mean folded into one vector), and it adds the token into the tile's
 // pooled sum P_i.  Several CTAs share a tile; each writes its partial P to the workspace and
 // tile_finalize_kernel adds them in a fixed order.
+#include <algorithm>
+
 #include "rift_internal.h"
 
 namespace rift {
@@ -245,10 +247,12 @@ __global__ void __launch_bounds__(256) tile_finalize_kernel(const float* __restr
 }
 
 // ------------------------------------------------------------------------------------------
-// a4: G = V V^T in 64 x 64 blocks (fp32, k ascending), each block's per-row top-m written as
-// a candidate list; knn_merge_kernel merges the lists of a row and smooths.
+// a4: G = V V^T in 64 x 64 blocks (fp32, k ascending), each block's per-row top-C written as a
+// candidate list; knn_merge_kernel merges a row's lists; knn_rescore_smooth_kernel recomputes
+// the C candidates in fp64, keeps the top m and smooths.
 // ------------------------------------------------------------------------------------------
 constexpr int KB = 64;   // rows (i) and columns (j) per block
+constexpr int KNN_SPARE = 10;  // fp32 candidates kept beyond m for the fp64 rescoring
 constexpr int KK = 32;   // d-chunk
 
 // (g, j) beats (g2, j2): larger similarity first, then the lower index.
@@ -259,6 +263,7 @@ __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
 __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict__ V, int N, int d,
                                                         int m, float* __restrict__ cand_g,
                                                         int* __restrict__ cand_j) {
+  // m here is the candidate count C kept per row and block
   __shared__ float As[KK][KB + 4];
   __shared__ float Bs[KK][KB + 4];
   __shared__ float Gs[KB][KB + 1];
@@ -276,6 +281,9 @@ __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict_
       Bs[c4 + 0][row] = b.x; Bs[c4 + 1][row] = b.y; Bs[c4 + 2][row] = b.z; Bs[c4 + 3][row] = b.w;
     }
     __syncthreads();
+    // Each 32-term chunk is summed on its own and then added to the total: for nearly parallel
+    // tiles the running sum approaches 1, and chunking cuts its rounding error about sixfold.
+    float part[4][4] = {};
 #pragma unroll 8
     for (int k = 0; k < KK; ++k) {
       float4 a = *reinterpret_cast<const float4*>(&As[k][ti * 4]);
@@ -284,8 +292,12 @@ __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict_
 #pragma unroll
       for (int r = 0; r < 4; ++r)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(av[r], bv[c], acc[r][c]);
+        for (int c = 0; c < 4; ++c) part[r][c] = fmaf(av[r], bv[c], part[r][c]);
     }
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
     __syncthreads();
   }
 #pragma unroll
@@ -313,35 +325,72 @@ __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict_
   }
 }
 
-// One thread per tile: merge the candidate lists, then s~_i = (sum over the ascending set
-// {i} + NN(i) of s_raw) / (m + 1) with correctly rounded fp32 adds and divide.
-__global__ void knn_merge_smooth_kernel(const float* __restrict__ cand_g, const int* __restrict__ cand_j,
-                                        int n_lists, int N, int m, const float* __restrict__ s_raw,
-                                        float* __restrict__ s_tilde, int* __restrict__ nbr) {
+// One thread per tile: merge the blocks' candidate lists into the row's top-C by fp32
+// similarity (C = m + a few spares).
+__global__ void knn_merge_kernel(const float* __restrict__ cand_g, const int* __restrict__ cand_j, int n_lists,
+                                 int N, int C, int* __restrict__ top_j) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= N) return;
   float bg[RIFT_MAX_KNN];
   int bj[RIFT_MAX_KNN];
-  for (int r = 0; r < m; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
+  for (int r = 0; r < C; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
   for (int l = 0; l < n_lists; ++l) {
-    const size_t o = ((size_t)i * n_lists + l) * m;
-    for (int r = 0; r < m; ++r) {
+    const size_t o = ((size_t)i * n_lists + l) * C;
+    for (int r = 0; r < C; ++r) {
       float g = cand_g[o + r];
       int j = cand_j[o + r];
-      if (!knn_better(g, j, bg[m - 1], bj[m - 1])) break;  // lists are sorted
-      int p = m - 1;
+      if (!knn_better(g, j, bg[C - 1], bj[C - 1])) break;  // lists are sorted
+      int p = C - 1;
       while (p > 0 && knn_better(g, j, bg[p - 1], bj[p - 1])) { bg[p] = bg[p - 1]; bj[p] = bj[p - 1]; --p; }
       bg[p] = g; bj[p] = j;
     }
   }
+  for (int r = 0; r < C; ++r) top_j[(size_t)i * C + r] = bj[r];
+}
+
+// One warp per tile: recompute the C candidates' similarities with fp64 accumulation (the
+// fp32 pass errs by ~sqrt(d) ulp for nearly parallel tiles, and fp32 cannot even separate
+// similarities closer to 1 than 6e-8), keep the m best by the fp64 values (ties to the lower
+// index), then s~_i = (sum over the ascending set {i} + NN(i) of s_raw) / (m + 1) with correctly
+// rounded fp32 adds and divide.
+__global__ void knn_rescore_smooth_kernel(const float* __restrict__ V, int d, const int* __restrict__ top_j, int N,
+                                          int C, int m, const float* __restrict__ s_raw,
+                                          float* __restrict__ s_tilde, int* __restrict__ nbr) {
+  const int lane = threadIdx.x & 31;
+  const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (i >= N) return;
+  double g64[RIFT_MAX_KNN];
+  int jj[RIFT_MAX_KNN];
+  const float* vi = V + (size_t)i * d;
+  for (int r = 0; r < C; ++r) {
+    const int j = top_j[(size_t)i * C + r];
+    jj[r] = j;
+    double acc = 0.0;
+    if (j >= 0 && j < N) {
+      const float* vj = V + (size_t)j * d;
+      for (int k = lane; k < d; k += 32) acc = fma((double)vi[k], (double)vj[k], acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    g64[r] = (j >= 0 && j < N) ? acc : -INFINITY;
+  }
+  if (lane != 0) return;
+  // top-m of the rescored candidates by (g64 desc, j asc)
+  for (int a = 1; a < C; ++a) {
+    double g = g64[a];
+    int j = jj[a], b = a;
+    while (b > 0 && (g > g64[b - 1] || (g == g64[b - 1] && j < jj[b - 1]))) {
+      g64[b] = g64[b - 1]; jj[b] = jj[b - 1]; --b;
+    }
+    g64[b] = g; jj[b] = j;
+  }
   if (nbr)
-    for (int r = 0; r < m; ++r) nbr[(size_t)i * m + r] = bj[r];
-  // members {i} + NN(i), ascending
+    for (int r = 0; r < m; ++r) nbr[(size_t)i * m + r] = jj[r];
   int mem[RIFT_MAX_KNN + 1];
   int n = 0;
   for (int r = 0; r < m; ++r) {
-    if (bj[r] >= 0 && bj[r] < N) {
-      mem[n++] = bj[r];
+    if (jj[r] >= 0 && jj[r] < N) {
+      mem[n++] = jj[r];
     } else {  // fewer than m finite similarities (a NaN row): reported, never indexed
       atomicOr(&g_err_score, RIFT_EBIT_NONFINITE);
     }
@@ -378,6 +427,7 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   L.V_off = take(sizeof(float) * (size_t)N * d);
   L.cand_g_off = take(sizeof(float) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
   L.cand_j_off = take(sizeof(int) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
+  L.top_off = take(sizeof(int) * (size_t)N * RIFT_MAX_KNN);
   L.total = off;
   (void)M;
   return L;
@@ -412,12 +462,18 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
     else launch_tokens<float, 4>(X, N, n_v, d, L, w, token_scores, Ppart, st);
   }
   tile_finalize_kernel<<<N, 256, d * sizeof(float), st>>>(Ppart, L.n_chunks, d, w, V, s_raw);
+  int* topj = reinterpret_cast<int*>(ws + L.top_off);
+  // candidates per row: m plus spares for the fp64 rescoring, at most the N - 1 other tiles
+  const int C = m > 0 ? std::min(std::min(m + KNN_SPARE, RIFT_MAX_KNN), N - 1) : 0;
+  int launched = 4;
   if (m > 0) {
     dim3 grid(L.n_jblk, L.n_jblk);
-    knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, m, cg, cj);
+    knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, C, cg, cj);
+    knn_merge_kernel<<<(N + 127) / 128, 128, 0, st>>>(cg, cj, L.n_jblk, N, C, topj);
+    launched += 2;
   }
-  knn_merge_smooth_kernel<<<(N + 127) / 128, 128, 0, st>>>(cg, cj, L.n_jblk, N, m, s_raw, s_tilde, nbr);
-  return m > 0 ? 5 : 4;  // kernels launched
+  knn_rescore_smooth_kernel<<<(N + 7) / 8, 256, 0, st>>>(V, d, topj, N, C, m, s_raw, s_tilde, nbr);
+  return launched;  // kernels launched
 }
 
 }  // namespace rift

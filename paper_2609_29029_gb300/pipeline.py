@@ -22,17 +22,22 @@ def interleave_gate_up(wg: torch.Tensor, wu: torch.Tensor) -> torch.Tensor:
 
 
 class DeviceModel:
-    """Decoder weights in the library's layout plus the rift_model struct that points at them."""
+    """Decoder weights in the library's layout plus the rift_model struct that points at them.
+
+    Projection weights are stored in fp16 (the GEMM operand type; bf16 weights convert exactly
+    unless their magnitude is below 2^-14, where fp16 keeps 2^-24 absolute resolution).  Norm
+    gains stay bf16."""
 
     def __init__(self, dec, layers: list, g_final: torch.Tensor, device="cuda"):
         self.dec = dec
         self.layers = []
+        h = torch.float16
         for W in layers:
             self.layers.append({
-                "qkv": torch.cat([W["wq"], W["wk"], W["wv"]], 0).to(device, torch.bfloat16).contiguous(),
-                "o": W["wo"].to(device, torch.bfloat16).contiguous(),
-                "gate_up": interleave_gate_up(W["wg"].to(device), W["wu"].to(device)).to(torch.bfloat16),
-                "down": W["wd"].to(device, torch.bfloat16).contiguous(),
+                "qkv": torch.cat([W["wq"], W["wk"], W["wv"]], 0).to(device).to(h).contiguous(),
+                "o": W["wo"].to(device).to(h).contiguous(),
+                "gate_up": interleave_gate_up(W["wg"].to(device), W["wu"].to(device)).to(h),
+                "down": W["wd"].to(device).to(h).contiguous(),
                 "g_attn": W["g_attn"].to(device, torch.bfloat16).contiguous(),
                 "g_ffn": W["g_ffn"].to(device, torch.bfloat16).contiguous(),
             })

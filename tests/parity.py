@@ -52,25 +52,48 @@ def oracle_select(wl, sc, p_ext=None):
     return O.select(sc.X, sc.embed, sc.query_ids, sc.bg_ids, wl.knn_m, wl.policy, p_ext=p_ext)
 
 
-DECISION_EPS = 1e-5  # relative bound on the fp32 score difference that a decision must clear
+# Bounds on |CUDA fp32 value - oracle fp32 value| of the quantities that decide integers.
+#  * similarity G (compared in fp64 on both sides): the CUDA path recomputes its kNN candidates
+#    with fp64 accumulation of the fp32 tile embeddings, whose elements carry ~1e-7 relative error
+#    from the fp32 pooled sums; in a 4096-term dot product that averages to ~3e-9; bound 3e-8.
+#  * tile score, utility: fp32 dot products whose running sums cancel: ~1e-7; bounds 1e-6.
+#  * token score r = x.w / ||x||: ~5e-9 absolute; bound 2e-6 of the tile's largest |r|.
+EPS_G = 3e-8        # cosine similarity of two tiles (|G| <= 1)
+EPS_S = 1e-6        # tile score, relative to max |s~| over the scene
+EPS_U = 1e-6        # utility U(c) (|dU/dp| <= 0.4, p = u)
+EPS_R = 2e-6        # token score, relative to max |r| over the tile
+
+# Seeds whose scene has every kNN / threshold / budget decision clear of its bound.  Seed 0 of the
+# 1600-tile scene has a kNN gap of 1.3e-8 and a kept tile whose p = 0.8903232 is one of the 11
+# fp32 values in [0.37, 1] where two utilities of the lambda = 0.10 table are equal; seed 3 clears
+# every bound (its remaining top-b near-ties are checked for validity).
+PARITY_SEED = {"rift1600_7b": 3}
+
+
+def parity_workload(wl):
+    seed = PARITY_SEED.get(wl.name, wl.scene.seed)
+    return replace(wl, scene=replace(wl.scene, seed=seed))
 
 
 def margins(sel: O.Selection, wl) -> dict:
-    """The oracle's smallest margin of each kind of decision, in units of the bound on the
-    CUDA/oracle score difference (>= 1 means the decision is unique at fp32 precision)."""
+    """The oracle's smallest margin of each kind of decision, in units of its bound (>= 1: the
+    decision is unique at the precision the CUDA path reaches).  'topb_tiles' lists the kept
+    slots whose rank-b gap is below its bound."""
     out = {}
     N = len(sel.s32)
     m = min(wl.knn_m, N - 1)
     worst = np.inf
     if 0 < m < N - 1:
         for i in range(N):
-            g = np.sort(np.delete(sel.G32[i].astype(np.float64), i))[::-1]
-            worst = min(worst, (g[m - 1] - g[m]) / DECISION_EPS)
+            g = np.sort(np.delete(sel.G[i].astype(np.float64), i))[::-1]
+            worst = min(worst, (g[m - 1] - g[m]) / EPS_G)
     out["knn"] = worst
     st = sel.s_tilde.astype(np.float64)
     span = st.max() - st.min()
-    if span > 0:
-        du = 3 * DECISION_EPS * np.abs(st).max() / span
+    if wl.policy.tau <= 0.0:
+        out["tau"] = np.inf  # u >= 0 holds exactly (s~ - min >= 0), so nothing can flip
+    elif span > 0:
+        du = 3 * EPS_S * np.abs(st).max() / span
         out["tau"] = float(np.min(np.abs(sel.u.astype(np.float64) - float(F32(wl.policy.tau)))) / du)
     else:
         out["tau"] = np.inf
@@ -78,21 +101,58 @@ def margins(sel: O.Selection, wl) -> dict:
     for p in sel.p:
         U = sorted([float(x) for x in O.utility(float(p), wl.policy)], reverse=True)
         if len(U) > 1:
-            wb = min(wb, (U[0] - U[1]) / DECISION_EPS)
+            wb = min(wb, (U[0] - U[1]) / EPS_U)
     out["budget"] = wb
-    wt = np.inf
-    for i, b in zip(sel.kept, sel.budgets):
+    wt, amb = np.inf, []
+    for j, (i, b) in enumerate(zip(sel.kept, sel.budgets)):
         r = np.sort(sel.r32[i].astype(np.float64))[::-1]
         if b < len(r):
-            wt = min(wt, (r[b - 1] - r[b]) / (DECISION_EPS * np.abs(r).max()))
+            mj = (r[b - 1] - r[b]) / (EPS_R * np.abs(r).max())
+            wt = min(wt, mj)
+            if mj < 1.0:
+                amb.append(j)
     out["topb"] = wt
+    out["topb_tiles"] = amb
     return out
 
 
-def assert_margins(sel, wl):
+def assert_margins(sel, wl, allow_topb=False):
+    """Every kNN, threshold and budget decision must clear its bound; top-b decisions too unless
+    allow_topb (then the ambiguous slots are returned and checked for validity instead)."""
     mg = margins(sel, wl)
-    bad = {k: v for k, v in mg.items() if not v >= 1.0}
+    keys = ["knn", "tau", "budget"] + ([] if allow_topb else ["topb"])
+    bad = {k: mg[k] for k in keys if not mg[k] >= 1.0}
     assert not bad, f"seeded input has decisions closer than the fp32 bound: {bad}"
+    return set(mg["topb_tiles"])
+
+
+def topb_is_valid(gpu_idx, r32_tile, b):
+    """A selection that differs from the oracle's only inside the fp32 bound of the boundary:
+    b indices, ascending, every token clearly above the b-th score taken, none clearly below."""
+    r = np.asarray(r32_tile, dtype=np.float64)
+    if len(gpu_idx) != b or list(gpu_idx) != sorted(set(gpu_idx)):
+        return False
+    vb = np.sort(r)[::-1][b - 1]
+    eps = EPS_R * np.abs(r).max()
+    chosen = set(gpu_idx)
+    must = {k for k in range(len(r)) if r[k] > vb + eps}
+    never = {k for k in range(len(r)) if r[k] < vb - eps}
+    return must <= chosen and not (chosen & never)
+
+
+def neighbours_match(gpu_nbr, sel) -> list:
+    """Rows whose neighbour SET differs from the oracle's (the set is what the smoothing uses),
+    plus rows whose emitted rank order contradicts the oracle's similarities by more than the
+    bound.  Equal sets with a swapped near-tie (|dG| < EPS_G) are accepted."""
+    bad = []
+    for i in range(len(gpu_nbr)):
+        g = [int(j) for j in gpu_nbr[i]]
+        if sorted(g) != sorted(int(j) for j in sel.nbr[i]):
+            bad.append(i)
+            continue
+        if any(sel.G[i, g[k]] < sel.G[i, g[k + 1]] - EPS_G for k in range(len(g) - 1)):
+            bad.append(i)
+    return bad
 
 
 def rel_err_rows(g: np.ndarray, o: np.ndarray) -> float:
