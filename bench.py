@@ -385,7 +385,7 @@ def main():
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16", "data": "synthetic",
+        "dtype": "f16", "data": "synthetic",
         "config": {"workload": wl.name, "tiles": s.N, "tokens_per_tile": s.n_v, "d": s.d,
                    "decoder": f"{dec.n_layers}x{dec.d} LLaMA/Vicuna-7B shape, random init",
                    "kept_tiles": n_kept, "retained_tokens_T": T,
