@@ -244,6 +244,23 @@ def run_reference(args, wl, ws, rank):
 
 # ------------------------------------------------------------------------------------------ main arm
 
+def gemm_traffic():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if it was taken on the current
+    gemm_tc.cu (source hash match); otherwise None."""
+    import hashlib
+    import re
+    prof = ROOT / "profiles" / "launches_rift400_7b.md"
+    src = ROOT / "paper_2609_29029_gb300" / "csrc" / "gemm_tc.cu"
+    if not prof.exists() or not src.exists():
+        return None
+    text = prof.read_text()
+    h = re.search(r"source_sha256_16: ([0-9a-f]{16})", text)
+    b = re.search(r"dram_bytes_per_launch: (\d+)", text)
+    if not h or not b or hashlib.sha256(src.read_bytes()).hexdigest()[:16] != h.group(1):
+        return None
+    return int(b.group(1))
+
+
 def kernel_case(name: str):
     """Small cases for ncu captures: inputs larger than L2, about 1 GB on the device."""
     import __graft_entry__
@@ -371,7 +388,7 @@ def main():
     gemm_ms, gemm_n = prof["gemm"]
     gemm_flops = args.steps * T * dec.linear_flops_per_token
     achieved = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
-    traffic = None
+    traffic = gemm_traffic()
     per_step = {k: round(v[0] / args.steps, 3) for k, v in prof.items()}
     sel_ms = (prof["score"][0] + prof["select"][0] + prof["pack"][0]) / args.steps
 

@@ -221,11 +221,15 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const uint16_t* __restric
 
 }  // namespace attn
 
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st) {
+  attn::schedule_kernel<<<1, 1024, 0, st>>>(cu_seqlens, n_seq, sched, n_sched_max);
+}
+
 void launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
                       int head_dim, const int2* sched, int n_sched_max, void* out, cudaStream_t st) {
   using namespace attn;
   (void)T;
-  schedule_kernel<<<1, 1024, 0, st>>>(cu_seqlens, n_seq, const_cast<int2*>(sched), n_sched_max);
+  (void)n_seq;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
   dim3 grid(n_sched_max, n_heads);
   if (head_dim == 128) {

@@ -10,7 +10,8 @@
 //               into one of two 256-column fp32 accumulators and commits to mbarriers
 //   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes (one row per thread), fused op, store
 // Two accumulators let the epilogue of one tile overlap the main loop of the next.  Tiles are
-// visited in bands of 16 M-tiles so a band's A rows and the current B tiles stay in L2.
+// visited in bands of M-tiles whose A rows fit in L2 (48 MB), so each weight tile is read from
+// DRAM once per band.
 // Every mbarrier wait is bounded (RIFT_SPIN_LIMIT iterations, ~4 s of globaltimer): on timeout
 // the kernel sets RIFT_EBIT_TIMEOUT, lets every role fall through, waits for its issued copies
 // and frees its tensor memory.
@@ -41,7 +42,6 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 192;
 constexpr int ACC_COLS = BN;        // fp32 accumulator columns per buffer
 constexpr int TMEM_COLS = 2 * ACC_COLS;
-constexpr int GROUP_M = 16;
 constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
 
 // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A fp16 (bits 7-9 = 0), B fp16
@@ -136,11 +136,11 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int& m_blk, int& n_blk) {
-  const int per_group = GROUP_M * nt;
+__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int group_m, int& m_blk, int& n_blk) {
+  const int per_group = group_m * nt;
   const int grp = tile / per_group;
-  const int first_m = grp * GROUP_M;
-  const int gsz = min(mt - first_m, GROUP_M);
+  const int first_m = grp * group_m;
+  const int gsz = min(mt - first_m, group_m);
   const int r = tile - grp * per_group;
   m_blk = first_m + r % gsz;
   n_blk = r / gsz;
@@ -231,7 +231,7 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, void* C, const EpiParams ep) {
+                   int K, void* C, const EpiParams ep, int group_m) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -280,7 +280,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
         int m_blk, n_blk;
-        tile_coords(tile, mt, nt, m_blk, n_blk);
+        tile_coords(tile, mt, nt, group_m, m_blk, n_blk);
         for (int k = 0; k < kt; ++k, ++it) {
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     int tl = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++tl) {
       int m_blk, n_blk;
-      tile_coords(tile, mt, nt, m_blk, n_blk);
+      tile_coords(tile, mt, nt, group_m, m_blk, n_blk);
       const int b = tl & 1;
       const uint32_t use = tl >> 1;
       if (!mbar_wait(tfull_bar(b), use & 1u, abort_flag)) break;
@@ -430,7 +430,11 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   }
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = tiles < sm_count() ? tiles : sm_count();
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep);
+  // Band height: as many M-tiles as keep the band's A rows within ~48 MB of L2 (8..64), so each
+  // weight tile is streamed from DRAM once per band.
+  int group_m = (int)((48u << 20) / ((size_t)BM * K * 2));
+  group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep, group_m);
   return 0;
 }
 

@@ -145,6 +145,9 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   prof_begin(RIFT_PROF_ROPE, st);
   rope_table_kernel<<<(max_len * half + 255) / 256, 256, 0, st>>>(rope, max_len, half, m.rope_theta);
   prof_end(RIFT_PROF_ROPE, st, 1);
+  prof_begin(RIFT_PROF_ATTN, st);
+  launch_attention_schedule(cu_seqlens, n_seq, sched, L.max_qblocks, st);
+  prof_end(RIFT_PROF_ATTN, st, 1);
   EpiParams rope_ep;
   rope_ep.positions = positions;
   rope_ep.rope = rope;
@@ -159,7 +162,7 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
     if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
     prof_begin(RIFT_PROF_ATTN, st);
     launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st);
-    prof_end(RIFT_PROF_ATTN, st, 2);
+    prof_end(RIFT_PROF_ATTN, st, 1);
     if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st)) return 1;
     norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
     if (launch_gemm(xn, m.w_gate_up[l], T, 2 * m.ffn, d, EPI_SWIGLU, act, st)) return 1;

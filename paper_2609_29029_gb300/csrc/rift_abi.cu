@@ -133,9 +133,9 @@ rift_status rift_query_prep(const void* embed, int vocab, int d, const int* phra
       n_phrase < 1 || M < 0 || M > 64 || (M > 0 && (!bg_ids || !B)))
     return RIFT_ERR_INVALID;
   prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
-  launch_query_prep(embed, vocab, d, phrase_ids, n_templates, n_phrase, bg_ids, M, t, B,
-                    static_cast<cudaStream_t>(stream));
-  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), 1);
+  const int nk = launch_query_prep(embed, vocab, d, phrase_ids, n_templates, n_phrase, bg_ids, M, t, B,
+                                   static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }

@@ -19,12 +19,12 @@ unsigned int read_clear_err_gemm();
 
 // ---- score.cu ----
 struct ScoreLayout {
-  int chunk_tokens, n_chunks, n_jblk;
-  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, total;
+  int chunk_tokens, n_chunks, n_jblk, n_split;
+  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, gpart_off, total;
 };
 ScoreLayout score_layout(int N, int n_v, int d, int M);
-void launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
-                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st);
+int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
+                      int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st);
 int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
                  int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
                  cudaStream_t st);
@@ -68,6 +68,8 @@ int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
                    cudaStream_t st);
 
+// q-block schedule of the varlen attention (built once per prefill from cu_seqlens)
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st);
 void launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
                       int head_dim, const int2* sched, int n_sched_max, void* out, cudaStream_t st);
 

@@ -78,6 +78,44 @@ __global__ void __launch_bounds__(256) query_prep_kernel(const uint16_t* __restr
   }
 }
 
+// One caption template: rows are plain means / copies, so every column is independent.  One
+// thread per column writes the unnormalised query row into t and the background rows into B;
+// normalize_rows_kernel then scales each row to unit length (one CTA per row).
+__global__ void query_rows_kernel(const uint16_t* __restrict__ embed, int vocab, int d,
+                                  const int* __restrict__ phrase_ids, int n_phrase,
+                                  const int* __restrict__ bg_ids, int M, float* __restrict__ t,
+                                  float* __restrict__ B) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= d) return;
+  float s = 0.f;
+  for (int q = 0; q < n_phrase; ++q) {
+    const int id = phrase_ids[q];
+    if (id < 0 || id >= vocab) {
+      atomicOr(&g_err_score, RIFT_EBIT_BADID);
+      continue;
+    }
+    s += bf16_bits_to_float(embed[(size_t)id * d + c]);
+  }
+  t[c] = s / (float)n_phrase;
+  for (int j = 0; j < M; ++j) {
+    const int id = bg_ids[j];
+    const bool ok = id >= 0 && id < vocab;
+    if (!ok && c == 0) atomicOr(&g_err_score, RIFT_EBIT_BADID);
+    B[(size_t)j * d + c] = ok ? bf16_bits_to_float(embed[(size_t)id * d + c]) : 0.f;
+  }
+}
+
+// Row r of {t, B_0, ..., B_{M-1}} divided by its length (zero rows stay zero).
+__global__ void __launch_bounds__(256) normalize_rows_kernel(float* __restrict__ t, float* __restrict__ B, int d) {
+  __shared__ float red[32];
+  float* row = blockIdx.x == 0 ? t : B + (size_t)(blockIdx.x - 1) * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += row[c] * row[c];
+  const float tot = block_sum(ss, red);
+  const float inv = tot > 0.f ? 1.f / sqrtf(tot) : 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) row[c] *= inv;
+}
+
 // w = t - (1/M) sum_j B_j  (M = 0: w = t)
 __global__ void fold_w_kernel(const float* __restrict__ t, const float* __restrict__ B, int M,
                               int d, float* __restrict__ w) {
@@ -247,9 +285,11 @@ __global__ void __launch_bounds__(256) tile_finalize_kernel(const float* __restr
 }
 
 // ------------------------------------------------------------------------------------------
-// a4: G = V V^T in 64 x 64 blocks (fp32, k ascending), each block's per-row top-C written as a
-// candidate list; knn_merge_kernel merges a row's lists; knn_rescore_smooth_kernel recomputes
-// the C candidates in fp64, keeps the top m and smooths.
+// a4: G = V V^T in 64 x 64 blocks (fp32, k ascending, 32-term chunks).  Small scenes split K
+// across CTAs and knn_row_topc_kernel picks each row's top-C from the summed slices; large ones
+// keep a top-C list per block and knn_merge_kernel merges a row's lists.  Then
+// knn_rescore_smooth_kernel recomputes the C candidates to ~fp64 accuracy, keeps the top m and
+// smooths.
 // ------------------------------------------------------------------------------------------
 constexpr int KB = 64;   // rows (i) and columns (j) per block
 constexpr int KNN_SPARE = 10;  // fp32 candidates kept beyond m for the fp64 rescoring
@@ -260,17 +300,22 @@ __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
   return g > g2 || (g == g2 && j < j2);
 }
 
+// grid (column blocks, row blocks, K slices).  With one slice the kernel also extracts each
+// row's top-C of the block (m here is C); with several it writes its partial similarities to
+// Gpart[slice][i][j] for knn_row_topc_kernel.
 __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict__ V, int N, int d,
                                                         int m, float* __restrict__ cand_g,
-                                                        int* __restrict__ cand_j) {
-  // m here is the candidate count C kept per row and block
+                                                        int* __restrict__ cand_j,
+                                                        float* __restrict__ Gpart) {
   __shared__ float As[KK][KB + 4];
   __shared__ float Bs[KK][KB + 4];
   __shared__ float Gs[KB][KB + 1];
   const int i0 = blockIdx.y * KB, j0 = blockIdx.x * KB;
   const int tid = threadIdx.x, ti = tid >> 4, tj = tid & 15;
+  const int kslice = d / gridDim.z;
+  const int kbeg = blockIdx.z * kslice, kend = kbeg + kslice;
   float acc[4][4] = {};
-  for (int k0 = 0; k0 < d; k0 += KK) {
+  for (int k0 = kbeg; k0 < kend; k0 += KK) {
     // 64 rows x 32 floats per operand = 512 float4; two per thread.
     for (int q = tid; q < KB * KK / 4; q += 256) {
       int row = q >> 3, c4 = (q & 7) * 4;
@@ -300,6 +345,16 @@ __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict_
       for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
     __syncthreads();
   }
+  if (gridDim.z > 1) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int i = i0 + ti * 4 + r, j = j0 + tj * 4 + c;
+        if (i < N && j < N) Gpart[((size_t)blockIdx.z * N + i) * N + j] = acc[r][c];
+      }
+    return;
+  }
 #pragma unroll
   for (int r = 0; r < 4; ++r)
 #pragma unroll
@@ -322,6 +377,41 @@ __global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict_
     }
     const size_t o = ((size_t)i * gridDim.x + blockIdx.x) * m;
     for (int r = 0; r < m; ++r) { cand_g[o + r] = bg[r]; cand_j[o + r] = bj[r]; }
+  }
+}
+
+// After a split-K Gram pass (N <= 1024): one warp per row sums the slices in slice order for
+// every column and extracts the row's top-C directly (C rounds of a warp-wide argmax, larger
+// similarity first, then the lower index).
+constexpr int RT_WARPS = 4;
+__global__ void __launch_bounds__(32 * RT_WARPS) knn_row_topc_kernel(const float* __restrict__ Gpart, int n_split,
+                                                                      int N, int C, int* __restrict__ top_j) {
+  __shared__ float gs[RT_WARPS][1024];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * RT_WARPS + w;
+  if (i >= N) return;
+  float* g = gs[w];
+  for (int j = lane; j < N; j += 32) {
+    float v = 0.f;
+    for (int z = 0; z < n_split; ++z) v += Gpart[((size_t)z * N + i) * N + j];
+    if (!(v == v)) { atomicOr(&g_err_score, RIFT_EBIT_NONFINITE); v = -INFINITY; }
+    g[j] = (j == i) ? -INFINITY : v;
+  }
+  __syncwarp();
+  for (int r = 0; r < C; ++r) {
+    float bv = -INFINITY;
+    int bj = 0x7fffffff;
+    for (int j = lane; j < N; j += 32)
+      if (knn_better(g[j], j, bv, bj)) { bv = g[j]; bj = j; }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+      if (knn_better(ov, oj, bv, bj)) { bv = ov; bj = oj; }
+    }
+    if (lane == 0) top_j[(size_t)i * C + r] = (bv == -INFINITY) ? 0x7fffffff : bj;
+    if (bj >= 0 && bj < N && (bj & 31) == lane) g[bj] = -INFINITY;
+    __syncwarp();
   }
 }
 
@@ -348,49 +438,67 @@ __global__ void knn_merge_kernel(const float* __restrict__ cand_g, const int* __
   for (int r = 0; r < C; ++r) top_j[(size_t)i * C + r] = bj[r];
 }
 
-// One warp per tile: recompute the C candidates' similarities with fp64 accumulation (the
-// fp32 pass errs by ~sqrt(d) ulp for nearly parallel tiles, and fp32 cannot even separate
-// similarities closer to 1 than 6e-8), keep the m best by the fp64 values (ties to the lower
-// index), then s~_i = (sum over the ascending set {i} + NN(i) of s_raw) / (m + 1) with correctly
-// rounded fp32 adds and divide.
-__global__ void knn_rescore_smooth_kernel(const float* __restrict__ V, int d, const int* __restrict__ top_j, int N,
-                                          int C, int m, const float* __restrict__ s_raw,
-                                          float* __restrict__ s_tilde, int* __restrict__ nbr) {
-  const int lane = threadIdx.x & 31;
-  const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (i >= N) return;
-  double g64[RIFT_MAX_KNN];
-  int jj[RIFT_MAX_KNN];
-  const float* vi = V + (size_t)i * d;
-  for (int r = 0; r < C; ++r) {
-    const int j = top_j[(size_t)i * C + r];
-    jj[r] = j;
-    double acc = 0.0;
+// One CTA per tile, one warp per candidate: recompute the C candidates' similarities to ~fp64
+// accuracy (the fp32 pass errs by ~sqrt(d) ulp for nearly parallel tiles, and fp32 cannot even
+// separate similarities closer to 1 than 6e-8), keep the m best by those values (ties to the
+// lower index), then s~_i = (sum over the ascending set {i} + NN(i) of s_raw) / (m + 1) with
+// correctly rounded fp32 adds and divide.
+__global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
+    const float* __restrict__ V, int d, const int* __restrict__ top_j, int N, int C, int m,
+    const float* __restrict__ s_raw, float* __restrict__ s_tilde, int* __restrict__ nbr) {
+  __shared__ double g64[RIFT_MAX_KNN];
+  __shared__ int jj[RIFT_MAX_KNN];
+  const int i = blockIdx.x;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (w < C) {
+    const int j = top_j[(size_t)i * C + w];
+    // Each lane keeps its partial sum as an unevaluated pair hi + lo of floats: the product of
+    // two floats is split exactly with an FMA (Dekker's TwoProduct as rewritten by Ogita, Rump
+    // and Oishi) and added with Knuth's TwoSum, so the lane sum is good to ~2^-44 relative.
+    float hi = 0.f, lo = 0.f;
     if (j >= 0 && j < N) {
-      const float* vj = V + (size_t)j * d;
-      for (int k = lane; k < d; k += 32) acc = fma((double)vi[k], (double)vj[k], acc);
+      const float4* vi = reinterpret_cast<const float4*>(V + (size_t)i * d);
+      const float4* vj = reinterpret_cast<const float4*>(V + (size_t)j * d);
+      for (int k = lane; k < d / 4; k += 32) {
+        const float4 a4 = vi[k], b4 = vj[k];
+        const float av[4] = {a4.x, a4.y, a4.z, a4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p = __fmul_rn(av[e], bv[e]);
+          const float pe = fmaf(av[e], bv[e], -p);
+          const float s = __fadd_rn(hi, p);
+          const float bb = __fsub_rn(s, hi);
+          const float er = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(p, bb));
+          hi = s;
+          lo = __fadd_rn(lo, __fadd_rn(er, pe));
+        }
+      }
     }
+    double acc = (double)hi + (double)lo;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    g64[r] = (j >= 0 && j < N) ? acc : -INFINITY;
+    if (lane == 0) {
+      g64[w] = (j >= 0 && j < N) ? acc : -INFINITY;
+      jj[w] = j;
+    }
   }
-  if (lane != 0) return;
-  // top-m of the rescored candidates by (g64 desc, j asc)
-  for (int a = 1; a < C; ++a) {
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+  double gl[RIFT_MAX_KNN];
+  int jl[RIFT_MAX_KNN];
+  for (int a = 0; a < C; ++a) {  // insertion into (g desc, j asc) order
     double g = g64[a];
     int j = jj[a], b = a;
-    while (b > 0 && (g > g64[b - 1] || (g == g64[b - 1] && j < jj[b - 1]))) {
-      g64[b] = g64[b - 1]; jj[b] = jj[b - 1]; --b;
-    }
-    g64[b] = g; jj[b] = j;
+    while (b > 0 && (g > gl[b - 1] || (g == gl[b - 1] && j < jl[b - 1]))) { gl[b] = gl[b - 1]; jl[b] = jl[b - 1]; --b; }
+    gl[b] = g; jl[b] = j;
   }
   if (nbr)
-    for (int r = 0; r < m; ++r) nbr[(size_t)i * m + r] = jj[r];
+    for (int r = 0; r < m; ++r) nbr[(size_t)i * m + r] = jl[r];
   int mem[RIFT_MAX_KNN + 1];
   int n = 0;
   for (int r = 0; r < m; ++r) {
-    if (jj[r] >= 0 && jj[r] < N) {
-      mem[n++] = jj[r];
+    if (jl[r] >= 0 && jl[r] < N) {
+      mem[n++] = jl[r];
     } else {  // fewer than m finite similarities (a NaN row): reported, never indexed
       atomicOr(&g_err_score, RIFT_EBIT_NONFINITE);
     }
@@ -409,10 +517,17 @@ __global__ void knn_rescore_smooth_kernel(const float* __restrict__ V, int d, co
 // ------------------------------------------------------------------------------------------
 // Launchers
 // ------------------------------------------------------------------------------------------
-void launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
-                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st) {
+int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
+                      int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st) {
+  if (n_tmpl == 1) {
+    query_rows_kernel<<<(d + 255) / 256, 256, 0, st>>>(static_cast<const uint16_t*>(embed), vocab, d, phrase_ids,
+                                                       n_phrase, bg_ids, M, t, B);
+    normalize_rows_kernel<<<1 + M, 256, 0, st>>>(t, B, d);
+    return 2;
+  }
   query_prep_kernel<<<1, 256, 2 * d * sizeof(float), st>>>(
       static_cast<const uint16_t*>(embed), vocab, d, phrase_ids, n_tmpl, n_phrase, bg_ids, M, t, B);
+  return 1;
 }
 
 ScoreLayout score_layout(int N, int n_v, int d, int M) {
@@ -428,6 +543,12 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   L.cand_g_off = take(sizeof(float) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
   L.cand_j_off = take(sizeof(int) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
   L.top_off = take(sizeof(int) * (size_t)N * RIFT_MAX_KNN);
+  // K slices of the Gram pass: enough CTAs for small scenes; each slice a whole number of
+  // 32-column chunks of d.
+  int split = N <= 512 ? 8 : (N <= 1024 ? 4 : 1);
+  while (split > 1 && (d / KK) % split != 0) split >>= 1;
+  L.n_split = split;
+  L.gpart_off = take(L.n_split > 1 ? sizeof(float) * (size_t)L.n_split * N * N : 0);
   L.total = off;
   (void)M;
   return L;
@@ -467,12 +588,16 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
   const int C = m > 0 ? std::min(std::min(m + KNN_SPARE, RIFT_MAX_KNN), N - 1) : 0;
   int launched = 4;
   if (m > 0) {
-    dim3 grid(L.n_jblk, L.n_jblk);
-    knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, C, cg, cj);
-    knn_merge_kernel<<<(N + 127) / 128, 128, 0, st>>>(cg, cj, L.n_jblk, N, C, topj);
+    float* gpart = reinterpret_cast<float*>(ws + L.gpart_off);
+    dim3 grid(L.n_jblk, L.n_jblk, L.n_split);
+    knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, C, cg, cj, gpart);
+    if (L.n_split > 1)
+      knn_row_topc_kernel<<<(N + RT_WARPS - 1) / RT_WARPS, 32 * RT_WARPS, 0, st>>>(gpart, L.n_split, N, C, topj);
+    else
+      knn_merge_kernel<<<(N + 127) / 128, 128, 0, st>>>(cg, cj, L.n_jblk, N, C, topj);
     launched += 2;
   }
-  knn_rescore_smooth_kernel<<<(N + 7) / 8, 256, 0, st>>>(V, d, topj, N, C, m, s_raw, s_tilde, nbr);
+  knn_rescore_smooth_kernel<<<N, 32 * RIFT_MAX_KNN, 0, st>>>(V, d, topj, N, C, m, s_raw, s_tilde, nbr);
   return launched;  // kernels launched
 }
 
