@@ -88,22 +88,28 @@ def barrier(ws):
         dist.barrier()
 
 
-def reduce_max(x: float, ws: int) -> float:
+def _reduce(x: float, ws: int, op: str, device) -> float:
     if ws == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
     return float(t.item())
 
 
-def reduce_sum(x: float, ws: int) -> float:
-    if ws == 1:
-        return x
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.SUM)
-    return float(t.item())
+def reduce_max(x: float, ws: int, device="cuda") -> float:
+    return _reduce(x, ws, "max", device)
+
+
+def reduce_sum(x: float, ws: int, device="cuda") -> float:
+    return _reduce(x, ws, "sum", device)
+
+
+def job_throughput(units_this_rank: float, ms_this_rank: float, ws: int, device="cuda"):
+    """Whole-job rate over replicas: units of all ranks / the slowest rank's time."""
+    ms_max = reduce_max(ms_this_rank, ws, device)
+    units = reduce_sum(units_this_rank, ws, device)
+    return units / (ms_max / 1e3), ms_max
 
 
 # ------------------------------------------------------------------------------------------ clocks
@@ -349,9 +355,7 @@ def main():
     prof = abi.profile_read()
     barrier(ws)
     ms = e0.elapsed_time(e1)
-    ms_max = reduce_max(ms, ws)
-    tokens_all = reduce_sum(float(T * args.steps), ws)
-    value = tokens_all / (ms_max / 1e3)
+    value, ms_max = job_throughput(float(T * args.steps), ms, ws)
 
     # ---- end to end: host buffers, H2D of the step's inputs and D2H of its result inside the region
     X_host = sc.X.cpu().pin_memory()
@@ -375,8 +379,7 @@ def main():
         out_host[:Te].copy_(pipe.packed[:Te], non_blocking=True)
     f1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = reduce_max(f0.elapsed_time(f1), ws)
-    e2e_val = reduce_sum(float(Te * args.e2e_steps), ws) / (e2e_ms / 1e3)
+    e2e_val, _ = job_throughput(float(Te * args.e2e_steps), f0.elapsed_time(f1), ws)
     h2d = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
     d2h = Te * s.d * 2 + 8
 

@@ -1,0 +1,60 @@
+"""Host-side logic of bench.py: replica aggregation over gloo ranks (world size 2, CPU) and the
+CPU reference arm's output line.  No GPU needed."""
+import json
+import os
+import subprocess
+import sys
+from pathlib import Path
+
+import pytest
+import torch
+import torch.multiprocessing as mp
+
+ROOT = Path(__file__).resolve().parent.parent
+
+
+def _rank(rank, ws, port, out):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=ws)
+    sys.path.insert(0, str(ROOT))
+    import bench
+    # rank r processed (r + 1) * 1000 units in (r + 1) * 100 ms
+    val, ms = bench.job_throughput(1000.0 * (rank + 1), 100.0 * (rank + 1), ws, device="cpu")
+    out.put((rank, val, ms))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_replica_throughput_is_all_units_over_the_slowest_rank():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = 29517
+    procs = [ctx.Process(target=_rank, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = [q.get(timeout=120) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for _, val, ms in res:
+        assert ms == 200.0
+        assert val == pytest.approx(3000.0 / 0.2)
+
+
+def test_single_rank_needs_no_process_group():
+    sys.path.insert(0, str(ROOT))
+    import bench
+    val, ms = bench.job_throughput(500.0, 250.0, 1)
+    assert ms == 250.0 and val == pytest.approx(2000.0)
+
+
+def test_reference_arm_prints_the_contract_line():
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    p = subprocess.run([sys.executable, str(ROOT / "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "1", "--warmup", "0"], capture_output=True, text=True, env=env, timeout=600)
+    assert p.returncode == 0, p.stderr[-2000:]
+    line = json.loads(p.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["metric"] == "retained prefill tokens/s"
+    assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
