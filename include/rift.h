@@ -242,6 +242,17 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
 rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int epilogue, void* out,
                         rift_stream_t stream);
 
+/* ---- The attention of a9 on its own (varlen, causal within each packed sequence) ----
+ *   qkv   fp16 [T, 3 n_heads head_dim]: per row q | k | v, each with heads contiguous, RoPE
+ *         already applied to q and k (as the prefill's QKV step leaves it)
+ *   cu_seqlens int32 [n_seq + 1]; out fp16 [T, n_heads head_dim] = softmax(q k^T / sqrt(head_dim)
+ *   + causal mask) v per sequence and head, softmax in fp32 with fp16 weights, fp32 accumulation
+ *   ws    rift_attention_workspace_bytes(T, n_seq) bytes (the q-block schedule)
+ * head_dim in {64, 128}. */
+size_t rift_attention_workspace_bytes(int max_T, int max_seqs);
+rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
+                                  int head_dim, void* out, void* ws, size_t ws_bytes, rift_stream_t stream);
+
 /* ---- Instrumentation for benchmarks (does not change any result) ----
  * Kernel classes timed by the profiler: */
 #define RIFT_PROF_GEMM 0      /* the prefill GEMMs (QKV, O, gate/up, down) */

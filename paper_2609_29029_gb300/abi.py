@@ -59,6 +59,8 @@ SIGNATURES = {
     "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _sz, _vp]),
     "rift_score_tiles_noalloc": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp]),
     "rift_linear": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
+    "rift_attention_workspace_bytes": (_sz, [_i, _i]),
+    "rift_attention_varlen": (_i, [_vp, _i, _vp, _i, _i, _i, _vp, _vp, _sz, _vp]),
     "rift_profile_enable": (None, [_i]),
     "rift_profile_read": (_i, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), _i]),
     "rift_launch_count": (C.c_longlong, []),
@@ -175,6 +177,15 @@ def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query
 
 def linear(A, W, M, N, K, epilogue, out, stream=None):
     _check(lib.rift_linear(ptr(A), ptr(W), M, N, K, epilogue, ptr(out), stream_handle(stream)), "rift_linear")
+
+
+def attention_workspace_bytes(max_T, max_seqs) -> int:
+    return lib.rift_attention_workspace_bytes(max_T, max_seqs)
+
+
+def attention_varlen(qkv, T, cu_seqlens, n_seq, n_heads, head_dim, out, ws, ws_bytes, stream=None):
+    _check(lib.rift_attention_varlen(ptr(qkv), T, ptr(cu_seqlens), n_seq, n_heads, head_dim, ptr(out), ptr(ws),
+                                     ws_bytes, stream_handle(stream)), "rift_attention_varlen")
 
 
 def prefill_workspace_bytes(model: Model, max_T, max_seqs, max_len) -> int:

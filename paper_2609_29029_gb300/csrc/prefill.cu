@@ -101,7 +101,7 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   L.attn_off = take(T * m.d * 2);
   L.act_off = take(T * m.ffn * 2);
   L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
-  L.max_qblocks = (max_T + 63) / 64 + max_seqs;
+  L.max_qblocks = attention_max_qblocks(max_T, max_seqs);
   L.sched_off = take((size_t)L.max_qblocks * sizeof(int2));
   L.total = off;
   return L;
@@ -161,7 +161,7 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
       norm_launch(1, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
     if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
     prof_begin(RIFT_PROF_ATTN, st);
-    launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st);
+    if (launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st)) return 1;
     prof_end(RIFT_PROF_ATTN, st, 1);
     if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st)) return 1;
     norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);

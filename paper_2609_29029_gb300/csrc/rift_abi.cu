@@ -117,7 +117,7 @@ const char* rift_status_string(rift_status s) {
 rift_status rift_sync_status(rift_stream_t stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return RIFT_ERR_CUDA;
   unsigned int f = read_clear_err_score() | read_clear_err_select() | read_clear_err_pack() |
-                   read_clear_err_prefill() | read_clear_err_gemm();
+                   read_clear_err_prefill() | read_clear_err_gemm() | read_clear_err_attn();
   if (cudaGetLastError() != cudaSuccess) return RIFT_ERR_CUDA;
   if (f & RIFT_EBIT_BADID) return RIFT_ERR_BAD_ID;
   if (f & RIFT_EBIT_NONFINITE) return RIFT_ERR_NONFINITE;
@@ -262,6 +262,31 @@ rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int e
   if (!aligned16(A) || !aligned16(W) || !aligned16(out)) return RIFT_ERR_INVALID;
   if (M == 0) return RIFT_OK;
   if (launch_gemm(A, W, M, N, K, epilogue, out, static_cast<cudaStream_t>(stream))) return RIFT_ERR_CUDA;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_attention_workspace_bytes(int max_T, int max_seqs) {
+  if (max_T < 0 || max_seqs < 0) return 0;
+  return (size_t)attention_max_qblocks(max_T, max_seqs) * sizeof(int2);
+}
+
+rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
+                                  int head_dim, void* out, void* ws, size_t ws_bytes, rift_stream_t stream) {
+  if (!qkv || !cu_seqlens || !out || T < 0 || n_seq < 0 || n_heads < 1) return RIFT_ERR_INVALID;
+  if (head_dim != 64 && head_dim != 128) return RIFT_ERR_INVALID;
+  if (T > 0 && n_seq < 1) return RIFT_ERR_INVALID;
+  if (!aligned16(qkv) || !aligned16(out)) return RIFT_ERR_INVALID;
+  const size_t need = rift_attention_workspace_bytes(T, n_seq);
+  if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
+  if (T == 0) return RIFT_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int2* sched = static_cast<int2*>(ws);
+  const int n_max = attention_max_qblocks(T, n_seq);
+  prof_begin(RIFT_PROF_ATTN, st);
+  launch_attention_schedule(cu_seqlens, n_seq, sched, n_max, st);
+  if (launch_attention(qkv, T, cu_seqlens, n_seq, n_heads, head_dim, sched, n_max, out, st)) return RIFT_ERR_CUDA;
+  prof_end(RIFT_PROF_ATTN, st, 2);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }

@@ -68,9 +68,12 @@ int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
                    cudaStream_t st);
 
-// q-block schedule of the varlen attention (built once per prefill from cu_seqlens)
+// Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
+// cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].
+int attention_max_qblocks(int max_T, int max_seqs);
 void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st);
-void launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
-                      int head_dim, const int2* sched, int n_sched_max, void* out, cudaStream_t st);
+int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
+                     const int2* sched, int n_sched_max, void* out, cudaStream_t st);
+unsigned int read_clear_err_attn();
 
 }  // namespace rift
