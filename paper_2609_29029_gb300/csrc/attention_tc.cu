@@ -142,6 +142,13 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
       : "memory");
 }
+// 2^x on the special-function unit (flushes subnormal results to zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
 
@@ -196,16 +203,23 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int n_items = n_entries * H;
   const int d = H * HD;
 
-  // number of 128-key blocks of an item (causal: keys up to the block's last valid row)
-  auto item_blocks = [&](int item, int& seq0, int& L, int& q0, int& h) -> int {
+  // An item's sequence start, length, first row, head and number of 128-key blocks (causal:
+  // keys up to the block's last valid row).  Every role reads the next item's entry while it
+  // works on the current one.
+  struct Item {
+    int seq0, L, q0, h, nkv;
+  };
+  auto load_item = [&](int item) -> Item {
+    Item it{0, 0, 0, 0, 0};
+    if (item >= n_items) return it;
     const int2 e = sched[item / H];
-    h = item % H;
-    if (e.x < 0) return 0;
-    seq0 = cu[e.x];
-    L = cu[e.x + 1] - seq0;
-    q0 = e.y;
-    const int last = min(L, q0 + BQ) - 1;
-    return last / BKV + 1;
+    it.h = item % H;
+    if (e.x < 0) return it;
+    it.seq0 = cu[e.x];
+    it.L = cu[e.x + 1] - it.seq0;
+    it.q0 = e.y;
+    it.nkv = (min(it.L, it.q0 + BQ) - 1) / BKV + 1;
+    return it;
   };
 
   if (warp == 0) {
@@ -213,9 +227,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       // ---------------- TMA producer
       uint32_t g = 0, it_local = 0;
       bool ok = true;
+      Item nxt = load_item(blockIdx.x);
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        int seq0 = 0, L = 0, q0 = 0, h = 0;
-        const int nkv = item_blocks(item, seq0, L, q0, h);
+        const Item cur = nxt;
+        nxt = load_item(item + gridDim.x);
+        const int seq0 = cur.seq0, q0 = cur.q0, h = cur.h, nkv = cur.nkv;
         if (nkv == 0) continue;
         if (!mbar_wait(Q_EMPTY, (it_local & 1u) ^ 1u, abort_flag)) { ok = false; break; }
         mbar_expect_tx(Q_FULL, CF::Q_BYTES);
@@ -255,9 +271,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         umma_commit(S_FULL(s));
         return true;
       };
+      Item nxt = load_item(blockIdx.x);
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        int seq0 = 0, L = 0, q0 = 0, h = 0;
-        const int nkv = item_blocks(item, seq0, L, q0, h);
+        const int nkv = nxt.nkv;
+        nxt = load_item(item + gridDim.x);
         if (nkv == 0) continue;
         if (!mbar_wait(Q_FULL, it_local & 1u, abort_flag)) break;
         fence_after();
@@ -293,12 +310,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     uint32_t g = 0, it_local = 0;
     bool ok = true;
+    Item nxt = load_item(blockIdx.x);
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-      int seq0 = 0, L = 0, q0 = 0, h = 0;
-      const int nkv = item_blocks(item, seq0, L, q0, h);
+      const Item cur = nxt;
+      nxt = load_item(item + gridDim.x);
+      const int seq0 = cur.seq0, L = cur.L, q0 = cur.q0, h = cur.h, nkv = cur.nkv;
       if (nkv == 0) continue;
       const int qrow = q0 + r;  // row within the sequence
-      float m = -INFINITY, l = 0.f;
+      float m = -INFINITY, l = 0.f;  // running maximum (log2 units, scaled) and sum
       for (int j = 0; j < nkv; ++j, ++g) {
         const int s = g & 1;
         if (!mbar_wait(S_FULL(s), (g >> 1) & 1u, abort_flag)) { ok = false; break; }
@@ -309,35 +328,39 @@ __global__ void __launch_bounds__(THREADS, 1)
         tmem_wait_ld();
         fence_before();
         mbar_arrive(S_EMPTY(s));
-        // scale and mask: key = j*128 + col valid iff key <= qrow and key < L
         const int k0 = j * BKV;
+        // Only the diagonal block and the block holding the sequence end need the mask: key
+        // valid iff key <= qrow and key < L (this branch is uniform over the CTA).
+        if (k0 + BKV - 1 > q0 || k0 + BKV > L) {
+          const int lim = min(qrow, L - 1) - k0;  // last valid column of this row
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (32 * c + e > lim) sv[c][e] = __float_as_uint(-INFINITY);
+        }
         float mx = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int key = k0 + 32 * c + e;
-            float v = __uint_as_float(sv[c][e]) * scale_log2;
-            if (key > qrow || key >= L) v = -INFINITY;
-            sv[c][e] = __float_as_uint(v);
-            mx = fmaxf(mx, v);
-          }
+          for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(sv[c][e]));
+        mx *= scale_log2;  // scale > 0: the maximum of the scaled scores
         float m_use = m, corr = 1.f;
         if (j == 0) {
           m_use = mx;
         } else if (mx > m + STALE) {
           m_use = mx;
-          corr = exp2f(m - mx);
+          corr = ex2(m - mx);
         }
-        const float base = (m_use == -INFINITY) ? 0.f : m_use;
+        const float nb = (m_use == -INFINITY) ? 0.f : -m_use;  // p = 2^(s * scale - m)
         float rs = 0.f;
         uint32_t pk[64];
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            const float p0 = exp2f(__uint_as_float(sv[c][e]) - base);
-            const float p1 = exp2f(__uint_as_float(sv[c][e + 1]) - base);
+            const float p0 = ex2(fmaf(__uint_as_float(sv[c][e]), scale_log2, nb));
+            const float p1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), scale_log2, nb));
             rs += p0 + p1;
             pk[c * 16 + e / 2] = pack_half2(p0, p1);
           }
