@@ -39,7 +39,7 @@ def parse():
     ap.add_argument("--workload", default="rift400_7b", choices=sorted(W.WORKLOADS))
     ap.add_argument("--impl", default="rift", choices=["rift", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--kernel-case", choices=["prefill", "score"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
@@ -357,30 +357,55 @@ def main():
     ms = e0.elapsed_time(e1)
     value, ms_max = job_throughput(float(T * args.steps), ms, ws)
 
-    # ---- end to end: host buffers, H2D of the step's inputs and D2H of its result inside the region
+    # ---- end to end: host buffers.  Every step copies its inputs (tokens, embedding table, ids)
+    # from pinned host memory and reads its result (the final hidden states) back.  The next
+    # step's inputs are copied on a second stream into the other of two device buffers while
+    # the current step computes, as a stream of scene queries would be served.
     X_host = sc.X.cpu().pin_memory()
     embed_host = sc.embed.cpu().pin_memory()
     ids_host = [torch.tensor(v, dtype=torch.int32).pin_memory() for v in (sc.query_ids, sc.bg_ids, sc.sys_ids)]
-    X_dev = torch.empty_like(sc.X)
-    emb_dev = torch.empty_like(sc.embed)
-    ids_dev = [torch.empty_like(h, device=dev) for h in ids_host]
+    bufs = [dict(X=torch.empty_like(sc.X), E=torch.empty_like(sc.embed),
+                 ids=[torch.empty_like(h, device=dev) for h in ids_host]) for _ in range(2)]
     out_host = torch.empty(T, s.d, dtype=torch.bfloat16).pin_memory()
+    copy_stream = torch.cuda.Stream(device=dev)
+
+    def h2d(buf):
+        with torch.cuda.stream(copy_stream):
+            buf["X"].copy_(X_host, non_blocking=True)
+            buf["E"].copy_(embed_host, non_blocking=True)
+            for hdst, hsrc in zip(buf["ids"], ids_host):
+                hdst.copy_(hsrc, non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(copy_stream)
+        return ev
+
+    def e2e_steps(n):
+        Te = 0
+        ready = h2d(bufs[0])
+        for k in range(n):
+            buf = bufs[k % 2]
+            stream.wait_event(ready)
+            if k + 1 < n:  # the other buffer is free: its last reader (step k - 1) has finished
+                nxt = torch.cuda.Event()
+                nxt.record(stream)
+                copy_stream.wait_event(nxt)
+                ready = h2d(bufs[(k + 1) % 2])
+            nk, Te = pipe.run(buf["X"], buf["E"], buf["ids"][0], buf["ids"][1], buf["ids"][2], buf["ids"][0],
+                              stream=stream)
+            out_host[:Te].copy_(pipe.packed[:Te], non_blocking=True)
+        return Te
+
+    e2e_steps(1)  # warm-up: first touch of the buffers
+    torch.cuda.synchronize()
     barrier(ws)
     torch.cuda.synchronize()
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     f0.record(stream)
-    Te = 0
-    for _ in range(args.e2e_steps):
-        X_dev.copy_(X_host, non_blocking=True)
-        emb_dev.copy_(embed_host, non_blocking=True)
-        for hdst, hsrc in zip(ids_dev, ids_host):
-            hdst.copy_(hsrc, non_blocking=True)
-        nk, Te = pipe.run(X_dev, emb_dev, ids_dev[0], ids_dev[1], ids_dev[2], ids_dev[0], stream=stream)
-        out_host[:Te].copy_(pipe.packed[:Te], non_blocking=True)
+    Te = e2e_steps(args.e2e_steps)
     f1.record(stream)
     torch.cuda.synchronize()
     e2e_val, _ = job_throughput(float(Te * args.e2e_steps), f0.elapsed_time(f1), ws)
-    h2d = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
+    h2d_bytes = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
     d2h = Te * s.d * 2 + 8
 
     if rank != 0:
@@ -421,7 +446,7 @@ def main():
                      "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (of measured)",
                      "launches": gemm_n},
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
