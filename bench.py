@@ -41,6 +41,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
+    ap.add_argument("--sweep", action="store_true",
+                    help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
     ap.add_argument("--kernel-case", choices=["prefill", "score"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
                          "'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); each runs 3 times")
@@ -267,6 +269,45 @@ def gemm_traffic():
     return int(b.group(1))
 
 
+def sweep(steps: int, warmup: int):
+    """Scoring + selection + packing (no prefill) of the Rift policy over N tiles: per-step device
+    time, per-kernel-class time, and the HBM rate of the token pass (N n_v d 2 bytes read)."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_29029_gb300 import ScenePipeline, abi
+    dev = torch.device("cuda", 0)
+    peaks = json.loads((ROOT / "MEASURED_PEAKS.json").read_text()) if (ROOT / "MEASURED_PEAKS.json").exists() else {}
+    hbm = peaks.get("hbm_gbs", 6796.5)
+    for N in W.SWEEP_N:
+        wl = W.sweep_workload(N)
+        s = wl.scene
+        sc = W.make_scene(s, wl.decoder.vocab, dev)
+        pipe = ScenePipeline(s.N, s.n_v, s.d, s.x_dtype, s.M, s.S, s.Q, wl.knn_m, wl.policy, device=dev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        q, bg, sy = (torch.tensor(v, **i32) for v in (sc.query_ids, sc.bg_ids, sc.sys_ids))
+        for _ in range(warmup):
+            pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False)
+        torch.cuda.synchronize()
+        abi.profile_enable(True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(steps):
+            n_kept, T = pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False)
+        e1.record()
+        torch.cuda.synchronize()
+        abi.profile_enable(False)
+        prof = abi.profile_read()
+        ms = e0.elapsed_time(e1) / steps
+        x_bytes = sc.X.numel() * sc.X.element_size()
+        line = {"sweep": f"select+gather N={N}", "ms_per_query": ms,
+                "kernels_ms": {k: round(v[0] / steps, 4) for k, v in prof.items() if v[1]},
+                "kept_tiles": n_kept, "packed_rows": T, "x_bytes": x_bytes,
+                "token_pass_lower_bound_ms": x_bytes / (hbm * 1e6)}
+        print(json.dumps(line), flush=True)
+        del sc, pipe
+        torch.cuda.empty_cache()
+
+
 def kernel_case(name: str):
     """Small cases for ncu captures: inputs larger than L2, about 1 GB on the device."""
     import __graft_entry__
@@ -307,6 +348,9 @@ def main():
         return
     if args.kernel_case:
         kernel_case(args.kernel_case)
+        return
+    if args.sweep:
+        sweep(args.steps, max(args.warmup, 1))
         return
     ws, rank, local = dist_setup()
     wl = W.WORKLOADS[args.workload]
