@@ -150,8 +150,20 @@ __device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
 
 // Epilogue for one row of one 32-column chunk (columns n0 .. n0 + 31 of the tile).
 template <int EPI>
-__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row, int col, int N, void* C) {
-  if constexpr (EPI == EPI_STORE_BF16) {
+__device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row, int col, int N, void* C,
+                                               float out_scale = 1.f) {
+  if constexpr (EPI == EPI_STORE_F32) {
+    float* out = static_cast<float*>(C) + (size_t)row * N + col;
+    if (col + 32 <= N) {
+      float4* o4 = reinterpret_cast<float4*>(out);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        o4[q] = make_float4(__uint_as_float(r[4 * q]) * out_scale, __uint_as_float(r[4 * q + 1]) * out_scale,
+                            __uint_as_float(r[4 * q + 2]) * out_scale, __uint_as_float(r[4 * q + 3]) * out_scale);
+    } else {
+      for (int j = 0; j < 32 && col + j < N; ++j) out[j] = __uint_as_float(r[j]) * out_scale;
+    }
+  } else if constexpr (EPI == EPI_STORE_BF16) {
     uint16_t* out = static_cast<uint16_t*>(C) + (size_t)row * N + col;
     if (col + 32 <= N) {
       uint4* o4 = reinterpret_cast<uint4*>(out);
@@ -185,7 +197,7 @@ __device__ __forceinline__ void epilogue_chunk(const uint32_t (&r)[32], int row,
       for (int j = 0; j < 32; ++j)
         if (col + j < N) out[j] += __uint_as_float(r[j]);
     }
-  } else {  // EPI_SWIGLU: columns col..col+15 are gate, col+16..col+31 the matching up rows
+  } else if constexpr (EPI == EPI_SWIGLU) {  // columns col..col+15 gate, col+16..col+31 the matching up
     if (col >= N) return;
     const int F = N / 2;
     uint16_t* out = static_cast<uint16_t*>(C) + (size_t)row * F + col / 2;
@@ -364,7 +376,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld32(taddr + c, r);
-          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C);
+          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C, ep.out_scale);
         }
       }
       fence_before();
@@ -456,6 +468,7 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, ep, st);
     case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, ep, st);
     case EPI_QKV_ROPE: return launch<EPI_QKV_ROPE>(ma, mb, M, N, K, C, ep, st);
+    case EPI_STORE_F32: return launch<EPI_STORE_F32>(ma, mb, M, N, K, C, ep, st);
     default: return 1;
   }
 }

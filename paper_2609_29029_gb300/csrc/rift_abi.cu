@@ -159,7 +159,8 @@ rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int 
   prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
   const int nk = launch_score(X, xdt, N, n_v, d, t, B, M, m, token_scores, tile_s_raw, tile_s, nbr,
                               static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
-  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk);
+  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk < 0 ? 0 : nk);
+  if (nk < 0) return RIFT_ERR_CUDA;
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }

@@ -20,11 +20,14 @@ unsigned int read_clear_err_gemm();
 // ---- score.cu ----
 struct ScoreLayout {
   int chunk_tokens, n_chunks, n_jblk, n_split;
-  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, gpart_off, total;
+  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, gpart_off, split_a_off, split_b_off, gram_off,
+      total;
+  bool tensor_gram;  // N > 1024: the Gram matrix on the tensor cores (fp16 hi/lo split)
 };
 ScoreLayout score_layout(int N, int n_v, int d, int M);
 int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st);
+// Returns the number of kernels launched, or -1 if a launch could not be set up.
 int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
                  int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
                  cudaStream_t st);
@@ -54,7 +57,8 @@ enum GemmEpilogue {
   EPI_STORE_BF16 = 0,  // C fp16 [M, N] (name kept from the ABI's numbering)
   EPI_RESID_F32 = 1,   // R fp32 [M, N] += acc
   EPI_SWIGLU = 2,      // N = 2F interleaved in 16-column groups; C fp16 [M, F] = silu(g) * u
-  EPI_QKV_ROPE = 3     // C fp16 [M, N]; columns < rope_cols get rotate-half RoPE at positions[row]
+  EPI_QKV_ROPE = 3,    // C fp16 [M, N]; columns < rope_cols get rotate-half RoPE at positions[row]
+  EPI_STORE_F32 = 4    // C fp32 [M, N] = acc * out_scale
 };
 struct EpiParams {
   const int* positions = nullptr;  // [M] position of each row (EPI_QKV_ROPE)
@@ -62,6 +66,7 @@ struct EpiParams {
   int rope_cols = 0;               // q and k columns: 2 d
   int head_dim = 0;
   int max_len = 0;
+  float out_scale = 1.f;           // EPI_STORE_F32
 };
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
                 cudaStream_t st, const EpiParams& ep = EpiParams());

@@ -415,6 +415,69 @@ __global__ void __launch_bounds__(32 * RT_WARPS) knn_row_topc_kernel(const float
   }
 }
 
+// Large scenes (N > 1024): the Gram matrix on the tensor cores.  Each fp32 row of V (scaled
+// by 2^10, so that the low parts stay normal in fp16) is split into hi = fp16(v) and
+// lo = fp16(v - hi); A = [hi | hi | lo] and B = [hi | lo | hi] along K, so one fp16 GEMM with
+// K = 3 d gives hi.hi + hi.lo + lo.hi, i.e. V V^T to ~2^-22 relative (lo.lo is below that).
+constexpr float KNN_SPLIT_SCALE = 1024.f;
+// Rows N .. Np - 1 of B (the padding of the Gram matrix's column count to a multiple of 8) are zero.
+__global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, uint16_t* __restrict__ A,
+                                 uint16_t* __restrict__ B) {
+  const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (size_t)Np * d) return;
+  const size_t i = idx / d;
+  const int k = (int)(idx % d);
+  if (i >= (size_t)N) {
+    uint16_t* b = B + i * 3 * d;
+    b[k] = 0; b[d + k] = 0; b[2 * d + k] = 0;
+    return;
+  }
+  const float v = V[idx] * KNN_SPLIT_SCALE;
+  const __half hi = __float2half_rn(v);
+  const __half lo = __float2half_rn(v - __half2float(hi));
+  const uint16_t h = *reinterpret_cast<const uint16_t*>(&hi), l = *reinterpret_cast<const uint16_t*>(&lo);
+  uint16_t* a = A + i * 3 * d;
+  uint16_t* b = B + i * 3 * d;
+  a[k] = h; a[d + k] = h; a[2 * d + k] = l;
+  b[k] = h; b[d + k] = l; b[2 * d + k] = h;
+}
+
+// One warp per row of the materialised Gram matrix: each lane keeps a sorted top-C of its
+// columns, then C rounds of a warp-wide argmax (larger similarity, then lower index) merge them.
+__global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld, int C, int* __restrict__ top_j) {
+  const int lane = threadIdx.x & 31;
+  const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (i >= N) return;
+  float bg[RIFT_MAX_KNN];
+  int bj[RIFT_MAX_KNN];
+  for (int r = 0; r < C; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
+  const float* row = G + (size_t)i * ld;
+  for (int j = lane; j < N; j += 32) {
+    if (j == i) continue;
+    const float g = row[j];
+    if (!(g == g)) { atomicOr(&g_err_score, RIFT_EBIT_NONFINITE); continue; }
+    if (!knn_better(g, j, bg[C - 1], bj[C - 1])) continue;
+    int p = C - 1;
+    while (p > 0 && knn_better(g, j, bg[p - 1], bj[p - 1])) { bg[p] = bg[p - 1]; bj[p] = bj[p - 1]; --p; }
+    bg[p] = g; bj[p] = j;
+  }
+  int head = 0;
+  for (int r = 0; r < C; ++r) {
+    float cg = head < C ? bg[head] : -INFINITY;
+    int cj = head < C ? bj[head] : 0x7fffffff;
+    int cl = lane;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float og = __shfl_xor_sync(0xffffffffu, cg, o);
+      const int oj = __shfl_xor_sync(0xffffffffu, cj, o);
+      const int ol = __shfl_xor_sync(0xffffffffu, cl, o);
+      if (knn_better(og, oj, cg, cj)) { cg = og; cj = oj; cl = ol; }
+    }
+    if (cl == lane) ++head;
+    if (lane == 0) top_j[(size_t)i * C + r] = (cg == -INFINITY) ? 0x7fffffff : cj;
+  }
+}
+
 // One thread per tile: merge the blocks' candidate lists into the row's top-C by fp32
 // similarity (C = m + a few spares).
 __global__ void knn_merge_kernel(const float* __restrict__ cand_g, const int* __restrict__ cand_j, int n_lists,
@@ -549,6 +612,11 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   while (split > 1 && (d / KK) % split != 0) split >>= 1;
   L.n_split = split;
   L.gpart_off = take(L.n_split > 1 ? sizeof(float) * (size_t)L.n_split * N * N : 0);
+  L.tensor_gram = N > 1024;
+  const size_t Np = ((size_t)N + 7) & ~size_t(7);
+  L.split_a_off = take(L.tensor_gram ? sizeof(uint16_t) * (size_t)N * 3 * d : 0);
+  L.split_b_off = take(L.tensor_gram ? sizeof(uint16_t) * Np * 3 * d : 0);
+  L.gram_off = take(L.tensor_gram ? sizeof(float) * (size_t)N * Np : 0);
   L.total = off;
   (void)M;
   return L;
@@ -587,7 +655,19 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
   // candidates per row: m plus spares for the fp64 rescoring, at most the N - 1 other tiles
   const int C = m > 0 ? std::min(std::min(m + KNN_SPARE, RIFT_MAX_KNN), N - 1) : 0;
   int launched = 4;
-  if (m > 0) {
+  if (m > 0 && L.tensor_gram) {
+    uint16_t* A16 = reinterpret_cast<uint16_t*>(ws + L.split_a_off);
+    uint16_t* B16 = reinterpret_cast<uint16_t*>(ws + L.split_b_off);
+    float* G = reinterpret_cast<float*>(ws + L.gram_off);
+    const int Np = (N + 7) & ~7;
+    const size_t n = (size_t)Np * d;
+    knn_split_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(V, N, Np, d, A16, B16);
+    EpiParams ep;
+    ep.out_scale = 1.f / (KNN_SPLIT_SCALE * KNN_SPLIT_SCALE);
+    if (launch_gemm_tc(A16, B16, N, Np, 3 * d, EPI_STORE_F32, G, ep, st)) return -1;
+    knn_gram_topc_kernel<<<(N + 3) / 4, 128, 0, st>>>(G, N, Np, C, topj);
+    launched += 3;
+  } else if (m > 0) {
     float* gpart = reinterpret_cast<float*>(ws + L.gpart_off);
     dim3 grid(L.n_jblk, L.n_jblk, L.n_split);
     knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, C, cg, cj, gpart);

@@ -66,7 +66,8 @@ extern "C" rift_status rift_score_tiles_noalloc(const void* X, rift_dtype xdt, i
   rift::prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
   const int nk = rift::launch_score(X, xdt, N, n_v, d, t, B, M, m, token_scores, tile_s_raw, tile_s, nbr,
                                     static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
-  rift::prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk);
+  rift::prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk < 0 ? 0 : nk);
+  if (nk < 0) return RIFT_ERR_CUDA;
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }
