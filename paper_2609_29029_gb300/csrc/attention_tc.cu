@@ -1,17 +1,26 @@
 // Varlen causal attention on Blackwell's tcgen05 tensor cores (sm_103a).
 //
-// Work item = (128-row q-block of one packed sequence, one head).  Persistent CTAs (one per SM)
-// walk the items; tensor memory and barriers are set up once per CTA.  Per CTA, 192 threads:
-//   warp 0      TMA: the item's Q tile, then K and V tiles of 128 keys into two stages
-//               (fp16, 128B swizzle; a 128-column box pair per 128-wide head)
-//   warp 1      one thread issues S_j = Q K_j^T (M = 128, N = 128 keys) into one of two TMEM
-//               S buffers, and O += P_j V_j (N = head_dim, V read as an MN-major operand)
+// Work item = (128-row q-block of one packed sequence, one head).  Persistent CTAs walk the
+// items; tensor memory and barriers are set up once per CTA.  Two shapes share one kernel:
+//   KB = 64   keys per block, two CTAs per SM (96 KB shared memory, 256 TMEM columns each): while
+//             one CTA waits on a load, a product or its softmax, the other keeps the SM busy
+//   KB = 128  keys per block, one CTA per SM, 3-stage rings and two O buffers
+// Per CTA, 192 threads:
+//   warp 0      TMA, two threads: lane 0 loads K tiles (KB keys) into a ring, lane 1 loads the
+//               item's Q tile and the V tiles into their own ring (fp16, 128B swizzle; a 64-column
+//               box per 64 head dims)
+//   warp 1      one thread issues S_j = Q K_j^T (M = 128, N = KB) into one of two TMEM S buffers,
+//               and O += P_j V_j with P_j read from tensor memory (the A operand of the TS form) and
+//               V_j from shared memory as an MN-major operand
 //   warps 2..5  softmax, one query row per thread (TMEM lane = row): scale, causal and
 //               sequence-end mask, online softmax with a stale maximum (O is rescaled in TMEM
-//               only when a row's maximum grows by more than 2^8), P_j written as fp16 into a
-//               swizzled shared tile for the PV product; at the end O / l is stored as fp16.
-// TMEM: O in columns [0, 128), S buffers at 128 and 256.  Every mbarrier wait is bounded; on
-// timeout the kernel sets RIFT_EBIT_TIMEOUT and every role falls through.
+//               only when a row's maximum grows by more than 2^8), P_j written back as packed fp16
+//               over the first KB / 2 columns of its own S buffer; at the end of an item O / l is
+//               stored as fp16.
+// K is released as soon as its S product completes and V after its PV product; S/P is
+// double-buffered, so the softmax of block j overlaps S_{j+1} and PV_{j-1}.  S_{j+2} is issued
+// only once PV_j (the reader of P_j in the same columns) has completed.  Every mbarrier wait is
+// bounded; on timeout the kernel sets RIFT_EBIT_TIMEOUT and every role falls through.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -32,24 +41,28 @@ unsigned int read_clear_err_attn() {
 
 namespace fa {
 
-constexpr int BQ = 128, BKV = 128, THREADS = 192;
-constexpr int TMEM_COLS = 512;
-constexpr uint32_t S_COL0 = 128;  // S buffers at columns 128 and 256; O at 0
-constexpr float STALE = 8.f;      // log2 units: P <= 2^8 before a rescale is forced
+constexpr int BQ = 128, THREADS = 192;
+constexpr float STALE = 8.f;  // log2 units: P <= 2^8 before a rescale is forced
 
-template <int HD>
+template <int HD, int KB>
 struct Cfg {
+  static constexpr int CTAS = KB == 64 ? 2 : 1;  // CTAs per SM
+  static constexpr int NST = KB == 64 ? 2 : 3;   // K and V ring stages
+  static constexpr int NO = KB == 64 ? 1 : 2;    // O buffers in TMEM
+  static constexpr int TMEM_COLS = NO * 128 + 2 * KB;
+  static constexpr uint32_t S_COL0 = NO * 128;   // S/P buffers after the O buffers
   static constexpr int Q_BYTES = BQ * HD * 2;
-  static constexpr int K_BYTES = BKV * HD * 2;
-  static constexpr int V_BYTES = BKV * HD * 2;
-  static constexpr int P_BYTES = BQ * BKV * 2;
-  static constexpr int STAGE = K_BYTES + V_BYTES;
-  static constexpr size_t SMEM = (size_t)Q_BYTES + 2 * STAGE + P_BYTES + 1024 + 256;
+  static constexpr int K_BYTES = KB * HD * 2;
+  static constexpr int V_BYTES = KB * HD * 2;
+  static constexpr size_t SMEM = (size_t)Q_BYTES + NST * (K_BYTES + V_BYTES) + 1024 + 512;
   // kind::f16 instruction descriptors: fp32 D, fp16 A and B, M = 128.
-  // S = Q K^T: both K-major, N = 128 keys.  O += P V: P K-major, V MN-major (bit 16), N = HD.
-  static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) | ((uint32_t)(BQ >> 4) << 24);
+  // S = Q K^T: both K-major, N = KB keys.  O += P V: P K-major (in TMEM), V MN-major (bit 16),
+  // N = HD.
+  static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(KB >> 3) << 17) | ((uint32_t)(BQ >> 4) << 24);
   static constexpr uint32_t IDESC_O =
       (1u << 4) | (1u << 16) | ((uint32_t)(HD >> 3) << 17) | ((uint32_t)(BQ >> 4) << 24);
+  static_assert(TMEM_COLS == 256 || TMEM_COLS == 512, "TMEM allocation must be a power of two");
+  static_assert(SMEM * CTAS <= 232448, "shared memory per SM");
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -115,6 +128,13 @@ __device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t a, uint64_t b, ui
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
       "l"(a), "l"(b), "r"(idesc), "r"(accum));
 }
+// A from tensor memory (TS form): row i of A in lane i, two fp16 per 32-bit column.
+__device__ __forceinline__ void umma_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "r"(tmem_a), "l"(b), "r"(idesc), "r"(accum));
+}
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
                : "memory");
@@ -149,42 +169,95 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Three-input maximum and packed pairs of fp32 (Blackwell's f32x2 FMA-pipe forms).
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ float2 unf2(uint64_t v) {
+  float2 r;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+  return r;
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+// 32-byte global store (address 32-byte aligned).
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* r) {
+  asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};\n" ::"l"(p), "r"(r[0]), "r"(r[1]), "r"(r[2]),
+               "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
+}
+
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
 
 // Item i -> (schedule entry, head): entries are q-blocks (sequence, first row); heads inner.
-template <int HD>
-__global__ void __launch_bounds__(THREADS, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tm, const int* __restrict__ cu, const int2* __restrict__ sched,
-                   int n_entries, int H, float scale_log2, uint16_t* __restrict__ out) {
-  using CF = Cfg<HD>;
+template <int HD, int KB>
+__global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+                   const int* __restrict__ cu, const int2* __restrict__ sched, int n_entries, int H, float scale_log2,
+                   uint16_t* __restrict__ out) {
+  using CF = Cfg<HD, KB>;
+  constexpr int NST = CF::NST, NO = CF::NO, NC = KB / 32;  // NC: 32-key chunks per block
+  constexpr uint32_t S_COL0 = CF::S_COL0;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
-  uint8_t* sKV = smem + CF::Q_BYTES;                 // stage s: K at sKV + s*STAGE, V after it
-  uint8_t* sP = sKV + 2 * CF::STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + CF::P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  uint8_t* sK = smem + CF::Q_BYTES;             // stage s at sK + s * K_BYTES
+  uint8_t* sV = sK + NST * CF::K_BYTES;         // stage s at sV + s * V_BYTES
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + NST * CF::V_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 32);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const uint32_t b0 = smem_u32(bars);
-  const uint32_t Q_FULL = b0, Q_EMPTY = b0 + 8, P_FULL = b0 + 16, PV_DONE = b0 + 24, O_EMPTY = b0 + 32;
-  auto KV_FULL = [&](int s) { return b0 + 40 + 8u * s; };
-  auto KV_EMPTY = [&](int s) { return b0 + 56 + 8u * s; };
-  auto S_FULL = [&](int s) { return b0 + 72 + 8u * s; };
-  auto S_EMPTY = [&](int s) { return b0 + 88 + 8u * s; };
+  // barrier k lives at b0 + 8 k; rings and buffers are indexed by the stage or buffer
+  const uint32_t Q_FULL = b0, Q_EMPTY = b0 + 8;
+  auto BAR = [&](int base, int i) { return b0 + 8u * (uint32_t)(base + i); };
+  enum { K_FULL = 2, K_EMPTY = K_FULL + NST, V_FULL = K_EMPTY + NST, V_EMPTY = V_FULL + NST, S_FULL = V_EMPTY + NST,
+         P_FULL = S_FULL + 2, PV_DONE = P_FULL + 2, O_FULL = PV_DONE + 2, O_EMPTY = O_FULL + NO, N_BARS = O_EMPTY + NO };
+  static_assert(N_BARS <= 32, "barrier slots");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     mbar_init(Q_FULL, 1);
     mbar_init(Q_EMPTY, 1);
-    mbar_init(P_FULL, 128);
-    mbar_init(PV_DONE, 1);
-    mbar_init(O_EMPTY, 128);
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(KV_FULL(s), 1);
-      mbar_init(KV_EMPTY(s), 1);
-      mbar_init(S_FULL(s), 1);
-      mbar_init(S_EMPTY(s), 128);
+    for (int b = 0; b < NST; ++b) {
+      mbar_init(BAR(K_FULL, b), 1);
+      mbar_init(BAR(K_EMPTY, b), 1);
+      mbar_init(BAR(V_FULL, b), 1);
+      mbar_init(BAR(V_EMPTY, b), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(BAR(S_FULL, b), 1);
+      mbar_init(BAR(P_FULL, b), 128);
+      mbar_init(BAR(PV_DONE, b), 1);
+    }
+    for (int b = 0; b < NO; ++b) {
+      mbar_init(BAR(O_FULL, b), 1);
+      mbar_init(BAR(O_EMPTY, b), 128);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
@@ -192,7 +265,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS)
+                 "r"(CF::TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
   }
@@ -203,7 +276,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int n_items = n_entries * H;
   const int d = H * HD;
 
-  // An item's sequence start, length, first row, head and number of 128-key blocks (causal:
+  // An item's sequence start, length, first row, head and number of KB-key blocks (causal:
   // keys up to the block's last valid row).  Every role reads the next item's entry while it
   // works on the current one.
   struct Item {
@@ -218,57 +291,65 @@ __global__ void __launch_bounds__(THREADS, 1)
     it.seq0 = cu[e.x];
     it.L = cu[e.x + 1] - it.seq0;
     it.q0 = e.y;
-    it.nkv = (min(it.L, it.q0 + BQ) - 1) / BKV + 1;
+    it.nkv = (min(it.L, it.q0 + BQ) - 1) / KB + 1;
     return it;
   };
+  // Counters shared by every role: g counts KB-key blocks, t counts items of this CTA.  Block g
+  // uses K/V stage g % NST (phase (g / NST) & 1) and S/P buffer g & 1 (phase (g >> 1) & 1); item t
+  // uses O buffer t % NO (phase (t / NO) & 1).
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ---------------- TMA producer
-      uint32_t g = 0, it_local = 0;
+    if (lane < 2) {
+      // ---------------- TMA producers: lane 0 K tiles; lane 1 Q and V tiles
+      uint32_t g = 0, t = 0;
       bool ok = true;
       Item nxt = load_item(blockIdx.x);
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
         const Item cur = nxt;
         nxt = load_item(item + gridDim.x);
-        const int seq0 = cur.seq0, q0 = cur.q0, h = cur.h, nkv = cur.nkv;
-        if (nkv == 0) continue;
-        if (!mbar_wait(Q_EMPTY, (it_local & 1u) ^ 1u, abort_flag)) { ok = false; break; }
-        mbar_expect_tx(Q_FULL, CF::Q_BYTES);
-        for (int c = 0; c < HD / 64; ++c)
-          tma_load_2d(smem_u32(sQ + c * BQ * 128), &tm, h * HD + c * 64, seq0 + q0, Q_FULL);
-        for (int j = 0; j < nkv; ++j, ++g) {
-          const int s = g & 1;
-          if (!mbar_wait(KV_EMPTY(s), ((g >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
-          mbar_expect_tx(KV_FULL(s), CF::STAGE);
-          uint8_t* sK = sKV + s * CF::STAGE;
-          uint8_t* sV = sK + CF::K_BYTES;
-          for (int c = 0; c < HD / 64; ++c) {
-            tma_load_2d(smem_u32(sK + c * BKV * 128), &tm, d + h * HD + c * 64, seq0 + j * BKV, KV_FULL(s));
-            tma_load_2d(smem_u32(sV + c * BKV * 128), &tm, 2 * d + h * HD + c * 64, seq0 + j * BKV, KV_FULL(s));
-          }
+        if (cur.nkv == 0) continue;
+        if (lane == 1) {
+          if (!mbar_wait(Q_EMPTY, (t & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+          mbar_expect_tx(Q_FULL, CF::Q_BYTES);
+          for (int c = 0; c < HD / 64; ++c)
+            tma_load_2d(smem_u32(sQ + c * BQ * 128), &tm_q, cur.h * HD + c * 64, cur.seq0 + cur.q0, Q_FULL);
         }
-        ++it_local;
+        for (int j = 0; j < cur.nkv; ++j, ++g) {
+          const int s = g % NST;
+          const uint32_t ph = (g / NST) & 1u;
+          const int col = (lane == 0 ? d : 2 * d) + cur.h * HD;
+          const int base = lane == 0 ? K_EMPTY : V_EMPTY;
+          if (!mbar_wait(BAR(base, s), ph ^ 1u, abort_flag)) { ok = false; break; }
+          const uint32_t full = BAR(lane == 0 ? K_FULL : V_FULL, s);
+          mbar_expect_tx(full, CF::K_BYTES);
+          uint8_t* dst = (lane == 0 ? sK + s * CF::K_BYTES : sV + s * CF::V_BYTES);
+          for (int c = 0; c < HD / 64; ++c)
+            tma_load_2d(smem_u32(dst + c * KB * 128), &tm_kv, col + c * 64, cur.seq0 + j * KB, full);
+        }
+        ++t;
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer
-      uint32_t g = 0, it_local = 0;
+      uint32_t g = 0, t = 0;
       bool ok = true;
       auto issue_s = [&](uint32_t gg) -> bool {
-        const int s = gg & 1;
-        if (!mbar_wait(KV_FULL(s), (gg >> 1) & 1u, abort_flag)) return false;
-        if (!mbar_wait(S_EMPTY(s), ((gg >> 1) & 1u) ^ 1u, abort_flag)) return false;
+        const int st = gg % NST, sb = gg & 1;
+        if (!mbar_wait(BAR(K_FULL, st), (gg / NST) & 1u, abort_flag)) return false;
+        // S/P buffer sb is free once PV_{gg-2}, the reader of P_{gg-2}, has completed
+        if (gg >= 2 && !mbar_wait(BAR(PV_DONE, sb), ((gg - 2) >> 1) & 1u, abort_flag)) return false;
         fence_after();
-        const uint32_t sK = smem_u32(sKV + s * CF::STAGE);
-        const uint32_t sQa = smem_u32(sQ);
+        const uint32_t kb = smem_u32(sK + st * CF::K_BYTES);
+        const uint32_t qb = smem_u32(sQ);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {  // 16 of the head dims per step
-          const uint32_t off = (kk >> 2) * (BQ * 128) + (kk & 3) * 32;
-          umma(tmem + S_COL0 + 128u * s, desc_kmajor(sQa + off), desc_kmajor(sK + off), CF::IDESC_S, kk > 0);
+          const uint32_t koff = (kk & 3) * 32;
+          umma(tmem + S_COL0 + (uint32_t)KB * sb, desc_kmajor(qb + (kk >> 2) * (BQ * 128) + koff),
+               desc_kmajor(kb + (kk >> 2) * (KB * 128) + koff), CF::IDESC_S, kk > 0);
         }
-        umma_commit(S_FULL(s));
+        umma_commit(BAR(S_FULL, sb));
+        umma_commit(BAR(K_EMPTY, st));
         return true;
       };
       Item nxt = load_item(blockIdx.x);
@@ -276,7 +357,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int nkv = nxt.nkv;
         nxt = load_item(item + gridDim.x);
         if (nkv == 0) continue;
-        if (!mbar_wait(Q_FULL, it_local & 1u, abort_flag)) break;
+        const int ob = t % NO;
+        if (!mbar_wait(Q_FULL, t & 1u, abort_flag)) break;
         fence_after();
         if (!issue_s(g)) break;
         for (int j = 0; j < nkv; ++j, ++g) {
@@ -285,65 +367,74 @@ __global__ void __launch_bounds__(THREADS, 1)
           } else {
             umma_commit(Q_EMPTY);  // Q is free once the item's S products complete
           }
-          if (!mbar_wait(P_FULL, g & 1u, abort_flag)) { ok = false; break; }
-          if (j == 0 && !mbar_wait(O_EMPTY, (it_local & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+          const int st = g % NST, sb = g & 1;
+          if (!mbar_wait(BAR(P_FULL, sb), (g >> 1) & 1u, abort_flag)) { ok = false; break; }
+          if (j == 0 && !mbar_wait(BAR(O_EMPTY, ob), ((t / NO) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(BAR(V_FULL, st), (g / NST) & 1u, abort_flag)) { ok = false; break; }
           fence_after();
-          const int s = g & 1;
-          const uint32_t sV = smem_u32(sKV + s * CF::STAGE + CF::K_BYTES);
-          const uint32_t sPa = smem_u32(sP);
+          const uint32_t vb = smem_u32(sV + st * CF::V_BYTES);
 #pragma unroll
-          for (int kk = 0; kk < BKV / 16; ++kk) {  // 16 keys per step
-            const uint64_t a = desc_kmajor(sPa + (kk >> 2) * (BQ * 128) + (kk & 3) * 32);
-            const uint64_t b = desc_mnmajor(sV + kk * 2048, BKV * 128);
-            umma(tmem, a, b, CF::IDESC_O, (j > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < KB / 16; ++kk) {  // 16 keys (8 TMEM columns of P) per step
+            const uint64_t bdesc = desc_mnmajor(vb + kk * 2048, KB * 128);
+            umma_ts(tmem + 128u * ob, tmem + S_COL0 + (uint32_t)KB * sb + 8u * kk, bdesc, CF::IDESC_O,
+                    (j > 0 || kk > 0) ? 1u : 0u);
           }
-          umma_commit(PV_DONE);
-          umma_commit(KV_EMPTY(s));
+          umma_commit(BAR(PV_DONE, sb));
+          umma_commit(BAR(V_EMPTY, st));
         }
-        ++it_local;
+        if (!ok) break;
+        umma_commit(BAR(O_FULL, ob));
+        ++t;
       }
     }
   } else {
-    // ---------------- softmax: thread = query row (TMEM lane)
+    // ---------------- softmax and output: thread = query row (TMEM lane)
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
-    uint32_t g = 0, it_local = 0;
+    uint32_t g = 0, t = 0;
     bool ok = true;
     Item nxt = load_item(blockIdx.x);
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
       const Item cur = nxt;
       nxt = load_item(item + gridDim.x);
-      const int seq0 = cur.seq0, L = cur.L, q0 = cur.q0, h = cur.h, nkv = cur.nkv;
+      const int L = cur.L, q0 = cur.q0, nkv = cur.nkv;
       if (nkv == 0) continue;
+      const int ob = t % NO;
+      const uint32_t o_base = lane_base + 128u * ob;
       const int qrow = q0 + r;  // row within the sequence
       float m = -INFINITY, l = 0.f;  // running maximum (log2 units, scaled) and sum
       for (int j = 0; j < nkv; ++j, ++g) {
-        const int s = g & 1;
-        if (!mbar_wait(S_FULL(s), (g >> 1) & 1u, abort_flag)) { ok = false; break; }
+        const int sb = g & 1;
+        if (!mbar_wait(BAR(S_FULL, sb), (g >> 1) & 1u, abort_flag)) { ok = false; break; }
         fence_after();
-        uint32_t sv[4][32];
+        const uint32_t sbase = lane_base + S_COL0 + (uint32_t)KB * sb;
+        uint32_t sv[NC][32];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + S_COL0 + 128u * s + 32u * c, sv[c]);
+        for (int c = 0; c < NC; ++c) tmem_ld32(sbase + 32u * c, sv[c]);
         tmem_wait_ld();
-        fence_before();
-        mbar_arrive(S_EMPTY(s));
-        const int k0 = j * BKV;
-        // Only the diagonal block and the block holding the sequence end need the mask: key
-        // valid iff key <= qrow and key < L (this branch is uniform over the CTA).
-        if (k0 + BKV - 1 > q0 || k0 + BKV > L) {
+        const int k0 = j * KB;
+        // Only the diagonal blocks and the block holding the sequence end need the mask: key
+        // valid iff key <= qrow and key < L (this branch is uniform over the CTA).  Within it a
+        // 32-key chunk is touched only where some row of the warp ends inside or before it.
+        if (k0 + KB - 1 > q0 || k0 + KB > L) {
           const int lim = min(qrow, L - 1) - k0;  // last valid column of this row
 #pragma unroll
-          for (int c = 0; c < 4; ++c)
+          for (int c = 0; c < NC; ++c)
+            if (__any_sync(0xffffffffu, lim < 32 * c + 31)) {
 #pragma unroll
-            for (int e = 0; e < 32; ++e)
-              if (32 * c + e > lim) sv[c][e] = __float_as_uint(-INFINITY);
+              for (int e = 0; e < 32; ++e)
+                if (32 * c + e > lim) sv[c][e] = __float_as_uint(-INFINITY);
+            }
         }
-        float mx = -INFINITY;
+        // row maximum over four independent chains of three-input maxima
+        float mc[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < NC; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(sv[c][e]));
+          for (int e = 0; e < 32; e += 2)
+            mc[(e >> 1) & 3] = max3(mc[(e >> 1) & 3], __uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1]));
+        float mx = max3(fmaxf(mc[0], mc[1]), mc[2], mc[3]);
         mx *= scale_log2;  // scale > 0: the maximum of the scaled scores
         float m_use = m, corr = 1.f;
         if (j == 0) {
@@ -353,75 +444,83 @@ __global__ void __launch_bounds__(THREADS, 1)
           corr = ex2(m - mx);
         }
         const float nb = (m_use == -INFINITY) ? 0.f : -m_use;  // p = 2^(s * scale - m)
-        float rs = 0.f;
-        uint32_t pk[64];
+        const uint64_t sc2 = f2(scale_log2, scale_log2), nb2 = f2(nb, nb);
+        uint64_t acc[4] = {0, 0, 0, 0};  // four independent pair sums (0 is +0.0f, +0.0f)
+        // P_g as packed fp16 over the first KB / 2 columns of S buffer sb, 32 keys (16 columns) at
+        // a time: chunk c lands in columns [16c, 16c + 16), whose S values are already in
+        // registers (PV_{g-2}, the previous reader of these columns, completed before S_g was
+        // issued)
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < NC; ++c) {
+          uint32_t pk[16];
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            const float p0 = ex2(fmaf(__uint_as_float(sv[c][e]), scale_log2, nb));
-            const float p1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), scale_log2, nb));
-            rs += p0 + p1;
-            pk[c * 16 + e / 2] = pack_half2(p0, p1);
+            const float2 x = unf2(fma2(f2(__uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1])), sc2, nb2));
+            const float p0 = ex2(x.x), p1 = ex2(x.y);
+            acc[(e >> 1) & 3] = add2(acc[(e >> 1) & 3], f2(p0, p1));
+            pk[e / 2] = pack_half2(p0, p1);
           }
-        // P buffer and O are free once the previous PV product completed
-        if (g > 0 && !mbar_wait(PV_DONE, (g - 1) & 1u, abort_flag)) { ok = false; break; }
-        fence_after();
+          tmem_st16(sbase + 16u * c, pk);
+        }
+        const float2 a01 = unf2(add2(acc[0], acc[1])), a23 = unf2(add2(acc[2], acc[3]));
+        const float rs = (a01.x + a01.y) + (a23.x + a23.y);
         if (__any_sync(0xffffffffu, corr != 1.f)) {  // rare: rescale this warp's O rows
+          // O must hold PV_{g-1} complete (j >= 1 here) before it is rescaled
+          if (!mbar_wait(BAR(PV_DONE, (g - 1) & 1), ((g - 1) >> 1) & 1u, abort_flag)) { ok = false; break; }
+          fence_after();
 #pragma unroll 1
           for (int c = 0; c < HD / 32; ++c) {
             uint32_t ov[32];
-            tmem_ld32(lane_base + 32u * c, ov);
+            tmem_ld32(o_base + 32u * c, ov);
             tmem_wait_ld();
 #pragma unroll
             for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
-            tmem_st32(lane_base + 32u * c, ov);
+            tmem_st32(o_base + 32u * c, ov);
           }
-          tmem_wait_st();
         }
         l = l * corr + rs;
         m = m_use;
-        // P row r: 16 chunks of 8 fp16; chunk c lives in key-atom c/8 at position (c%8)^(r%8)
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          uint8_t* dst = sP + (c >> 3) * (BQ * 128) + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
-          *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-        }
-        asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+        tmem_wait_st();
         fence_before();
-        mbar_arrive(P_FULL);
+        mbar_arrive(BAR(P_FULL, sb));
       }
       if (!ok) break;
       // output: wait for the item's last PV product, O / l
-      if (!mbar_wait(PV_DONE, (g - 1) & 1u, abort_flag)) break;
+      if (!mbar_wait(BAR(O_FULL, ob), (t / NO) & 1u, abort_flag)) break;
       fence_after();
       const float inv = 1.f / l;
-      uint16_t* dst = out + (size_t)(seq0 + qrow) * d + h * HD;
+      uint16_t* dst = out + (size_t)(cur.seq0 + qrow) * d + cur.h * HD;
+      const bool v8 = (reinterpret_cast<uintptr_t>(out) & 31u) == 0;  // rows then start on 32 B
 #pragma unroll 1
       for (int c = 0; c < HD / 32; ++c) {
         uint32_t ov[32];
-        tmem_ld32(lane_base + 32u * c, ov);
+        tmem_ld32(o_base + 32u * c, ov);
         tmem_wait_ld();
-        if (qrow < L) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * c);
+        uint32_t hv[16];
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            d4[q] = make_uint4(pack_half2(__uint_as_float(ov[8 * q]) * inv, __uint_as_float(ov[8 * q + 1]) * inv),
-                               pack_half2(__uint_as_float(ov[8 * q + 2]) * inv, __uint_as_float(ov[8 * q + 3]) * inv),
-                               pack_half2(__uint_as_float(ov[8 * q + 4]) * inv, __uint_as_float(ov[8 * q + 5]) * inv),
-                               pack_half2(__uint_as_float(ov[8 * q + 6]) * inv, __uint_as_float(ov[8 * q + 7]) * inv));
+        for (int q = 0; q < 16; ++q) hv[q] = pack_half2(__uint_as_float(ov[2 * q]) * inv, __uint_as_float(ov[2 * q + 1]) * inv);
+        if (qrow < L) {
+          if (v8) {  // one full 32-byte sector per row and store
+#pragma unroll
+            for (int q = 0; q < 2; ++q)
+              st_global_v8(dst + 32 * c + 16 * q, hv + 8 * q);
+          } else {
+            uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * c);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) d4[q] = make_uint4(hv[4 * q], hv[4 * q + 1], hv[4 * q + 2], hv[4 * q + 3]);
+          }
         }
       }
       fence_before();
-      mbar_arrive(O_EMPTY);
-      ++it_local;
+      mbar_arrive(BAR(O_EMPTY, ob));
+      ++t;
     }
   }
   fence_before();
   __syncthreads();
   if (warp == 1) {
     fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(CF::TMEM_COLS) : "memory");
   }
 }
 
@@ -477,47 +576,60 @@ void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, in
 
 int attention_max_qblocks(int max_T, int max_seqs) { return (max_T + fa::BQ - 1) / fa::BQ + max_seqs; }
 
+namespace {
+
+// Keys per block of the launched kernel shape (64: two CTAs per SM; 128: one).
+constexpr int kAttnKB = 64;
+
+template <int HD, int KB>
+int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const int* cu_seqlens, const int2* sched,
+                 int n_sched_max, int n_heads, float scale_log2, void* out, cudaStream_t st) {
+  using namespace fa;
+  using CF = Cfg<HD, KB>;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(attn_tc_kernel<HD, KB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)CF::SMEM) !=
+        cudaSuccess)
+      return 1;
+    attr = true;
+  }
+  const int items = n_sched_max * n_heads;
+  const int slots = CF::CTAS * sm_count();
+  const int grid = items < slots ? items : slots;
+  attn_tc_kernel<HD, KB><<<grid, THREADS, CF::SMEM, st>>>(mq, mkv, cu_seqlens, sched, n_sched_max, n_heads, scale_log2,
+                                                          static_cast<uint16_t*>(out));
+  return 0;
+}
+
+}  // namespace
+
 // qkv fp16 [T, 3 H hd] (q | k | v, heads contiguous), out fp16 [T, H hd].
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
                      const int2* sched, int n_sched_max, void* out, cudaStream_t st) {
   using namespace fa;
   (void)n_seq;
   if (T <= 0) return 0;
+  if (head_dim != 64 && head_dim != 128) return 1;
   auto fn = encode_fn();
   if (!fn) return 1;
   const int d = n_heads * head_dim;
-  CUtensorMap map;
-  cuuint64_t dims[2] = {(cuuint64_t)(3 * d), (cuuint64_t)T};
-  cuuint64_t strides[1] = {(cuuint64_t)(3 * d) * 2};
-  cuuint32_t box[2] = {64, (cuuint32_t)BQ};
-  cuuint32_t estr[2] = {1, 1};
-  if (fn(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(qkv), dims, strides, box, estr,
-         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-    return 1;
-  const float scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
-  const int items = n_sched_max * n_heads;
-  const int grid = items < sm_count() ? items : sm_count();
-  if (head_dim == 128) {
-    static bool attr = false;
-    if (!attr) {
-      cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
-      attr = true;
-    }
-    attn_tc_kernel<128><<<grid, THREADS, Cfg<128>::SMEM, st>>>(map, cu_seqlens, sched, n_sched_max, n_heads,
-                                                               scale_log2, static_cast<uint16_t*>(out));
-  } else if (head_dim == 64) {
-    static bool attr = false;
-    if (!attr) {
-      cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<64>::SMEM);
-      attr = true;
-    }
-    attn_tc_kernel<64><<<grid, THREADS, Cfg<64>::SMEM, st>>>(map, cu_seqlens, sched, n_sched_max, n_heads,
-                                                             scale_log2, static_cast<uint16_t*>(out));
-  } else {
-    return 1;
+  // Q tiles of 128 rows and K/V tiles of kAttnKB rows, each a 64-column (128-byte) box
+  CUtensorMap maps[2];
+  const cuuint32_t rows[2] = {(cuuint32_t)BQ, (cuuint32_t)kAttnKB};
+  for (int i = 0; i < 2; ++i) {
+    cuuint64_t dims[2] = {(cuuint64_t)(3 * d), (cuuint64_t)T};
+    cuuint64_t strides[1] = {(cuuint64_t)(3 * d) * 2};
+    cuuint32_t box[2] = {64, rows[i]};
+    cuuint32_t estr[2] = {1, 1};
+    if (fn(&maps[i], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(qkv), dims, strides, box, estr,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return 1;
   }
-  return 0;
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
+  if (head_dim == 128)
+    return launch_shape<128, kAttnKB>(maps[0], maps[1], cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out, st);
+  return launch_shape<64, kAttnKB>(maps[0], maps[1], cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out, st);
 }
 
 }  // namespace rift
