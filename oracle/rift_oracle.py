@@ -12,7 +12,9 @@ Each function restates one step of the paper in the paper's order:
   Section 2.3, Stage 2, Eq. 2 ......... U_i(c) = A_i(c) - lambda E_c,
                                          A_i(c) = p_i a+_c + (1 - p_i) a-_c, c* = argmax
   Section 2.3, Stage 2 ................ keep each retained tile's dominant tokens
-  Section 2.1 ......................... decoder prefill over [system | vision | query]
+  Section 2.1 ......................... decoder prefill over [system | vision | query],
+                                         the KV cache it builds, the last-token logits
+                                         and the decode step that follows it
 
 Precision.  Scores are computed in fp64 and rounded once to fp32; every
 decision (min-max, threshold, utility argmax, top-b order) is then taken in
@@ -44,6 +46,11 @@ Readings of points the paper leaves open (each also used by the CUDA path):
     0 .. L_i - 1, tiles in ascending index order.
   * Decoder: LLaMA block, RMSNorm (eps 1e-6), rotate-half RoPE (theta 1e4),
     causal softmax attention with scale 1/sqrt(head_dim), SwiGLU, final RMSNorm.
+  * KV cache: per layer, the keys after RoPE and the values, [L, H * head_dim]
+    with heads contiguous.  Logits: final hidden state of a sequence's last
+    token times the untied output matrix, [vocab, d].  Decode: one new token
+    per sequence at position L_i (the next after its prompt), attending to the
+    cached keys and values of its own sequence and to itself.
 """
 from __future__ import annotations
 
@@ -292,6 +299,78 @@ def decoder_layer(h: torch.Tensor, W: dict, dec, pos: torch.Tensor) -> torch.Ten
     x = rmsnorm(h, f["g_ffn"], dec.eps)
     h = h + (silu(x @ f["wg"].T) * (x @ f["wu"].T)) @ f["wd"].T
     return h
+
+
+def attention_with_past(q, k, v, n_past: int) -> torch.Tensor:
+    """Attention of n new rows (q: [n, H, hd]) over n_past cached rows followed by the new
+    rows themselves (k, v: [n_past + n, H, hd]): new row i sees keys 0 .. n_past + i."""
+    n, H, hd = q.shape
+    P = k.shape[0]
+    out = torch.empty_like(q)
+    key = torch.arange(P)[None, :]
+    mask = key > (n_past + torch.arange(n))[:, None]
+    for h in range(H):
+        sc = (q[:, h] @ k[:, h].T) / math.sqrt(hd)
+        sc = sc.masked_fill(mask, float("-inf"))
+        sc = sc - sc.max(dim=1, keepdim=True).values
+        p = torch.exp(sc)
+        p = p / p.sum(dim=1, keepdim=True)
+        out[:, h] = p @ v[:, h]
+    return out
+
+
+def decoder_layer_cached(h: torch.Tensor, W: dict, dec, pos: torch.Tensor, k_past=None, v_past=None):
+    """One decoder layer for new rows h at positions pos, given the layer's cached keys (after
+    RoPE) and values of the rows before them ([P, H, hd] each, or None).  Returns the new rows'
+    hidden states and their keys and values (the rows this layer appends to its cache)."""
+    n = h.shape[0]
+    f = {k: v.to(torch.float64) for k, v in W.items()}
+    x = rmsnorm(h, f["g_attn"], dec.eps)
+    q = (x @ f["wq"].T).view(n, dec.n_heads, dec.head_dim)
+    k = (x @ f["wk"].T).view(n, dec.n_heads, dec.head_dim)
+    v = (x @ f["wv"].T).view(n, dec.n_heads, dec.head_dim)
+    q, k = rope(q, pos, dec.rope_theta), rope(k, pos, dec.rope_theta)
+    n_past = 0 if k_past is None else k_past.shape[0]
+    k_all = k if k_past is None else torch.cat([k_past, k], 0)
+    v_all = v if v_past is None else torch.cat([v_past, v], 0)
+    a = attention_with_past(q, k_all, v_all, n_past).reshape(n, dec.d)
+    h = h + a @ f["wo"].T
+    x = rmsnorm(h, f["g_ffn"], dec.eps)
+    h = h + (silu(x @ f["wg"].T) * (x @ f["wu"].T)) @ f["wd"].T
+    return h, k, v
+
+
+def prefill_with_cache(H0_seq: torch.Tensor, get_layer, g_final, dec):
+    """Prefill of one sequence that also returns the KV cache it builds (Section 2.1): final
+    hidden states fp64 [L, d] and, per layer, (keys after RoPE, values) as fp64 [L, d]."""
+    h = H0_seq.to(torch.float64)
+    pos = torch.arange(h.shape[0])
+    cache = []
+    for l in range(dec.n_layers):
+        h, k, v = decoder_layer_cached(h, get_layer(l), dec, pos)
+        cache.append((k.reshape(-1, dec.d), v.reshape(-1, dec.d)))
+    return rmsnorm(h, g_final.to(torch.float64), dec.eps), cache
+
+
+def decode_token(x_emb: torch.Tensor, cache, get_layer, g_final, dec):
+    """One decode step of one sequence: the new token's input embedding x_emb [d] at position
+    P = len(cache rows), attending to the cached rows and itself.  Returns its final hidden
+    state fp64 [d] and, per layer, its (key after RoPE, value) rows fp64 [d]."""
+    h = x_emb.to(torch.float64)[None, :]
+    P = cache[0][0].shape[0]
+    pos = torch.tensor([P])
+    new = []
+    for l in range(dec.n_layers):
+        kp = cache[l][0].view(P, dec.n_heads, dec.head_dim)
+        vp = cache[l][1].view(P, dec.n_heads, dec.head_dim)
+        h, k, v = decoder_layer_cached(h, get_layer(l), dec, pos, kp, vp)
+        new.append((k.reshape(dec.d), v.reshape(dec.d)))
+    return rmsnorm(h, g_final.to(torch.float64), dec.eps)[0], new
+
+
+def logits(h_final: torch.Tensor, W_lm: torch.Tensor) -> torch.Tensor:
+    """Output logits of final hidden states h_final [..., d]: h W_lm^T with W_lm [vocab, d]."""
+    return h_final.to(torch.float64) @ W_lm.to(torch.float64).T
 
 
 def prefill_sequence(H0_seq: torch.Tensor, get_layer, g_final, dec) -> torch.Tensor:

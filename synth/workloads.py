@@ -267,3 +267,8 @@ def make_layer(dec: DecoderShape, layer: int, device="cpu", seed: int = 0) -> di
 
 def make_final_norm(dec: DecoderShape, device="cpu", seed: int = 0) -> torch.Tensor:
     return _weight(seed, "g_final", -1, (dec.d,), device)
+
+
+def make_lm_head(dec: DecoderShape, device="cpu", seed: int = 0) -> torch.Tensor:
+    """Untied output matrix [vocab, d] (LLaMA/Vicuna keep it separate from the embedding)."""
+    return _weight(seed, "lm_head", -1, (dec.vocab, dec.d), device)

@@ -350,3 +350,124 @@ def test_attention_matches_sdpa():
     ref = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1),
                                          is_causal=True).transpose(0, 1)
     assert torch.allclose(O.causal_attention(q, k, v), ref, atol=1e-13)
+
+
+# ------------------------------------------- KV cache, logits and the decode step (Section 2.1)
+
+def _textbook_prefill_kv(H0, layers, dec):
+    """The textbook formulation above, also returning each layer's keys (complex-number RoPE)
+    and values as [L, d]."""
+    h = H0.to(torch.float64)
+    L = h.shape[0]
+    hd, H = dec.head_dim, dec.n_heads
+    half = hd // 2
+    freqs = 1.0 / (dec.rope_theta ** (torch.arange(0, hd, 2, dtype=torch.float64) / hd))
+    rot = torch.polar(torch.ones(L, half, dtype=torch.float64), torch.outer(torch.arange(L, dtype=torch.float64), freqs))
+
+    def rope(x):
+        z = torch.complex(x[..., :half], x[..., half:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], dim=-1)
+
+    cache = []
+    for Wl in layers:
+        f = {k: v.to(torch.float64) for k, v in Wl.items()}
+        x = F.rms_norm(h, (dec.d,), f["g_attn"], dec.eps)
+        q = rope((x @ f["wq"].T).view(L, H, hd))
+        k = rope((x @ f["wk"].T).view(L, H, hd))
+        v = (x @ f["wv"].T).view(L, H, hd)
+        cache.append((k.reshape(L, dec.d), v.reshape(L, dec.d)))
+        a = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1),
+                                           is_causal=True).transpose(0, 1).reshape(L, dec.d)
+        h = h + a @ f["wo"].T
+        x = F.rms_norm(h, (dec.d,), f["g_ffn"], dec.eps)
+        h = h + (F.silu(x @ f["wg"].T) * (x @ f["wu"].T)) @ f["wd"].T
+    return cache
+
+
+def test_cached_prefill_matches_textbook_hidden_states_and_cache():
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    H0 = (torch.randn(23, dec.d, generator=torch.Generator().manual_seed(7))).to(torch.bfloat16)
+    out, cache = O.prefill_with_cache(H0, lambda l: layers[l], gf, dec)
+    assert torch.allclose(out, _textbook_prefill(H0, layers, gf, dec), rtol=0, atol=1e-10)
+    ref = _textbook_prefill_kv(H0, layers, dec)
+    assert len(cache) == dec.n_layers
+    for (k, v), (rk, rv) in zip(cache, ref):
+        assert k.shape == (23, dec.d) and v.shape == (23, dec.d)
+        assert torch.allclose(k, rk, rtol=0, atol=1e-12)
+        assert torch.allclose(v, rv, rtol=0, atol=1e-12)
+
+
+def test_decode_after_prefill_equals_the_longer_prefill():
+    # Prefill of L - 1 tokens, then one decode step with token L - 1, must give the same final
+    # hidden state and the same new cache rows as prefilling all L tokens at once: catches a
+    # wrong decode position, a dropped or duplicated cached row, or the new key left unrotated.
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    H0 = torch.randn(17, dec.d, generator=torch.Generator().manual_seed(8), dtype=torch.float64)
+    full, full_cache = O.prefill_with_cache(H0, lambda l: layers[l], gf, dec)
+    _, cache = O.prefill_with_cache(H0[:16], lambda l: layers[l], gf, dec)
+    h, new = O.decode_token(H0[16], cache, lambda l: layers[l], gf, dec)
+    assert torch.allclose(h, full[16], rtol=0, atol=1e-12)
+    for (k, v), (fk, fv) in zip(new, full_cache):
+        assert torch.allclose(k, fk[16], rtol=0, atol=1e-12)
+        assert torch.allclose(v, fv[16], rtol=0, atol=1e-12)
+
+
+def test_decode_of_the_second_token_by_hand():
+    # One layer, P = 1 cached row: the new row's attention is the 2-key softmax written out.
+    dec = W.DecoderShape(n_layers=1, d=64, n_heads=2, head_dim=32, ffn=96, vocab=50)
+    layers, gf = _tiny_layers(dec, seed=3)
+    f = {k: v.to(torch.float64) for k, v in layers[0].items()}
+    x0, x1 = torch.randn(2, dec.d, generator=torch.Generator().manual_seed(9), dtype=torch.float64)
+    _, cache = O.prefill_with_cache(x0[None], lambda l: layers[l], gf, dec)
+    h, _ = O.decode_token(x1, cache, lambda l: layers[l], gf, dec)
+
+    def nrm(v, g):
+        return v / math.sqrt(float((v * v).mean()) + dec.eps) * g
+
+    def rot(u, p):  # rotate-half RoPE of one head vector at position p
+        half = u.shape[0] // 2
+        ang = p * dec.rope_theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / u.shape[0])
+        return torch.cat([u[:half] * torch.cos(ang) - u[half:] * torch.sin(ang),
+                          u[half:] * torch.cos(ang) + u[:half] * torch.sin(ang)])
+
+    a0, a1 = nrm(x0, f["g_attn"]), nrm(x1, f["g_attn"])
+    att = []
+    for hh in range(dec.n_heads):
+        sl = slice(hh * 32, hh * 32 + 32)
+        q = rot((f["wq"] @ a1)[sl], 1)
+        k0, k1 = (f["wk"] @ a0)[sl], rot((f["wk"] @ a1)[sl], 1)
+        v0, v1 = (f["wv"] @ a0)[sl], (f["wv"] @ a1)[sl]
+        s0, s1 = float(q @ k0) / math.sqrt(32), float(q @ k1) / math.sqrt(32)
+        w0 = 1.0 / (1.0 + math.exp(s1 - s0))
+        att.append(w0 * v0 + (1.0 - w0) * v1)
+    r = x1 + f["wo"] @ torch.cat(att)
+    y = nrm(r, f["g_ffn"])
+    g = f["wg"] @ y
+    r = r + f["wd"] @ ((g / (1.0 + torch.exp(-g))) * (f["wu"] @ y))
+    assert torch.allclose(h, nrm(r, gf.to(torch.float64)), rtol=0, atol=1e-12)
+
+
+def test_attention_with_past_matches_masked_sdpa():
+    q = torch.randn(4, 3, 16, generator=torch.Generator().manual_seed(10), dtype=torch.float64)
+    k, v = (torch.randn(11, 3, 16, generator=torch.Generator().manual_seed(s), dtype=torch.float64) for s in (11, 12))
+    allowed = torch.arange(11)[None, :] <= (7 + torch.arange(4))[:, None]
+    ref = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1),
+                                         attn_mask=allowed).transpose(0, 1)
+    assert torch.allclose(O.attention_with_past(q, k, v, 7), ref, atol=1e-13)
+    assert torch.allclose(O.attention_with_past(q, k[:4], v[:4], 0), O.causal_attention(q, k[:4], v[:4]), atol=1e-14)
+
+
+def test_logits_select_rows_of_the_output_matrix():
+    # A permutation output matrix picks hidden coordinates: logits[r] = h[perm[r]]; a transposed
+    # operand would give h[perm^-1[r]] instead.
+    d = 12
+    perm = torch.randperm(d, generator=torch.Generator().manual_seed(13))
+    W_lm = torch.zeros(d, d, dtype=torch.float64)
+    W_lm[torch.arange(d), perm] = 1.0
+    h = torch.randn(3, d, generator=torch.Generator().manual_seed(14), dtype=torch.float64)
+    assert torch.equal(O.logits(h, W_lm), h[:, perm])
+    assert not torch.equal(h[:, perm], h[:, torch.argsort(perm)])
+    W2 = torch.randn(5, d, generator=torch.Generator().manual_seed(15), dtype=torch.float64)
+    assert torch.allclose(O.logits(h[0], W2), torch.stack([W2[r] @ h[0] for r in range(5)]), atol=1e-14)
