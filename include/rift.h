@@ -94,6 +94,8 @@ typedef struct {
  *              rows 16g..16g+15 (ffn must be a multiple of 16)
  *   w_down     [d, ffn]
  *   g_attn, g_ffn [d]    RMSNorm gains;  g_final [d] (one device pointer)
+ *   lm_head    [vocab, d] fp16, the untied output matrix (one device pointer), or NULL when no
+ *              call asks for logits; vocab % 8 == 0 when it is given
  * Requirements: d % 64 == 0, head_dim in {64, 128}, n_heads * head_dim == d. */
 typedef struct {
   int n_layers, d, n_heads, head_dim, ffn;
@@ -105,6 +107,8 @@ typedef struct {
   const void* const* g_attn;
   const void* const* g_ffn;
   const void* g_final;
+  int vocab;
+  const void* lm_head;
 } rift_model;
 
 /* Version of this ABI (bumped on any signature change). */
@@ -221,12 +225,37 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
  * Each layer: h += W_o Attn(RoPE(q), RoPE(k), v) with x = RMSNorm(h) g_attn, causal within
  * each sequence only; h += W_down(SiLU(W_gate x) * (W_up x)) with x = RMSNorm(h) g_ffn.
  * GEMM and attention operands are fp16 (normalised activations, q/k/v, softmax weights,
- * attention output, SwiGLU output), accumulation fp32, residual stream fp32. */
+ * attention output, SwiGLU output), accumulation fp32, residual stream fp32.
+ * Optional outputs (NULL = not written):
+ *   kv_out      fp16 [n_layers][2][T][d]: per layer the keys after RoPE ([l][0]) and the values
+ *               ([l][1]) of every packed row, heads contiguous: the KV cache the prefill builds
+ *               (Section 2.1), as rift_decode_step reads it.  16-byte aligned.
+ *   last_logits fp32 [n_seq, vocab]: logits of each sequence's last row,
+ *               (RMSNorm(h_last) g_final) lm_head^T; needs m->lm_head.  16-byte aligned. */
 size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len);
 rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 const int* cu_seqlens, int n_seq, int max_len,
-                                const int* positions,
+                                const int* positions, void* kv_out, float* last_logits,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
+
+/* ---- Decode step after the prefill (Section 2.1: decoding extends the prefilled KV cache one
+ * token at a time) ----
+ * One new token per sequence: sequence i's token token_ids[i] (an id into embed [vocab_embed, d]
+ * bf16) at position L_i = cu_seqlens[i+1] - cu_seqlens[i], attending to that sequence's cached
+ * rows and to itself, through every layer and the final RMSNorm.
+ *   kv_cache   fp16 [n_layers][2][T][d] as written by rift_prefill_layers (kv_out) for the
+ *              same cu_seqlens
+ *   max_len    an upper bound on every L_i + 1 (host int, at most 32768)
+ *   hidden_out bf16 [n_seq, d] final hidden states of the new tokens, or NULL
+ *   kv_new     fp16 [n_layers][2][n_seq][d] the new tokens' keys (after RoPE) and values, or NULL
+ *   logits     fp32 [n_seq, vocab] (needs m->lm_head), or NULL
+ * An id outside [0, vocab_embed) sets RIFT_ERR_BAD_ID (its row is computed from a zero
+ * embedding); L_i + 1 > max_len sets RIFT_ERR_CAPACITY or RIFT_ERR_BAD_ID. */
+size_t rift_decode_workspace_bytes(const rift_model* m, int n_seq, int max_len);
+rift_status rift_decode_step(const rift_model* m, const void* kv_cache, int T, const int* cu_seqlens,
+                             int n_seq, int max_len, const int* token_ids, const void* embed,
+                             int vocab_embed, void* hidden_out, void* kv_new, float* logits,
+                             void* ws, size_t ws_bytes, rift_stream_t stream);
 
 /* ---- The linear layer of a9 on its own (the GEMM every prefill layer runs four times) ----
  * out = A W^T with A fp16 [M, K], W fp16 [N, K] (both row-major, K contiguous), products

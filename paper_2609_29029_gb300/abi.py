@@ -38,7 +38,7 @@ class Model(C.Structure):
                 ("w_qkv", C.POINTER(C.c_void_p)), ("w_o", C.POINTER(C.c_void_p)),
                 ("w_gate_up", C.POINTER(C.c_void_p)), ("w_down", C.POINTER(C.c_void_p)),
                 ("g_attn", C.POINTER(C.c_void_p)), ("g_ffn", C.POINTER(C.c_void_p)),
-                ("g_final", C.c_void_p)]
+                ("g_final", C.c_void_p), ("vocab", C.c_int), ("lm_head", C.c_void_p)]
 
 
 _vp, _i, _f, _sz = C.c_void_p, C.c_int, C.c_float, C.c_size_t
@@ -56,7 +56,10 @@ SIGNATURES = {
     "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _i,
                               _vp, _vp, _vp, _vp]),
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
-    "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _sz, _vp]),
+    "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "rift_decode_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i]),
+    "rift_decode_step": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _sz,
+                              _vp]),
     "rift_score_tiles_noalloc": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp]),
     "rift_linear": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
     "rift_attention_workspace_bytes": (_sz, [_i, _i]),
@@ -192,10 +195,24 @@ def prefill_workspace_bytes(model: Model, max_T, max_seqs, max_len) -> int:
     return lib.rift_prefill_workspace_bytes(C.byref(model), max_T, max_seqs, max_len)
 
 
-def prefill_layers(model: Model, hidden, T, cu_seqlens, n_seq, max_len, positions, ws, ws_bytes, stream=None):
+def prefill_layers(model: Model, hidden, T, cu_seqlens, n_seq, max_len, positions, ws, ws_bytes, stream=None,
+                   kv_out=None, last_logits=None):
     _check(lib.rift_prefill_layers(C.byref(model), ptr(hidden), T, ptr(cu_seqlens), n_seq, max_len,
-                                   ptr(positions), ptr(ws), ws_bytes, stream_handle(stream)),
+                                   ptr(positions), ptr(kv_out), ptr(last_logits), ptr(ws), ws_bytes,
+                                   stream_handle(stream)),
            "rift_prefill_layers")
+
+
+def decode_workspace_bytes(model: Model, n_seq, max_len) -> int:
+    return lib.rift_decode_workspace_bytes(C.byref(model), n_seq, max_len)
+
+
+def decode_step(model: Model, kv_cache, T, cu_seqlens, n_seq, max_len, token_ids, embed, vocab_embed,
+                hidden_out, kv_new, logits, ws, ws_bytes, stream=None):
+    _check(lib.rift_decode_step(C.byref(model), ptr(kv_cache), T, ptr(cu_seqlens), n_seq, max_len, ptr(token_ids),
+                                ptr(embed), vocab_embed, ptr(hidden_out), ptr(kv_new), ptr(logits), ptr(ws), ws_bytes,
+                                stream_handle(stream)),
+           "rift_decode_step")
 
 
 def profile_enable(on: bool):

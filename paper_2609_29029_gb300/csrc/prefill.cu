@@ -9,7 +9,13 @@
 //   xn  = RMSNorm(h) g_ffn
 //   act = SiLU(xn W_g^T) * (xn W_u^T)            GEMM, SwiGLU epilogue (interleaved gate/up)
 //   h  += act W_down^T                           GEMM, fp32 residual epilogue
-// and finally hidden = RMSNorm(h) g_final in bf16.
+// and finally hidden = RMSNorm(h) g_final in bf16.  Optional outputs: each layer's keys (after
+// RoPE) and values copied out of the QKV buffer (the KV cache), and the logits of every
+// sequence's last token, RMSNorm(h_last) g_final times the output matrix.
+//
+// The decode step runs the same layer sequence for one new token per sequence, at position L_i,
+// with the attention replaced by decode_attn_kernel over the sequence's cached keys and values
+// plus the token's own.
 // fp16 rather than bf16 operands: after 32 layers the bf16 rounding of the GEMM inputs alone
 // moves the final hidden states by about 3% of their largest magnitude; fp16 (3 more mantissa
 // bits, same tensor-core rate, LLaVA-1.5-7B's checkpoint dtype) keeps the whole path near 0.5%.
@@ -90,6 +96,39 @@ __global__ void rope_table_kernel(float2* __restrict__ tab, int max_len, int hal
   tab[i] = make_float2((float)c, (float)s);
 }
 
+// KV cache rows: k_out[r] = qkv[r, d .. 2d), v_out[r] = qkv[r, 2d .. 3d) (fp16, heads contiguous).
+__global__ void kv_store_kernel(const uint16_t* __restrict__ qkv, int rows, int d, uint16_t* __restrict__ k_out,
+                                uint16_t* __restrict__ v_out) {
+  const int nv = d / 8;  // uint4 per row half
+  const size_t total = (size_t)rows * 2 * nv;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total; e += (size_t)gridDim.x * blockDim.x) {
+    const size_t r = e / (2 * nv);
+    const int c = (int)(e % (2 * nv));
+    const uint4 v = reinterpret_cast<const uint4*>(qkv + r * 3 * d + d)[c];
+    if (c < nv)
+      reinterpret_cast<uint4*>(k_out + r * d)[c] = v;
+    else
+      reinterpret_cast<uint4*>(v_out + r * d)[c - nv] = v;
+  }
+}
+
+static void kv_store(const uint16_t* qkv, int rows, int d, uint16_t* k_out, uint16_t* v_out, cudaStream_t st) {
+  const size_t total = (size_t)rows * (d / 4);
+  const int grid = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
+  kv_store_kernel<<<grid, 256, 0, st>>>(qkv, rows, d, k_out, v_out);
+}
+
+// out[i] = h32[cu[i + 1] - 1]: the residual stream of each sequence's last row (zeros for an
+// empty sequence).
+__global__ void last_rows_kernel(const float* __restrict__ h32, const int* __restrict__ cu, int d,
+                                 float* __restrict__ out) {
+  const int i = blockIdx.x;
+  const bool empty = cu[i + 1] <= cu[i];
+  const float4* src = reinterpret_cast<const float4*>(h32 + (size_t)(empty ? 0 : cu[i + 1] - 1) * d);
+  float4* dst = reinterpret_cast<float4*>(out + (size_t)i * d);
+  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) dst[c] = empty ? make_float4(0.f, 0.f, 0.f, 0.f) : src[c];
+}
+
 PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len) {
   PrefillLayout L{};
   size_t off = 0;
@@ -103,6 +142,8 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
   L.max_qblocks = attention_max_qblocks(max_T, max_seqs);
   L.sched_off = take((size_t)L.max_qblocks * sizeof(int2));
+  L.last32_off = take((size_t)max_seqs * m.d * 4);
+  L.last16_off = take((size_t)max_seqs * m.d * 2);
   L.total = off;
   return L;
 }
@@ -130,7 +171,8 @@ static void norm_launch(int kind, int T, const void* in, float* h32, const void*
 }
 
 int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                   int max_len, const int* positions, char* ws, cudaStream_t st) {
+                   int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
+                   cudaStream_t st) {
   if (T == 0) return 0;
   const PrefillLayout L = prefill_layout(m, T, n_seq, max_len);
   float* h32 = reinterpret_cast<float*>(ws + L.h32_off);
@@ -160,6 +202,10 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
     else
       norm_launch(1, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
     if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
+    if (kv_out) {
+      uint16_t* kl = static_cast<uint16_t*>(kv_out) + (size_t)l * 2 * T * d;
+      kv_store(qkv, T, d, kl, kl + (size_t)T * d, st);
+    }
     prof_begin(RIFT_PROF_ATTN, st);
     if (launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st)) return 1;
     prof_end(RIFT_PROF_ATTN, st, 1);
@@ -169,6 +215,231 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
     if (launch_gemm(act, m.w_down[l], T, d, m.ffn, EPI_RESID_F32, h32, st)) return 1;
   }
   norm_launch(2, T, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden), d, m.eps, st);
+  if (last_logits) {
+    float* last32 = reinterpret_cast<float*>(ws + L.last32_off);
+    uint16_t* last16 = reinterpret_cast<uint16_t*>(ws + L.last16_off);
+    last_rows_kernel<<<n_seq, 256, 0, st>>>(h32, cu_seqlens, d, last32);
+    norm_launch(1, n_seq, last32, nullptr, m.g_final, last16, d, m.eps, st);
+    if (launch_gemm(last16, m.lm_head, n_seq, m.vocab, d, EPI_STORE_F32, last_logits, st)) return 1;
+  }
+  return 0;
+}
+
+// ------------------------------------------------------------------------------------------
+// Decode step: one new token per sequence
+// ------------------------------------------------------------------------------------------
+
+DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len) {
+  DecodeLayout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
+  const size_t n = (size_t)(n_seq > 0 ? n_seq : 1);
+  L.h32_off = take(n * m.d * 4);
+  L.x0_off = take(n * m.d * 2);
+  L.xn_off = take(n * m.d * 2);
+  L.qkv_off = take(n * 3 * m.d * 2);
+  L.attn_off = take(n * m.d * 2);
+  L.act_off = take(n * m.ffn * 2);
+  L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
+  L.pos_off = take(n * sizeof(int));
+  L.total = off;
+  return L;
+}
+
+// x0[i] = embed[ids[i]] (bf16) and pos[i] = L_i = cu[i + 1] - cu[i], the new token's position.
+// An id outside [0, vocab) sets RIFT_EBIT_BADID and gives a zero row.
+__global__ void decode_embed_kernel(const int* __restrict__ ids, const int* __restrict__ cu,
+                                    const uint16_t* __restrict__ embed, int vocab, int d,
+                                    uint16_t* __restrict__ x0, int* __restrict__ pos) {
+  const int i = blockIdx.x;
+  const int id = ids[i];
+  const bool ok = id >= 0 && id < vocab;
+  if (threadIdx.x == 0) {
+    pos[i] = cu[i + 1] - cu[i];
+    if (!ok) atomicOr(&g_err_prefill, RIFT_EBIT_BADID);
+  }
+  uint4* dst = reinterpret_cast<uint4*>(x0 + (size_t)i * d);
+  const uint4* src = reinterpret_cast<const uint4*>(embed + (size_t)(ok ? id : 0) * d);
+  for (int c = threadIdx.x; c < d / 8; c += blockDim.x) dst[c] = ok ? src[c] : make_uint4(0, 0, 0, 0);
+}
+
+constexpr int DEC_THREADS = 128;
+
+// Attention of each sequence's new token over its P = L_i cached rows and itself: one CTA per
+// (sequence, head).  Scores go to shared memory (exact softmax, fp32), then every warp
+// accumulates p_j v_j over its share of the keys with lanes across head dims (one coalesced row
+// read per key) and the four partial sums are added.  A sequence with more than max_keys keys
+// sets RIFT_EBIT_CAPACITY and writes zeros.
+template <int HD>
+__global__ void __launch_bounds__(DEC_THREADS) decode_attn_kernel(const uint16_t* __restrict__ qkv,
+                                                                  const uint16_t* __restrict__ Kc,
+                                                                  const uint16_t* __restrict__ Vc,
+                                                                  const int* __restrict__ cu, int H,
+                                                                  float scale_log2, int max_keys,
+                                                                  uint16_t* __restrict__ out) {
+  constexpr int DPL = HD / 32;  // head dims per lane
+  constexpr int NW = DEC_THREADS / 32;
+  extern __shared__ float dsm[];
+  float* sc = dsm;                       // [max_keys] scores, then weights
+  float* part = dsm + max_keys;          // [NW][HD] partial outputs
+  float* red = part + NW * HD;           // [32] reductions
+  const int i = blockIdx.x / H, h = blockIdx.x % H;
+  const int d = H * HD;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int s0 = cu[i], P = cu[i + 1] - s0, nk = P + 1;
+  uint16_t* o = out + (size_t)i * d + h * HD;
+  if (nk > max_keys) {
+    if (threadIdx.x == 0) atomicOr(&g_err_prefill, RIFT_EBIT_CAPACITY);
+    if (threadIdx.x < HD) o[threadIdx.x] = 0;
+    return;
+  }
+  const uint16_t* self = qkv + (size_t)i * 3 * d + h * HD;  // q, then k at + d, v at + 2d
+  float q[DPL];
+#pragma unroll
+  for (int e = 0; e < DPL; ++e) q[e] = __half2float(__ushort_as_half(self[lane * DPL + e]));
+  auto key_row = [&](int j) { return j < P ? Kc + (size_t)(s0 + j) * d + h * HD : self + d; };
+  auto val_row = [&](int j) { return j < P ? Vc + (size_t)(s0 + j) * d + h * HD : self + 2 * d; };
+  auto load = [&](const uint16_t* row, float (&x)[DPL]) {
+    if constexpr (DPL == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(row + lane * 4);
+      const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
+      const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
+      x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
+    } else {
+      const float2 a = __half22float2(*reinterpret_cast<const __half2*>(row + lane * 2));
+      x[0] = a.x; x[1] = a.y;
+    }
+  };
+  // scores, four keys per warp in flight
+  for (int j0 = warp; j0 < nk; j0 += 4 * NW) {
+    float kx[4][DPL];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * NW;
+      if (j < nk) load(key_row(j), kx[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * NW;
+      float dot = 0.f;
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) dot = fmaf(q[e], kx[u][e], dot);
+      dot = warp_sum(dot);
+      if (lane == 0 && j < nk) sc[j] = dot * scale_log2;
+    }
+  }
+  __syncthreads();
+  float mx = -INFINITY;
+  for (int j = threadIdx.x; j < nk; j += DEC_THREADS) mx = fmaxf(mx, sc[j]);
+  mx = warp_max(mx);
+  if (lane == 0) red[warp] = mx;
+  __syncthreads();
+  mx = red[0];
+#pragma unroll
+  for (int w = 1; w < NW; ++w) mx = fmaxf(mx, red[w]);
+  float sum = 0.f;
+  for (int j = threadIdx.x; j < nk; j += DEC_THREADS) {
+    const float p = exp2f(sc[j] - mx);
+    sc[j] = p;
+    sum += p;
+  }
+  sum = block_sum(sum, red + 8);
+  // weighted values
+  float acc[DPL];
+#pragma unroll
+  for (int e = 0; e < DPL; ++e) acc[e] = 0.f;
+  for (int j0 = warp; j0 < nk; j0 += 4 * NW) {
+    float vx[4][DPL];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * NW;
+      if (j < nk) load(val_row(j), vx[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * NW;
+      if (j < nk) {
+        const float p = sc[j];
+#pragma unroll
+        for (int e = 0; e < DPL; ++e) acc[e] = fmaf(p, vx[u][e], acc[e]);
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < DPL; ++e) part[warp * HD + lane * DPL + e] = acc[e];
+  __syncthreads();
+  if (threadIdx.x < HD) {
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) v += part[w * HD + threadIdx.x];
+    o[threadIdx.x] = __half_as_ushort(__float2half_rn(v / sum));
+  }
+}
+
+int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* cu_seqlens, int n_seq, int max_len,
+                  const int* token_ids, const void* embed, int vocab_embed, void* hidden_out, void* kv_new,
+                  float* logits, char* ws, cudaStream_t st) {
+  if (n_seq == 0) return 0;
+  const DecodeLayout L = decode_layout(m, n_seq, max_len);
+  float* h32 = reinterpret_cast<float*>(ws + L.h32_off);
+  uint16_t* x0 = reinterpret_cast<uint16_t*>(ws + L.x0_off);
+  uint16_t* xn = reinterpret_cast<uint16_t*>(ws + L.xn_off);
+  uint16_t* qkv = reinterpret_cast<uint16_t*>(ws + L.qkv_off);
+  uint16_t* att = reinterpret_cast<uint16_t*>(ws + L.attn_off);
+  uint16_t* act = reinterpret_cast<uint16_t*>(ws + L.act_off);
+  float2* rope = reinterpret_cast<float2*>(ws + L.rope_off);
+  int* pos = reinterpret_cast<int*>(ws + L.pos_off);
+  const int d = m.d, half = m.head_dim / 2, n = n_seq;
+
+  rope_table_kernel<<<(max_len * half + 255) / 256, 256, 0, st>>>(rope, max_len, half, m.rope_theta);
+  decode_embed_kernel<<<n, 128, 0, st>>>(token_ids, cu_seqlens, static_cast<const uint16_t*>(embed), vocab_embed, d,
+                                         x0, pos);
+  EpiParams rope_ep;
+  rope_ep.positions = pos;
+  rope_ep.rope = rope;
+  rope_ep.rope_cols = 2 * d;
+  rope_ep.head_dim = m.head_dim;
+  rope_ep.max_len = max_len;
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)m.head_dim);
+  const size_t smem = ((size_t)max_len + 4 * m.head_dim + 64) * sizeof(float);
+  if (smem > 48 * 1024) {
+    if (smem > 200 * 1024) return 1;
+    if (m.head_dim == 128)
+      cudaFuncSetAttribute(decode_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    else
+      cudaFuncSetAttribute(decode_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  }
+  const uint16_t* kv = static_cast<const uint16_t*>(kv_cache);
+  for (int l = 0; l < m.n_layers; ++l) {
+    if (l == 0)
+      norm_launch(0, n, x0, h32, m.g_attn[0], xn, d, m.eps, st);
+    else
+      norm_launch(1, n, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
+    if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
+    if (kv_new) {
+      uint16_t* kl = static_cast<uint16_t*>(kv_new) + (size_t)l * 2 * n * d;
+      kv_store(qkv, n, d, kl, kl + (size_t)n * d, st);
+    }
+    const uint16_t* Kc = kv + (size_t)l * 2 * T * d;
+    const uint16_t* Vc = Kc + (size_t)T * d;
+    prof_begin(RIFT_PROF_ATTN, st);
+    if (m.head_dim == 128)
+      decode_attn_kernel<128><<<n * m.n_heads, DEC_THREADS, smem, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, scale_log2,
+                                                                        max_len, att);
+    else
+      decode_attn_kernel<64><<<n * m.n_heads, DEC_THREADS, smem, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, scale_log2,
+                                                                       max_len, att);
+    prof_end(RIFT_PROF_ATTN, st, 1);
+    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st)) return 1;
+    norm_launch(1, n, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
+    if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st)) return 1;
+    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st)) return 1;
+  }
+  if (hidden_out) norm_launch(2, n, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden_out), d, m.eps, st);
+  if (logits) {
+    norm_launch(1, n, h32, nullptr, m.g_final, xn, d, m.eps, st);
+    if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st)) return 1;
+  }
   return 0;
 }
 

@@ -98,7 +98,7 @@ rift_status rift_profile_read(double* ms, long long* launches, int n_classes) {
 
 long long rift_launch_count(void) { return g_launches.load(); }
 
-int rift_abi_version(void) { return 1; }
+int rift_abi_version(void) { return 2; }
 
 const char* rift_status_string(rift_status s) {
   switch (s) {
@@ -239,17 +239,48 @@ size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs
   return prefill_layout(*m, max_T, max_seqs, max_len).total;
 }
 
+static bool lm_head_ok(const rift_model* m) {
+  return m->lm_head && aligned16(m->lm_head) && m->vocab >= 8 && m->vocab % 8 == 0;
+}
+
 rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                                int max_len, const int* positions, void* ws, size_t ws_bytes,
-                                rift_stream_t stream) {
+                                int max_len, const int* positions, void* kv_out, float* last_logits, void* ws,
+                                size_t ws_bytes, rift_stream_t stream) {
   if (!model_ok(m) || !hidden || !cu_seqlens || !positions || T < 0 || n_seq < 0 || max_len < 1)
     return RIFT_ERR_INVALID;
   if (T > 0 && n_seq < 1) return RIFT_ERR_INVALID;
-  if (!aligned16(hidden)) return RIFT_ERR_INVALID;
+  if (!aligned16(hidden) || (kv_out && !aligned16(kv_out)) || (last_logits && !aligned16(last_logits)))
+    return RIFT_ERR_INVALID;
+  if (last_logits && !lm_head_ok(m)) return RIFT_ERR_INVALID;
   const size_t need = prefill_layout(*m, T, n_seq, max_len).total;
   if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
-  if (launch_prefill(*m, hidden, T, cu_seqlens, n_seq, max_len, positions, static_cast<char*>(ws),
-                     static_cast<cudaStream_t>(stream)))
+  if (launch_prefill(*m, hidden, T, cu_seqlens, n_seq, max_len, positions, kv_out, last_logits,
+                     static_cast<char*>(ws), static_cast<cudaStream_t>(stream)))
+    return RIFT_ERR_INVALID;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_decode_workspace_bytes(const rift_model* m, int n_seq, int max_len) {
+  if (!model_ok(m) || n_seq < 0 || max_len < 1 || max_len > 32768) return 0;
+  return decode_layout(*m, n_seq, max_len).total;
+}
+
+rift_status rift_decode_step(const rift_model* m, const void* kv_cache, int T, const int* cu_seqlens, int n_seq,
+                             int max_len, const int* token_ids, const void* embed, int vocab_embed,
+                             void* hidden_out, void* kv_new, float* logits, void* ws, size_t ws_bytes,
+                             rift_stream_t stream) {
+  if (!model_ok(m) || !kv_cache || !cu_seqlens || !token_ids || !embed || T < 0 || n_seq < 0 || max_len < 1 ||
+      max_len > 32768 || vocab_embed < 1)
+    return RIFT_ERR_INVALID;
+  if (!aligned16(kv_cache) || !aligned16(embed) || (hidden_out && !aligned16(hidden_out)) ||
+      (kv_new && !aligned16(kv_new)) || (logits && !aligned16(logits)))
+    return RIFT_ERR_INVALID;
+  if (logits && !lm_head_ok(m)) return RIFT_ERR_INVALID;
+  const size_t need = decode_layout(*m, n_seq, max_len).total;
+  if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
+  if (launch_decode(*m, kv_cache, T, cu_seqlens, n_seq, max_len, token_ids, embed, vocab_embed, hidden_out, kv_new,
+                    logits, static_cast<char*>(ws), static_cast<cudaStream_t>(stream)))
     return RIFT_ERR_INVALID;
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;

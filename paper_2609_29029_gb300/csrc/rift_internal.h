@@ -45,12 +45,20 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
 
 // ---- prefill (prefill.cu, gemm.cu, attention.cu) ----
 struct PrefillLayout {
-  size_t h32_off, xn_off, qkv_off, attn_off, act_off, rope_off, sched_off, total;
+  size_t h32_off, xn_off, qkv_off, attn_off, act_off, rope_off, sched_off, last32_off, last16_off, total;
   int max_qblocks;
 };
 PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len);
 int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                   int max_len, const int* positions, char* ws, cudaStream_t st);
+                   int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
+                   cudaStream_t st);
+struct DecodeLayout {
+  size_t h32_off, x0_off, xn_off, qkv_off, attn_off, act_off, rope_off, pos_off, total;
+};
+DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len);
+int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* cu_seqlens, int n_seq, int max_len,
+                  const int* token_ids, const void* embed, int vocab_embed, void* hidden_out, void* kv_new,
+                  float* logits, char* ws, cudaStream_t st);
 
 // GEMM: C[M, N] = A[M, K] . B[N, K]^T (fp16 operands, fp32 accumulation) + epilogue.
 enum GemmEpilogue {

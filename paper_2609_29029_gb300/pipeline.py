@@ -28,7 +28,7 @@ class DeviceModel:
     unless their magnitude is below 2^-14, where fp16 keeps 2^-24 absolute resolution).  Norm
     gains stay bf16."""
 
-    def __init__(self, dec, layers: list, g_final: torch.Tensor, device="cuda"):
+    def __init__(self, dec, layers: list, g_final: torch.Tensor, device="cuda", lm_head: torch.Tensor | None = None):
         self.dec = dec
         self.layers = []
         h = torch.float16
@@ -53,6 +53,9 @@ class DeviceModel:
         m.w_gate_up, m.w_down = self._ptrs["gate_up"], self._ptrs["down"]
         m.g_attn, m.g_ffn = self._ptrs["g_attn"], self._ptrs["g_ffn"]
         m.g_final = self.g_final.data_ptr()
+        self.lm_head = None if lm_head is None else lm_head.to(device).to(h).contiguous()
+        m.vocab = 0 if lm_head is None else lm_head.shape[0]
+        m.lm_head = None if lm_head is None else self.lm_head.data_ptr()
         self.struct = m
 
 
@@ -146,11 +149,21 @@ class ScenePipeline:
         abi.sync_status(s)
         return int(self.counts_host[0]), int(self.counts_host[1])
 
-    def prefill(self, T, n_seq, stream=None):
-        """a9: decoder prefill over the packed batch, in place."""
+    def prefill(self, T, n_seq, stream=None, kv_out=None, last_logits=None):
+        """a9: decoder prefill over the packed batch, in place; optionally the KV cache
+        (fp16 [n_layers, 2, T, d]) and the last-token logits (fp32 [n_seq, vocab])."""
         ws, need = self._prefill_ws(T, n_seq)
         abi.prefill_layers(self.model.struct, self.packed, T, self.cu, n_seq, self.max_len, self.positions, ws,
-                           need, stream)
+                           need, stream, kv_out=kv_out, last_logits=last_logits)
+
+    def decode(self, kv_cache, T, n_seq, token_ids, embed, hidden_out=None, kv_new=None, logits=None,
+               stream=None):
+        """One decode step after the prefill: token_ids[i] appended to sequence i."""
+        max_len = self.max_len + 1
+        need = abi.decode_workspace_bytes(self.model.struct, n_seq, max_len)
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=self.device)
+        abi.decode_step(self.model.struct, kv_cache, T, self.cu, n_seq, max_len, token_ids, embed, embed.shape[0],
+                        hidden_out, kv_new, logits, ws, need, stream)
 
     def run(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, prefill=True, stream=None):
         self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)

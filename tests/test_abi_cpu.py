@@ -31,7 +31,7 @@ def test_library_exports_every_declared_symbol(riftlib):
 def test_status_strings(riftlib):
     assert riftlib.status_string(0) == "ok"
     assert riftlib.status_string(riftlib.RIFT_ERR_CAPACITY) == "output capacity exceeded"
-    assert riftlib.abi_version() == 1
+    assert riftlib.abi_version() == 2
 
 
 FAKE = 0x10000  # a 16-byte aligned non-null address; validation rejects before using it
@@ -110,7 +110,43 @@ def test_pack_and_prefill_reject_bad_arguments(riftlib):
     m.head_dim = 96
     assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0
     m.head_dim, m.ffn = 64, 690
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, None, FAKE, 1 << 30, 0) == INV
+    m.ffn = 688
+    # last-token logits need an output matrix; optional outputs must be 16-byte aligned
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, FAKE + 8, None, FAKE, 1 << 30, 0) == INV
+    m.vocab, m.lm_head = 1000, FAKE
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE + 4, FAKE, 1 << 30, 0) == INV
+    m.vocab = 1001  # not a multiple of 8
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
+
+
+def test_decode_rejects_bad_arguments(riftlib):
+    lib = riftlib.lib
+    INV = riftlib.RIFT_ERR_INVALID
+    m = riftlib.Model()
+    m.n_layers, m.d, m.n_heads, m.head_dim, m.ffn, m.eps, m.rope_theta = 2, 256, 4, 64, 688, 1e-6, 1e4
+    arr = (C.c_void_p * 2)(FAKE, FAKE)
+    for f in ("w_qkv", "w_o", "w_gate_up", "w_down", "g_attn", "g_ffn"):
+        setattr(m, f, arr)
+    m.g_final = FAKE
+    ws = lib.rift_decode_workspace_bytes(C.byref(m), 3, 100)
+    assert ws > 0
+    assert lib.rift_decode_workspace_bytes(C.byref(m), 3, 40000) == 0     # max_len above 32768
+    assert lib.rift_decode_workspace_bytes(C.byref(m), -1, 100) == 0
+
+    def call(**kw):
+        a = dict(kv=FAKE, T=10, cu=FAKE, n=3, max_len=100, ids=FAKE, embed=FAKE, ve=50, hid=FAKE, kvn=None,
+                 lg=None, ws=FAKE, wsb=ws)
+        a.update(kw)
+        return lib.rift_decode_step(C.byref(m), a["kv"], a["T"], a["cu"], a["n"], a["max_len"], a["ids"], a["embed"],
+                                    a["ve"], a["hid"], a["kvn"], a["lg"], a["ws"], a["wsb"], 0)
+
+    assert call(kv=None) == INV and call(ids=None) == INV and call(embed=None) == INV
+    assert call(max_len=0) == INV and call(max_len=40000) == INV and call(ve=0) == INV
+    assert call(kv=FAKE + 2) == INV and call(hid=FAKE + 8) == INV
+    assert call(lg=FAKE) == INV                   # logits without an output matrix
+    assert call(wsb=ws - 1) == INV                # workspace too small
 
 
 def test_query_prep_rejects_bad_arguments(riftlib):
