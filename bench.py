@@ -25,7 +25,7 @@ sys.path.insert(0, str(ROOT))
 
 import torch  # noqa: E402
 
-from synth import workloads as W  # noqa: E402
+from synth import rng, workloads as W  # noqa: E402
 
 METRIC = "retained prefill tokens/s"
 UNIT = "tokens/s"
@@ -40,10 +40,11 @@ def parse():
     ap.add_argument("--impl", default="rift", choices=["rift", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode-step measurement")
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
-    ap.add_argument("--kernel-case", choices=["prefill", "score"],
+    ap.add_argument("--kernel-case", choices=["prefill", "score", "decode"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
                          "'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); each runs 3 times")
     return ap.parse_args()
@@ -308,6 +309,61 @@ def sweep(steps: int, warmup: int):
         torch.cuda.empty_cache()
 
 
+def decode_measure(pipe, dm, sc, dec, n_kept, T, stream, steps):
+    """The first decode step after the prefill (Section 2.1), timed on its own: the prefill runs
+    once more writing its KV cache, then `steps` decode steps of one seeded token per retained
+    tile.  Reported beside the prefill metric (not part of it), with its HBM roofline: every
+    weight, the output matrix and the whole KV cache are read once per step."""
+    from paper_2609_29029_gb300 import abi
+    dev = sc.X.device
+    d = dec.d
+    pipe.run(sc.X, sc.embed, *(torch.tensor(v, dtype=torch.int32, device=dev)
+                               for v in (sc.query_ids, sc.bg_ids, sc.sys_ids, sc.query_ids)),
+             prefill=False, stream=stream)
+    kv = torch.empty(dec.n_layers, 2, T, d, dtype=torch.float16, device=dev)
+    last = torch.empty(n_kept, dec.vocab, dtype=torch.float32, device=dev)
+    pipe.prefill(T, n_kept, stream, kv_out=kv, last_logits=last)
+    key = rng.stream_key(0, rng.stream_id("bench-decode"))
+    ids = torch.tensor([rng.hash_u32_int(key, i) % dec.vocab for i in range(n_kept)], dtype=torch.int32, device=dev)
+    hid = torch.empty(n_kept, d, dtype=torch.bfloat16, device=dev)
+    lg = torch.empty(n_kept, dec.vocab, dtype=torch.float32, device=dev)
+    max_len = pipe.max_len + 1
+    need = abi.decode_workspace_bytes(dm.struct, n_kept, max_len)
+    ws = torch.empty(need, dtype=torch.uint8, device=dev)
+
+    def one():
+        abi.decode_step(dm.struct, kv, T, pipe.cu, n_kept, max_len, ids, sc.embed, sc.embed.shape[0], hid, None, lg,
+                        ws, need, stream)
+
+    for _ in range(3):
+        one()
+    abi.sync_status(stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    abi.sync_status(stream)
+    ms = e0.elapsed_time(e1) / steps
+    abi.profile_enable(True)  # per-class breakdown, in a separate untimed pass
+    for _ in range(steps):
+        one()
+    torch.cuda.synchronize()
+    abi.profile_enable(False)
+    breakdown = {k: round(v[0] / steps, 3) for k, v in abi.profile_read().items() if v[1]}
+    weights = dec.n_layers * dec.params_per_layer * 2 + dec.vocab * d * 2
+    kv_bytes = dec.n_layers * 2 * T * d * 2
+    peaks = json.loads((ROOT / "MEASURED_PEAKS.json").read_text()) if (ROOT / "MEASURED_PEAKS.json").exists() else {}
+    hbm = peaks.get("hbm_gbs", 6800.0)
+    gbs = (weights + kv_bytes) / (ms / 1e3) / 1e9
+    del kv
+    torch.cuda.empty_cache()
+    return {"ms": ms, "tokens_per_s": n_kept / (ms / 1e3), "sequences": n_kept, "cached_rows": T,
+            "kernels_ms": breakdown, "algorithmic_bytes": weights + kv_bytes, "achieved_gbs": gbs, "peak_gbs": hbm, "frac_hbm": gbs / hbm,
+            "bound": "hbm", "inputs": "seeded token ids; KV cache from the prefill of the same query"}
+
+
 def kernel_case(name: str):
     """Small cases for ncu captures: inputs larger than L2, about 1 GB on the device."""
     import __graft_entry__
@@ -328,6 +384,26 @@ def kernel_case(name: str):
         for _ in range(3):
             hid = H0.clone()
             abi.prefill_layers(dm.struct, hid, T, cu, len(lens), 635, pos, ws, need)
+        abi.sync_status()
+    elif name == "decode":
+        # 4 layers of the 7B shape, 73 sequences of 130..635 cached rows (about the retained set
+        # of the 400-tile query), a random fp16 KV cache: three decode steps
+        dec = W.DecoderShape(n_layers=4, d=4096, n_heads=32, head_dim=128, ffn=11008, vocab=32000)
+        dm = DeviceModel(dec, [W.make_layer(dec, l, dev) for l in range(dec.n_layers)], W.make_final_norm(dec, dev),
+                         dev, lm_head=W.make_lm_head(dec, dev))
+        lens = [35 + 24 + (72, 144, 288, 432, 576)[i % 5] for i in range(73)]
+        T, n = sum(lens), len(lens)
+        cu = torch.tensor([0] + [sum(lens[:i + 1]) for i in range(n)], dtype=torch.int32, device=dev)
+        from synth import rng
+        kv = rng.normal_f32(0, rng.stream_id("case-kv"), dec.n_layers * 2 * T * dec.d, dev).to(torch.float16)
+        embed = rng.normal_f32(0, rng.stream_id("case-embed"), 1024 * dec.d, dev).view(1024, dec.d).to(torch.bfloat16)
+        ids = torch.arange(n, dtype=torch.int32, device=dev)
+        hid = torch.empty(n, dec.d, dtype=torch.bfloat16, device=dev)
+        lg = torch.empty(n, dec.vocab, dtype=torch.float32, device=dev)
+        need = abi.decode_workspace_bytes(dm.struct, n, 636)
+        ws = torch.empty(need, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            abi.decode_step(dm.struct, kv, T, cu, n, 636, ids, embed, 1024, hid, None, lg, ws, need)
         abi.sync_status()
     else:
         wl = W.sweep_workload(64)
@@ -366,7 +442,7 @@ def main():
     s, dec = wl.scene, wl.decoder
     sc = W.make_scene(s, dec.vocab, dev)
     layers = [W.make_layer(dec, l, dev) for l in range(dec.n_layers)]
-    dm = DeviceModel(dec, layers, W.make_final_norm(dec, dev), dev)
+    dm = DeviceModel(dec, layers, W.make_final_norm(dec, dev), dev, lm_head=W.make_lm_head(dec, dev))
     del layers
     pipe = ScenePipeline(s.N, s.n_v, s.d, s.x_dtype, s.M, s.S, s.Q, wl.knn_m, wl.policy, model=dm, device=dev)
     i32 = dict(dtype=torch.int32, device=dev)
@@ -451,6 +527,7 @@ def main():
     e2e_val, _ = job_throughput(float(Te * args.e2e_steps), f0.elapsed_time(f1), ws)
     h2d_bytes = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
     d2h = Te * s.d * 2 + 8
+    decode = None if args.no_decode else decode_measure(pipe, dm, sc, dec, n_kept, T, stream, args.steps)
 
     if rank != 0:
         return
@@ -491,6 +568,7 @@ def main():
                      "launches": gemm_n},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h},
+        "decode_step": decode,
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }

@@ -12,6 +12,10 @@
 // Two accumulators let the epilogue of one tile overlap the main loop of the next.  Tiles are
 // visited in bands of M-tiles whose A rows fit in L2 (48 MB), so each weight tile is read from
 // DRAM once per band.
+// Split-K (for few rows, where the tiles alone would leave most SMs idle, as in the decode
+// step): the work units are (tile, K-slice) pairs, each unit stores its fp32 partial product
+// into a caller workspace, and splitk_reduce_kernel sums the slices in a fixed order and
+// applies the epilogue.
 // Every mbarrier wait is bounded (RIFT_SPIN_LIMIT iterations, ~4 s of globaltimer): on timeout
 // the kernel sets RIFT_EBIT_TIMEOUT, lets every role fall through, waits for its issued copies
 // and frees its tensor memory.
@@ -243,7 +247,7 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, void* C, const EpiParams ep, int group_m) {
+                   int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -284,16 +288,24 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   const int mt = (M + BM - 1) / BM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
   const int n_tiles = mt * nt;
+  // unit u: tile u / splits, K-blocks [k0, k1) of slice u % splits (the host makes every slice
+  // non-empty)
+  const int n_units = n_tiles * splits, k_per = (kt + splits - 1) / splits;
+  auto unit_k = [&](int u, int& k0, int& k1) {
+    k0 = (u % splits) * k_per;
+    k1 = min(kt, k0 + k_per);
+  };
 
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer
       int it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        int m_blk, n_blk;
-        tile_coords(tile, mt, nt, group_m, m_blk, n_blk);
-        for (int k = 0; k < kt; ++k, ++it) {
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        int m_blk, n_blk, k0, k1;
+        tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
+        unit_k(u, k0, k1);
+        for (int k = k0; k < k1; ++k, ++it) {
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
           if (!mbar_wait(empty_bar(s), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
@@ -316,13 +328,15 @@ __global__ void __launch_bounds__(THREADS, 1)
       // ---------------- MMA issuer
       int it = 0, tl = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tl) {
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++tl) {
+        int k0, k1;
+        unit_k(u, k0, k1);
         const int b = tl & 1;
         const uint32_t use = tl >> 1;
         if (!mbar_wait(tempty_bar(b), (use & 1u) ^ 1u, abort_flag)) break;
         fence_after();
         const uint32_t tmem_d = tmem_base + (uint32_t)(b * ACC_COLS);
-        for (int k = 0; k < kt; ++k, ++it) {
+        for (int k = k0; k < k1; ++k, ++it) {
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
           if (!mbar_wait(full_bar(s), round & 1u, abort_flag)) { ok = false; break; }
@@ -331,7 +345,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t bd = smem_desc(smem_u32(sB + s * B_BYTES));
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along K per step (encoded >> 4)
-            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k | kk) != 0 ? 1u : 0u);
+            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k != k0 || kk != 0) ? 1u : 0u);
           umma_commit(empty_bar(s));
         }
         if (ok) umma_commit(tfull_bar(b));
@@ -341,9 +355,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     // ---------------- epilogue (warps 2..5 -> TMEM lane quarters 2, 3, 0, 1)
     const int quarter = warp & 3;
     int tl = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++tl) {
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++tl) {
       int m_blk, n_blk;
-      tile_coords(tile, mt, nt, group_m, m_blk, n_blk);
+      tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
+      // split-K partials (EPI_STORE_F32 only): slice u % splits at C + slice * split_stride
+      void* Cu = splits > 1 ? static_cast<void*>(static_cast<float*>(C) + (size_t)(u % splits) * split_stride) : C;
       const int b = tl & 1;
       const uint32_t use = tl >> 1;
       if (!mbar_wait(tfull_bar(b), use & 1u, abort_flag)) break;
@@ -376,7 +392,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld32(taddr + c, r);
-          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, C, ep.out_scale);
+          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, Cu, ep.out_scale);
         }
       }
       fence_before();
@@ -434,28 +450,94 @@ static int sm_count() {
 
 template <int EPI>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
-                  cudaStream_t st) {
+                  cudaStream_t st, int splits = 1) {
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
     attr = true;
   }
-  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-  const int grid = tiles < sm_count() ? tiles : sm_count();
+  const int units = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * splits;
+  const int grid = units < sm_count() ? units : sm_count();
   // Band height: as many M-tiles as keep the band's A rows within ~48 MB of L2 (8..64), so each
   // weight tile is streamed from DRAM once per band.
   int group_m = (int)((48u << 20) / ((size_t)BM * K * 2));
   group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep, group_m);
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep, group_m, splits, (size_t)M * N);
   return 0;
 }
 
-}  // namespace tc
+// Sum of the split-K slices (in slice order) and the epilogue EPI, one output element per thread
+// and step: the same arithmetic as epilogue_chunk / rope_chunk on the summed accumulator.
+template <int EPI>
+__global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, int M, int N, void* C,
+                                     const EpiParams ep) {
+  const size_t stride = (size_t)M * N;
+  const int n_out = EPI == EPI_SWIGLU ? N / 2 : N;
+  const size_t total = (size_t)M * n_out;
+  auto acc = [&](int row, int col) {
+    float v = 0.f;
+    for (int sp = 0; sp < splits; ++sp) v += part[sp * stride + (size_t)row * N + col];
+    return v;
+  };
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total; e += (size_t)gridDim.x * blockDim.x) {
+    const int row = (int)(e / n_out), col = (int)(e % n_out);
+    if constexpr (EPI == EPI_STORE_F32) {
+      static_cast<float*>(C)[e] = acc(row, col) * ep.out_scale;
+    } else if constexpr (EPI == EPI_RESID_F32) {
+      static_cast<float*>(C)[e] += acc(row, col);
+    } else if constexpr (EPI == EPI_STORE_BF16) {
+      static_cast<__half*>(C)[e] = __float2half_rn(acc(row, col));
+    } else if constexpr (EPI == EPI_SWIGLU) {  // output f: gate column 32 (f / 16) + f % 16, up 16 further
+      const int gc = 32 * (col / 16) + col % 16;
+      static_cast<__half*>(C)[e] = __float2half_rn(silu(acc(row, gc)) * acc(row, gc + 16));
+    } else if constexpr (EPI == EPI_QKV_ROPE) {
+      float y = acc(row, col);
+      if (col < ep.rope_cols) {
+        const int half = ep.head_dim >> 1, j = col % ep.head_dim;
+        const int pos = ep.positions[row];
+        if (pos < 0 || pos >= ep.max_len) {
+          if (j == 0) atomicOr(&g_err_gemm, RIFT_EBIT_BADID);
+          continue;  // as the fused epilogue: q and k of a row without a valid position stay unwritten
+        }
+        const float2 cs = ep.rope[(size_t)pos * half + (j < half ? j : j - half)];
+        if (j < half)
+          y = y * cs.x - acc(row, col + half) * cs.y;
+        else
+          y = y * cs.x + acc(row, col - half) * cs.y;
+      }
+      static_cast<__half*>(C)[e] = __float2half_rn(y);
+    }
+  }
+}
+
+// Split count for an M x N x K product whose tiles leave SMs idle: the K-slice count (1..16, at
+// least 4 K-blocks a slice, partials within the workspace) that minimises the makespan, i.e. the
+// rounds of units over the SMs times the K-blocks of a slice.  1 = no split.
+static int choose_splits(int M, int N, int K, size_t ws_bytes) {
+  const int sms = sm_count();
+  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN), kt = (K + BK - 1) / BK;
+  if (tiles >= sms) return 1;
+  int best = 1;
+  long best_cost = (long)((tiles + sms - 1) / sms) * kt;
+  for (int s = 2; s <= 16 && kt / s >= 4; ++s) {
+    if ((size_t)s * M * N * sizeof(float) > ws_bytes) break;
+    const int per = (kt + s - 1) / s;
+    const int se = (kt + per - 1) / per;  // every slice non-empty
+    const long cost = (long)((tiles * se + sms - 1) / sms) * per;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = se;
+    }
+  }
+  return best;
+}
+
+}  // namespace tc}  // namespace tc
 
 // Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
 // the RoPE epilogue), A, B and C 16-byte aligned.
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st) {
+                   cudaStream_t st, void* split_ws, size_t split_ws_bytes) {
   using namespace tc;
   if (M <= 0 || N <= 0 || K <= 0) return 0;
   if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
@@ -463,6 +545,22 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     return 1;
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
+  const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
+  if (splits > 1) {
+    if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits)) return 1;
+    const float* part = static_cast<const float*>(split_ws);
+    const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N);
+    const int grid = (int)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048);
+    switch (epi) {
+      case EPI_STORE_BF16: splitk_reduce_kernel<EPI_STORE_BF16><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+      case EPI_RESID_F32: splitk_reduce_kernel<EPI_RESID_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+      case EPI_SWIGLU: splitk_reduce_kernel<EPI_SWIGLU><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+      case EPI_QKV_ROPE: splitk_reduce_kernel<EPI_QKV_ROPE><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+      case EPI_STORE_F32: splitk_reduce_kernel<EPI_STORE_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+      default: return 1;
+    }
+    return 0;
+  }
   switch (epi) {
     case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, ep, st);
     case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, ep, st);

@@ -149,9 +149,9 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
 }
 
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st,
-                const EpiParams& ep) {
+                const EpiParams& ep, void* split_ws, size_t split_ws_bytes) {
   prof_begin(RIFT_PROF_GEMM, st);
-  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, ep, st);
+  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, ep, st, split_ws, split_ws_bytes);
   prof_end(RIFT_PROF_GEMM, st, 1);
   return r;
 }
@@ -229,6 +229,9 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
 // Decode step: one new token per sequence
 // ------------------------------------------------------------------------------------------
 
+constexpr int DEC_CHUNK = 128;  // keys per decode-attention work unit
+constexpr int DEC_HG = 8;       // heads per decode-attention CTA (one warp each)
+
 DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len) {
   DecodeLayout L{};
   size_t off = 0;
@@ -242,6 +245,17 @@ DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len) {
   L.act_off = take(n * m.ffn * 2);
   L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
   L.pos_off = take(n * sizeof(int));
+  // decode attention partials: (m, l, o[head_dim]) per (sequence, key chunk, head)
+  L.dpart_off = take(n * (size_t)((max_len + DEC_CHUNK - 1) / DEC_CHUNK) * m.n_heads * (m.head_dim + 2) * 4);
+  // split-K partial products of the few-row GEMMs: up to 16 slices of [min(n, 128), widest
+  // output] fp32, at most 128 MB
+  const size_t rows = n < 128 ? n : 128;
+  size_t widest = (size_t)3 * m.d;
+  if ((size_t)2 * m.ffn > widest) widest = (size_t)2 * m.ffn;
+  if (m.lm_head && (size_t)m.vocab > widest) widest = (size_t)m.vocab;
+  L.split_bytes = 16 * rows * widest * 4;
+  if (L.split_bytes > (size_t)128 << 20) L.split_bytes = (size_t)128 << 20;
+  L.split_off = take(L.split_bytes);
   L.total = off;
   return L;
 }
@@ -263,116 +277,139 @@ __global__ void decode_embed_kernel(const int* __restrict__ ids, const int* __re
   for (int c = threadIdx.x; c < d / 8; c += blockDim.x) dst[c] = ok ? src[c] : make_uint4(0, 0, 0, 0);
 }
 
-constexpr int DEC_THREADS = 128;
 
-// Attention of each sequence's new token over its P = L_i cached rows and itself: one CTA per
-// (sequence, head).  Scores go to shared memory (exact softmax, fp32), then every warp
-// accumulates p_j v_j over its share of the keys with lanes across head dims (one coalesced row
-// read per key) and the four partial sums are added.  A sequence with more than max_keys keys
-// sets RIFT_EBIT_CAPACITY and writes zeros.
+// Attention of each sequence's new token over its P = L_i cached rows and itself, split like
+// flash decoding: CTA (sequence i, chunk c of DEC_CHUNK keys, group of hg heads: the largest of
+// 8, 4, 2, 1 that divides H), one warp per head.  A key row's hg head slices are hg * head_dim * 2
+// contiguous bytes, read together by the CTA's warps.  Lanes read 16 bytes (8 head dims) each, so
+// one warp-wide load covers KPL = 256 / head_dim keys, LPK = head_dim / 8 lanes per key; each
+// lane group keeps its own running maximum m, sum l and output o over its keys (online softmax,
+// fp32, log2 units) and the groups are merged at the end of the chunk.  (m, l, o) of the chunk go
+// to `part`, and decode_combine_kernel merges a sequence's chunks.  Units past a sequence's last
+// key exit at once.
 template <int HD>
-__global__ void __launch_bounds__(DEC_THREADS) decode_attn_kernel(const uint16_t* __restrict__ qkv,
-                                                                  const uint16_t* __restrict__ Kc,
-                                                                  const uint16_t* __restrict__ Vc,
-                                                                  const int* __restrict__ cu, int H,
-                                                                  float scale_log2, int max_keys,
-                                                                  uint16_t* __restrict__ out) {
-  constexpr int DPL = HD / 32;  // head dims per lane
-  constexpr int NW = DEC_THREADS / 32;
-  extern __shared__ float dsm[];
-  float* sc = dsm;                       // [max_keys] scores, then weights
-  float* part = dsm + max_keys;          // [NW][HD] partial outputs
-  float* red = part + NW * HD;           // [32] reductions
-  const int i = blockIdx.x / H, h = blockIdx.x % H;
-  const int d = H * HD;
+__global__ void __launch_bounds__(DEC_HG * 32, 3) decode_attn_kernel(const uint16_t* __restrict__ qkv,
+                                                                     const uint16_t* __restrict__ Kc,
+                                                                     const uint16_t* __restrict__ Vc,
+                                                                     const int* __restrict__ cu, int H, int hg,
+                                                                     int max_chunks, float scale_log2,
+                                                                     float* __restrict__ part) {
+  constexpr int LPK = HD / 8, KPL = 32 / LPK;  // lanes per key, keys per warp-wide load
+  constexpr int NL = 4;                        // warp-wide loads of K (and of V) in flight
+  const int groups = H / hg;  // hg = blockDim.x / 32 heads per CTA
+  const int g = blockIdx.x % groups, c = (blockIdx.x / groups) % max_chunks, i = blockIdx.x / (groups * max_chunks);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = g * hg + warp;
+  const int d = H * HD;
   const int s0 = cu[i], P = cu[i + 1] - s0, nk = P + 1;
-  uint16_t* o = out + (size_t)i * d + h * HD;
-  if (nk > max_keys) {
-    if (threadIdx.x == 0) atomicOr(&g_err_prefill, RIFT_EBIT_CAPACITY);
-    if (threadIdx.x < HD) o[threadIdx.x] = 0;
-    return;
-  }
+  const int j_begin = c * DEC_CHUNK, j_end = min(nk, j_begin + DEC_CHUNK);
+  if (j_begin >= nk) return;
+  const int sub = lane / LPK, dl = (lane % LPK) * 8;  // key within a load, first head dim of the lane
   const uint16_t* self = qkv + (size_t)i * 3 * d + h * HD;  // q, then k at + d, v at + 2d
-  float q[DPL];
+  auto unpack = [](const uint4& u, float (&x)[8]) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-  for (int e = 0; e < DPL; ++e) q[e] = __half2float(__ushort_as_half(self[lane * DPL + e]));
-  auto key_row = [&](int j) { return j < P ? Kc + (size_t)(s0 + j) * d + h * HD : self + d; };
-  auto val_row = [&](int j) { return j < P ? Vc + (size_t)(s0 + j) * d + h * HD : self + 2 * d; };
-  auto load = [&](const uint16_t* row, float (&x)[DPL]) {
-    if constexpr (DPL == 4) {
-      const uint2 u = *reinterpret_cast<const uint2*>(row + lane * 4);
-      const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
-      const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
-      x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
-    } else {
-      const float2 a = __half22float2(*reinterpret_cast<const __half2*>(row + lane * 2));
-      x[0] = a.x; x[1] = a.y;
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[e]));
+      x[2 * e] = f.x;
+      x[2 * e + 1] = f.y;
     }
   };
-  // scores, four keys per warp in flight
-  for (int j0 = warp; j0 < nk; j0 += 4 * NW) {
-    float kx[4][DPL];
+  float q[8];
+  unpack(__ldg(reinterpret_cast<const uint4*>(self + dl)), q);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = j0 + u * NW;
-      if (j < nk) load(key_row(j), kx[u]);
+  for (int e = 0; e < 8; ++e) q[e] *= scale_log2;  // scores in log2 units
+  float m = -INFINITY, l = 0.f, acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+  for (int j0 = j_begin; j0 < j_end; j0 += NL * KPL) {
+    uint4 kr[NL], vr[NL];
+#pragma unroll
+    for (int u = 0; u < NL; ++u) {  // rows past the chunk end read the last row, weight 0
+      const int j = min(j0 + u * KPL + sub, j_end - 1);
+      const size_t r = (size_t)(s0 + j) * d + h * HD + dl;
+      kr[u] = __ldg(reinterpret_cast<const uint4*>(j < P ? Kc + r : self + d + dl));
+      vr[u] = __ldg(reinterpret_cast<const uint4*>(j < P ? Vc + r : self + 2 * d + dl));
     }
+    float sc[NL];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = j0 + u * NW;
+    for (int u = 0; u < NL; ++u) {
+      float kx[8];
+      unpack(kr[u], kx);
       float dot = 0.f;
 #pragma unroll
-      for (int e = 0; e < DPL; ++e) dot = fmaf(q[e], kx[u][e], dot);
-      dot = warp_sum(dot);
-      if (lane == 0 && j < nk) sc[j] = dot * scale_log2;
+      for (int e = 0; e < 8; ++e) dot = fmaf(q[e], kx[e], dot);
+#pragma unroll
+      for (int o = LPK / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      sc[u] = (j0 + u * KPL + sub < j_end) ? dot : -INFINITY;
     }
-  }
-  __syncthreads();
-  float mx = -INFINITY;
-  for (int j = threadIdx.x; j < nk; j += DEC_THREADS) mx = fmaxf(mx, sc[j]);
-  mx = warp_max(mx);
-  if (lane == 0) red[warp] = mx;
-  __syncthreads();
-  mx = red[0];
+    float mx = m;
 #pragma unroll
-  for (int w = 1; w < NW; ++w) mx = fmaxf(mx, red[w]);
-  float sum = 0.f;
-  for (int j = threadIdx.x; j < nk; j += DEC_THREADS) {
-    const float p = exp2f(sc[j] - mx);
-    sc[j] = p;
-    sum += p;
-  }
-  sum = block_sum(sum, red + 8);
-  // weighted values
-  float acc[DPL];
+    for (int u = 0; u < NL; ++u) mx = fmaxf(mx, sc[u]);
+    // a lane group whose keys are all past the end keeps m = -inf (mx = -inf): nothing to add
+    const float corr = mx == -INFINITY ? 1.f : exp2f(m - mx);
+    l *= corr;
 #pragma unroll
-  for (int e = 0; e < DPL; ++e) acc[e] = 0.f;
-  for (int j0 = warp; j0 < nk; j0 += 4 * NW) {
-    float vx[4][DPL];
+    for (int e = 0; e < 8; ++e) acc[e] *= corr;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = j0 + u * NW;
-      if (j < nk) load(val_row(j), vx[u]);
+    for (int u = 0; u < NL; ++u) {
+      const float p = mx == -INFINITY ? 0.f : exp2f(sc[u] - mx);
+      float vx[8];
+      unpack(vr[u], vx);
+      l += p;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = fmaf(p, vx[e], acc[e]);
     }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = j0 + u * NW;
-      if (j < nk) {
-        const float p = sc[j];
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) acc[e] = fmaf(p, vx[u][e], acc[e]);
-      }
-    }
+    m = mx;
   }
+  // merge the KPL lane groups (lanes l, l + LPK, ... hold the same head dims)
 #pragma unroll
-  for (int e = 0; e < DPL; ++e) part[warp * HD + lane * DPL + e] = acc[e];
-  __syncthreads();
-  if (threadIdx.x < HD) {
-    float v = 0.f;
+  for (int o = LPK; o < 32; o <<= 1) {
+    const float mo = __shfl_xor_sync(0xffffffffu, m, o), lo = __shfl_xor_sync(0xffffffffu, l, o);
+    const float M = fmaxf(m, mo);
+    const float fa = m == -INFINITY ? 0.f : exp2f(m - M), fb = mo == -INFINITY ? 0.f : exp2f(mo - M);
+    l = l * fa + lo * fb;
 #pragma unroll
-    for (int w = 0; w < NW; ++w) v += part[w * HD + threadIdx.x];
-    o[threadIdx.x] = __half_as_ushort(__float2half_rn(v / sum));
+    for (int e = 0; e < 8; ++e) acc[e] = acc[e] * fa + __shfl_xor_sync(0xffffffffu, acc[e], o) * fb;
+    m = M;
+  }
+  float* dst = part + (((size_t)i * max_chunks + c) * H + h) * (HD + 2);
+  if (lane == 0) {
+    dst[0] = m;
+    dst[1] = l;
+  }
+  if (lane < LPK) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) dst[2 + dl + e] = acc[e];
+  }
+}
+
+// out[i, h] = sum_c o_c 2^(m_c - M) / sum_c l_c 2^(m_c - M), chunks in order (M = max_c m_c).
+// A sequence with more than max_keys keys sets RIFT_EBIT_CAPACITY and gets zeros.
+__global__ void decode_combine_kernel(const float* __restrict__ part, const int* __restrict__ cu, int H, int HD,
+                                      int max_chunks, int max_keys, uint16_t* __restrict__ out) {
+  const int i = blockIdx.x / H, h = blockIdx.x % H;
+  const int nk = cu[i + 1] - cu[i] + 1;
+  uint16_t* o = out + ((size_t)i * H + h) * HD;
+  if (nk > max_keys) {
+    if (threadIdx.x == 0) atomicOr(&g_err_prefill, RIFT_EBIT_CAPACITY);
+    for (int e = threadIdx.x; e < HD; e += blockDim.x) o[e] = 0;
+    return;
+  }
+  const int nch = (nk + DEC_CHUNK - 1) / DEC_CHUNK;
+  const float* p0 = part + ((size_t)i * max_chunks * H + h) * (HD + 2);
+  const size_t cstride = (size_t)H * (HD + 2);
+  float M = -INFINITY;
+  for (int c = 0; c < nch; ++c) M = fmaxf(M, p0[c * cstride]);
+  for (int e = threadIdx.x; e < HD; e += blockDim.x) {
+    float L = 0.f, v = 0.f;
+    for (int c = 0; c < nch; ++c) {
+      const float* pc = p0 + c * cstride;
+      const float f = exp2f(pc[0] - M);
+      L += pc[1] * f;
+      v += pc[2 + e] * f;
+    }
+    o[e] = __half_as_ushort(__float2half_rn(v / L));
   }
 }
 
@@ -389,6 +426,12 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
   uint16_t* act = reinterpret_cast<uint16_t*>(ws + L.act_off);
   float2* rope = reinterpret_cast<float2*>(ws + L.rope_off);
   int* pos = reinterpret_cast<int*>(ws + L.pos_off);
+  void* split = ws + L.split_off;
+  const size_t sb = L.split_bytes;
+  float* dpart = reinterpret_cast<float*>(ws + L.dpart_off);
+  const int max_chunks = (max_len + DEC_CHUNK - 1) / DEC_CHUNK;
+  int hg = DEC_HG;
+  while (m.n_heads % hg != 0) hg /= 2;
   const int d = m.d, half = m.head_dim / 2, n = n_seq;
 
   rope_table_kernel<<<(max_len * half + 255) / 256, 256, 0, st>>>(rope, max_len, half, m.rope_theta);
@@ -401,21 +444,13 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
   rope_ep.head_dim = m.head_dim;
   rope_ep.max_len = max_len;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)m.head_dim);
-  const size_t smem = ((size_t)max_len + 4 * m.head_dim + 64) * sizeof(float);
-  if (smem > 48 * 1024) {
-    if (smem > 200 * 1024) return 1;
-    if (m.head_dim == 128)
-      cudaFuncSetAttribute(decode_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    else
-      cudaFuncSetAttribute(decode_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  }
   const uint16_t* kv = static_cast<const uint16_t*>(kv_cache);
   for (int l = 0; l < m.n_layers; ++l) {
     if (l == 0)
       norm_launch(0, n, x0, h32, m.g_attn[0], xn, d, m.eps, st);
     else
       norm_launch(1, n, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
-    if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
+    if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep, split, sb)) return 1;
     if (kv_new) {
       uint16_t* kl = static_cast<uint16_t*>(kv_new) + (size_t)l * 2 * n * d;
       kv_store(qkv, n, d, kl, kl + (size_t)n * d, st);
@@ -423,22 +458,25 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
     const uint16_t* Kc = kv + (size_t)l * 2 * T * d;
     const uint16_t* Vc = Kc + (size_t)T * d;
     prof_begin(RIFT_PROF_ATTN, st);
+    const int units = n * max_chunks * (m.n_heads / hg);
     if (m.head_dim == 128)
-      decode_attn_kernel<128><<<n * m.n_heads, DEC_THREADS, smem, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, scale_log2,
-                                                                        max_len, att);
+      decode_attn_kernel<128><<<units, hg * 32, 0, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, hg, max_chunks, scale_log2,
+                                                         dpart);
     else
-      decode_attn_kernel<64><<<n * m.n_heads, DEC_THREADS, smem, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, scale_log2,
-                                                                       max_len, att);
-    prof_end(RIFT_PROF_ATTN, st, 1);
-    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st)) return 1;
+      decode_attn_kernel<64><<<units, hg * 32, 0, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, hg, max_chunks, scale_log2,
+                                                        dpart);
+    decode_combine_kernel<<<n * m.n_heads, m.head_dim, 0, st>>>(dpart, cu_seqlens, m.n_heads, m.head_dim, max_chunks,
+                                                                max_len, att);
+    prof_end(RIFT_PROF_ATTN, st, 2);
+    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st, EpiParams(), split, sb)) return 1;
     norm_launch(1, n, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
-    if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st)) return 1;
-    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st)) return 1;
+    if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st, EpiParams(), split, sb)) return 1;
+    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st, EpiParams(), split, sb)) return 1;
   }
   if (hidden_out) norm_launch(2, n, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden_out), d, m.eps, st);
   if (logits) {
     norm_launch(1, n, h32, nullptr, m.g_final, xn, d, m.eps, st);
-    if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st)) return 1;
+    if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st, EpiParams(), split, sb)) return 1;
   }
   return 0;
 }

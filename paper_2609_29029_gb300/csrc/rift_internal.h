@@ -53,7 +53,8 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
                    int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
                    cudaStream_t st);
 struct DecodeLayout {
-  size_t h32_off, x0_off, xn_off, qkv_off, attn_off, act_off, rope_off, pos_off, total;
+  size_t h32_off, x0_off, xn_off, qkv_off, attn_off, act_off, rope_off, pos_off, dpart_off, split_off, split_bytes,
+      total;
 };
 DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len);
 int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* cu_seqlens, int n_seq, int max_len,
@@ -76,10 +77,13 @@ struct EpiParams {
   int max_len = 0;
   float out_scale = 1.f;           // EPI_STORE_F32
 };
+// split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
+// most SMs idle run as (tile, K-slice) units plus a reduction kernel.
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
-                cudaStream_t st, const EpiParams& ep = EpiParams());
+                cudaStream_t st, const EpiParams& ep = EpiParams(), void* split_ws = nullptr,
+                size_t split_ws_bytes = 0);
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st);
+                   cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0);
 
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].

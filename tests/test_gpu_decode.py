@@ -119,3 +119,50 @@ def test_decode_flags_bad_ids_and_short_max_len(cuda, riftlib):
     st = riftlib.lib.rift_decode_step(riftlib.C.byref(dm.struct), kv.data_ptr(), T, cu.data_ptr(), 2, 11,
                                       ids.data_ptr(), embed.data_ptr(), 20, None, None, 1, ws.data_ptr(), need, None)
     assert st == riftlib.RIFT_ERR_INVALID                        # misaligned logits pointer
+
+
+# d = 1024 with 4 heads of 128 and one layer: every GEMM of the decode step (a few rows) runs
+# split-K (QKV with RoPE 4 slices, W_o 4, gate/up with SwiGLU 4, W_down 11, output matrix 4),
+# the prefill's GEMMs do not.
+MID = W.DecoderShape(n_layers=1, d=1024, n_heads=8, head_dim=128, ffn=2816, vocab=4096)
+
+
+def test_split_k_decode_on_a_synthetic_batch(cuda, riftlib):
+    dec = MID
+    dm, layers, gf, lm = _model(dec, cuda)
+    lens = [5, 64, 130]
+    T, n, d = sum(lens), len(lens), dec.d
+    cu = [0, 5, 69, T]
+    H0 = rng.normal_f32(11, rng.stream_id("mid-batch"), T * d, cuda).view(T, d).to(torch.bfloat16)
+    hidden = H0.clone()
+    cu_d = torch.tensor(cu, dtype=torch.int32, device=cuda)
+    pos_d = torch.cat([torch.arange(L, dtype=torch.int32, device=cuda) for L in lens])
+    kv = torch.empty(dec.n_layers, 2, T, d, dtype=torch.float16, device=cuda)
+    last = torch.empty(n, dec.vocab, dtype=torch.float32, device=cuda)
+    max_len = max(lens) + 1
+    need = riftlib.prefill_workspace_bytes(dm.struct, T, n, max_len)
+    ws = torch.empty(need, dtype=torch.uint8, device=cuda)
+    riftlib.prefill_layers(dm.struct, hidden, T, cu_d, n, max_len, pos_d, ws, need, kv_out=kv, last_logits=last)
+    embed = rng.normal_f32(12, rng.stream_id("mid-embed"), 300 * d, cuda).view(300, d).to(torch.bfloat16)
+    ids = _token_ids(n, 300, 2)
+    hid = torch.empty(n, d, dtype=torch.bfloat16, device=cuda)
+    kvn = torch.empty(dec.n_layers, 2, n, d, dtype=torch.float16, device=cuda)
+    lg = torch.empty(n, dec.vocab, dtype=torch.float32, device=cuda)
+    need = riftlib.decode_workspace_bytes(dm.struct, n, max_len)
+    ws = torch.empty(need, dtype=torch.uint8, device=cuda)
+    riftlib.decode_step(dm.struct, kv, T, cu_d, n, max_len, torch.tensor(ids, dtype=torch.int32, device=cuda),
+                        embed, 300, hid, kvn, lg, ws, need)
+    riftlib.sync_status()
+    get = lambda l: layers[l]
+    worst = {}
+    for j in range(n):
+        h_ref, cache = O.prefill_with_cache(H0[cu[j]:cu[j + 1]].cpu(), get, gf, dec)
+        hd, new = O.decode_token(embed[ids[j]].cpu(), cache, get, gf, dec)
+        errs = [_rel(hidden[cu[j]:cu[j + 1]], h_ref), _rel(last[j], O.logits(h_ref[-1], lm)),
+                _rel(hid[j], hd), _rel(lg[j], O.logits(hd, lm))]
+        for l in range(dec.n_layers):
+            errs += [_rel(kv[l, 0, cu[j]:cu[j + 1]], cache[l][0]), _rel(kv[l, 1, cu[j]:cu[j + 1]], cache[l][1]),
+                     _rel(kvn[l, 0, j], new[l][0]), _rel(kvn[l, 1, j], new[l][1])]
+        worst[j] = max(errs)
+    print("worst", worst)
+    assert max(worst.values()) < P.HIDDEN_TOL, worst
