@@ -466,32 +466,58 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   return 0;
 }
 
-// Sum of the split-K slices (in slice order) and the epilogue EPI, one output element per thread
-// and step: the same arithmetic as epilogue_chunk / rope_chunk on the summed accumulator.
+// Sum of the split-K slices (in slice order) and the epilogue EPI, four consecutive outputs per
+// thread and step (float4 partial reads): the same arithmetic as epilogue_chunk / rope_chunk on
+// the summed accumulator.  N % 8 == 0, so a group of four never straddles a row, a SwiGLU
+// 16-column group or a RoPE half.
 template <int EPI>
 __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, int M, int N, void* C,
                                      const EpiParams ep) {
   const size_t stride = (size_t)M * N;
   const int n_out = EPI == EPI_SWIGLU ? N / 2 : N;
-  const size_t total = (size_t)M * n_out;
-  auto acc = [&](int row, int col) {
-    float v = 0.f;
-    for (int sp = 0; sp < splits; ++sp) v += part[sp * stride + (size_t)row * N + col];
+  const int q_out = n_out / 4;
+  const size_t total = (size_t)M * q_out;
+  auto acc4 = [&](int row, int col) {
+    const float* p = part + (size_t)row * N + col;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int sp = 0; sp < splits; ++sp) {
+      const float4 f = *reinterpret_cast<const float4*>(p + sp * stride);
+      v.x += f.x;
+      v.y += f.y;
+      v.z += f.z;
+      v.w += f.w;
+    }
     return v;
   };
+  auto store_h4 = [](void* dst, float a, float b, float c, float d) {
+    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_half2(a, b), pack_half2(c, d));
+  };
   for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total; e += (size_t)gridDim.x * blockDim.x) {
-    const int row = (int)(e / n_out), col = (int)(e % n_out);
+    const int row = (int)(e / q_out), col = (int)(e % q_out) * 4;
     if constexpr (EPI == EPI_STORE_F32) {
-      static_cast<float*>(C)[e] = acc(row, col) * ep.out_scale;
+      const float4 v = acc4(row, col);
+      *reinterpret_cast<float4*>(static_cast<float*>(C) + (size_t)row * N + col) =
+          make_float4(v.x * ep.out_scale, v.y * ep.out_scale, v.z * ep.out_scale, v.w * ep.out_scale);
     } else if constexpr (EPI == EPI_RESID_F32) {
-      static_cast<float*>(C)[e] += acc(row, col);
+      const float4 v = acc4(row, col);
+      float4* o = reinterpret_cast<float4*>(static_cast<float*>(C) + (size_t)row * N + col);
+      float4 r = *o;
+      r.x += v.x;
+      r.y += v.y;
+      r.z += v.z;
+      r.w += v.w;
+      *o = r;
     } else if constexpr (EPI == EPI_STORE_BF16) {
-      static_cast<__half*>(C)[e] = __float2half_rn(acc(row, col));
-    } else if constexpr (EPI == EPI_SWIGLU) {  // output f: gate column 32 (f / 16) + f % 16, up 16 further
+      const float4 v = acc4(row, col);
+      store_h4(static_cast<uint16_t*>(C) + (size_t)row * N + col, v.x, v.y, v.z, v.w);
+    } else if constexpr (EPI == EPI_SWIGLU) {  // outputs f..f+3: gate column 32 (f / 16) + f % 16, up 16 further
       const int gc = 32 * (col / 16) + col % 16;
-      static_cast<__half*>(C)[e] = __float2half_rn(silu(acc(row, gc)) * acc(row, gc + 16));
+      const float4 g = acc4(row, gc), u = acc4(row, gc + 16);
+      store_h4(static_cast<uint16_t*>(C) + (size_t)row * n_out + col, silu(g.x) * u.x, silu(g.y) * u.y,
+               silu(g.z) * u.z, silu(g.w) * u.w);
     } else if constexpr (EPI == EPI_QKV_ROPE) {
-      float y = acc(row, col);
+      float4 y = acc4(row, col);
       if (col < ep.rope_cols) {
         const int half = ep.head_dim >> 1, j = col % ep.head_dim;
         const int pos = ep.positions[row];
@@ -499,13 +525,58 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits,
           if (j == 0) atomicOr(&g_err_gemm, RIFT_EBIT_BADID);
           continue;  // as the fused epilogue: q and k of a row without a valid position stay unwritten
         }
-        const float2 cs = ep.rope[(size_t)pos * half + (j < half ? j : j - half)];
-        if (j < half)
-          y = y * cs.x - acc(row, col + half) * cs.y;
-        else
-          y = y * cs.x + acc(row, col - half) * cs.y;
+        const float2* cs = ep.rope + (size_t)pos * half + (j < half ? j : j - half);
+        const float4 x = acc4(row, j < half ? col + half : col - half);  // the partner dims
+        const float sg = j < half ? -1.f : 1.f;  // first half: x cos - x' sin; second: x cos + x' sin
+        y = make_float4(y.x * cs[0].x + sg * x.x * cs[0].y, y.y * cs[1].x + sg * x.y * cs[1].y,
+                        y.z * cs[2].x + sg * x.z * cs[2].y, y.w * cs[3].x + sg * x.w * cs[3].y);
       }
-      static_cast<__half*>(C)[e] = __float2half_rn(y);
+      store_h4(static_cast<uint16_t*>(C) + (size_t)row * N + col, y.x, y.y, y.z, y.w);
+    }
+  }
+}
+
+// The residual add of a split-K product fused with the RMSNorm that follows it: one CTA per row,
+// h[row] += sum of the slices (in slice order), then out[row] = fp16(h / sqrt(mean(h^2) + eps) g)
+// with the bf16 gain g (the arithmetic of the standalone RMSNorm kernel).  N % 4 == 0, N <= 8192.
+__global__ void __launch_bounds__(256) splitk_resid_norm_kernel(const float* __restrict__ part, int splits, int M,
+                                                                int N, float* __restrict__ h32,
+                                                                const uint16_t* __restrict__ gain, float eps,
+                                                                uint16_t* __restrict__ out) {
+  __shared__ float red[32];
+  const size_t row = blockIdx.x, stride = (size_t)M * N;
+  const int nv = N / 4;
+  float4 v[8];
+  float ss = 0.f;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const int c = threadIdx.x + q * 256;
+    if (c < nv) {
+      float4 a = reinterpret_cast<const float4*>(h32 + row * N)[c];
+      const float4* p = reinterpret_cast<const float4*>(part + row * N) + c;
+#pragma unroll 4
+      for (int sp = 0; sp < splits; ++sp) {
+        const float4 f = p[sp * stride / 4];
+        a.x += f.x;
+        a.y += f.y;
+        a.z += f.z;
+        a.w += f.w;
+      }
+      reinterpret_cast<float4*>(h32 + row * N)[c] = a;
+      v[q] = a;
+      ss += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+    }
+  }
+  const float inv = rsqrtf(block_sum(ss, red) / (float)N + eps);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const int c = threadIdx.x + q * 256;
+    if (c < nv) {
+      const uint2 gr = reinterpret_cast<const uint2*>(gain)[c];
+      const float g0 = __uint_as_float(gr.x << 16), g1 = __uint_as_float(gr.x & 0xffff0000u);
+      const float g2 = __uint_as_float(gr.y << 16), g3 = __uint_as_float(gr.y & 0xffff0000u);
+      reinterpret_cast<uint2*>(out + row * N)[c] =
+          make_uint2(pack_half2(v[q].x * inv * g0, v[q].y * inv * g1), pack_half2(v[q].z * inv * g2, v[q].w * inv * g3));
     }
   }
 }
@@ -532,7 +603,7 @@ static int choose_splits(int M, int N, int K, size_t ws_bytes) {
   return best;
 }
 
-}  // namespace tc}  // namespace tc
+}  // namespace tc
 
 // Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
 // the RoPE epilogue), A, B and C 16-byte aligned.
@@ -545,11 +616,20 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     return 1;
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
+  // The residual product with a following RMSNorm (ep.norm_out) always goes through the
+  // scratch, one slice or more, into the fused reduction + norm kernel.
+  const bool fuse_norm = epi == EPI_RESID_F32 && ep.norm_out;
+  if (fuse_norm && (!split_ws || N > 8192 || (size_t)M * N * sizeof(float) > split_ws_bytes)) return 1;
   const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
-  if (splits > 1) {
+  if (splits > 1 || fuse_norm) {
     if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits)) return 1;
     const float* part = static_cast<const float*>(split_ws);
-    const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N);
+    if (fuse_norm) {
+      splitk_resid_norm_kernel<<<M, 256, 0, st>>>(part, splits, M, N, static_cast<float*>(C),
+                                                   static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out);
+      return 0;
+    }
+    const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N) / 4;
     const int grid = (int)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048);
     switch (epi) {
       case EPI_STORE_BF16: splitk_reduce_kernel<EPI_STORE_BF16><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;

@@ -255,6 +255,8 @@ DecodeLayout decode_layout(const rift_model& m, int n_seq, int max_len) {
   if (m.lm_head && (size_t)m.vocab > widest) widest = (size_t)m.vocab;
   L.split_bytes = 16 * rows * widest * 4;
   if (L.split_bytes > (size_t)128 << 20) L.split_bytes = (size_t)128 << 20;
+  // at least one slice of the residual products, which always go through the scratch
+  if (L.split_bytes < n * m.d * 4) L.split_bytes = n * m.d * 4;
   L.split_off = take(L.split_bytes);
   L.total = off;
   return L;
@@ -445,11 +447,17 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
   rope_ep.max_len = max_len;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)m.head_dim);
   const uint16_t* kv = static_cast<const uint16_t*>(kv_cache);
+  // The residual products carry the RMSNorm that follows them (g_ffn after W_o; the next layer's
+  // g_attn, or g_final after the last W_down) into their split-K reduction.
+  auto resid_norm = [&](const void* gain) {
+    EpiParams e;
+    e.norm_gain = gain;
+    e.norm_out = xn;
+    e.norm_eps = m.eps;
+    return e;
+  };
+  norm_launch(0, n, x0, h32, m.g_attn[0], xn, d, m.eps, st);
   for (int l = 0; l < m.n_layers; ++l) {
-    if (l == 0)
-      norm_launch(0, n, x0, h32, m.g_attn[0], xn, d, m.eps, st);
-    else
-      norm_launch(1, n, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
     if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep, split, sb)) return 1;
     if (kv_new) {
       uint16_t* kl = static_cast<uint16_t*>(kv_new) + (size_t)l * 2 * n * d;
@@ -468,14 +476,14 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
     decode_combine_kernel<<<n * m.n_heads, m.head_dim, 0, st>>>(dpart, cu_seqlens, m.n_heads, m.head_dim, max_chunks,
                                                                 max_len, att);
     prof_end(RIFT_PROF_ATTN, st, 2);
-    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st, EpiParams(), split, sb)) return 1;
-    norm_launch(1, n, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
+    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st, resid_norm(m.g_ffn[l]), split, sb)) return 1;
     if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st, EpiParams(), split, sb)) return 1;
-    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st, EpiParams(), split, sb)) return 1;
+    const void* next_gain = l + 1 < m.n_layers ? m.g_attn[l + 1] : m.g_final;
+    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st, resid_norm(next_gain), split, sb)) return 1;
   }
+  // xn now holds RMSNorm(h) g_final in fp16 (the logits operand)
   if (hidden_out) norm_launch(2, n, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden_out), d, m.eps, st);
   if (logits) {
-    norm_launch(1, n, h32, nullptr, m.g_final, xn, d, m.eps, st);
     if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st, EpiParams(), split, sb)) return 1;
   }
   return 0;

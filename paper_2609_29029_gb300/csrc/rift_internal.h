@@ -76,6 +76,10 @@ struct EpiParams {
   int head_dim = 0;
   int max_len = 0;
   float out_scale = 1.f;           // EPI_STORE_F32
+  // EPI_RESID_F32 with split scratch: also norm_out fp16 [M, N] = RMSNorm(C) norm_gain (bf16 [N])
+  const void* norm_gain = nullptr;
+  uint16_t* norm_out = nullptr;
+  float norm_eps = 0.f;
 };
 // split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
 // most SMs idle run as (tile, K-slice) units plus a reduction kernel.
