@@ -51,24 +51,50 @@ def parse():
 
 
 def ncu_summary(path: str) -> str:
-    """Per kernel: launches, total device time and share of an ncu --csv launch list."""
+    """Per kernel of an ncu --csv launch list: launches, total device time, share and, when the
+    list has dram__bytes_read.sum / dram__bytes_write.sum, DRAM traffic.  Ends with the GEMM
+    traffic block that bench.py reads back (mean DRAM bytes per gemm_tc_kernel launch and the
+    hash of the gemm_tc.cu it was measured on)."""
     import csv
+    import hashlib
     with open(path) as f:
         rows = list(csv.DictReader([ln for ln in f if ln.startswith('"')]))
-    agg = {}
+    tscale = {"ns": 1e-6, "nsecond": 1e-6, "us": 1e-3, "usecond": 1e-3, "ms": 1.0, "msecond": 1.0}
+    bscale = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
+    launches = {}
     for r in rows:
-        if r.get("Metric Name") != "gpu__time_duration.sum":
-            continue
-        name = r["Kernel Name"].split("(")[0]
-        scale = {"ns": 1e-6, "us": 1e-3, "usecond": 1e-3, "ms": 1.0, "msecond": 1.0}.get(r["Metric Unit"], 1e-6)
-        t = float(r["Metric Value"].replace(",", "")) * scale
-        n, tot = agg.get(name, (0, 0.0))
-        agg[name] = (n + 1, tot + t)
+        d = launches.setdefault(r["ID"], {"name": r["Kernel Name"].split("(")[0]})
+        v = float(r["Metric Value"].replace(",", ""))
+        if r["Metric Name"] == "gpu__time_duration.sum":
+            d["ms"] = v * tscale.get(r["Metric Unit"], 1e-6)
+        elif r["Metric Name"] in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            d[r["Metric Name"]] = v * bscale.get(r["Metric Unit"], 1.0)
+    agg = {}
+    for d in launches.values():
+        a = agg.setdefault(d["name"], [0, 0.0, 0.0, 0.0])
+        a[0] += 1
+        a[1] += d.get("ms", 0.0)
+        a[2] += d.get("dram__bytes_read.sum", 0.0)
+        a[3] += d.get("dram__bytes_write.sum", 0.0)
     total = sum(v[1] for v in agg.values())
-    out = [f"{'kernel':<44} {'launches':>8} {'total ms':>11} {'share':>7}"]
-    for name, (n, t) in sorted(agg.items(), key=lambda kv: -kv[1][1]):
-        out.append(f"{name:<44} {n:>8} {t:>11.3f} {100 * t / total:>6.2f}%")
-    out.append(f"{'all':<44} {sum(v[0] for v in agg.values()):>8} {total:>11.3f} 100.00%")
+    dram = any(v[2] or v[3] for v in agg.values())
+    out = [f"{'kernel':<46} {'launches':>8} {'total ms':>10} {'share':>7}" + (
+        f" {'DRAM rd GB':>10} {'DRAM wr GB':>10} {'GB/s':>6}" if dram else "")]
+    for name, (n, t, rd, wr) in sorted(agg.items(), key=lambda kv: -kv[1][1]):
+        line = f"{name[:46]:<46} {n:>8} {t:>10.3f} {100 * t / total:>6.2f}%"
+        if dram:
+            line += f" {rd / 1e9:>10.3f} {wr / 1e9:>10.3f} {(rd + wr) / 1e6 / t if t else 0:>6.0f}"
+        out.append(line)
+    out.append(f"{'all':<46} {sum(v[0] for v in agg.values()):>8} {total:>10.3f}")
+    gemm = [(n, a) for n, a in agg.items() if "gemm_tc_kernel" in n]
+    if dram and gemm:
+        n = sum(a[0] for _, a in gemm)
+        b = sum(a[2] + a[3] for _, a in gemm)
+        src = ROOT / "paper_2609_29029_gb300" / "csrc" / "gemm_tc.cu"
+        out += ["", "GEMM traffic used by bench.py (mean over the gemm_tc_kernel launches of the list):", "",
+                "- kernel: gemm_tc_kernel",
+                f"- source_sha256_16: {hashlib.sha256(src.read_bytes()).hexdigest()[:16]}",
+                f"- dram_bytes_per_launch: {int(b / n)}", f"- launches: {n}"]
     return "\n".join(out)
 
 
