@@ -11,7 +11,8 @@ Each function restates one step of the paper in the paper's order:
   Appendix B, Step 3 / Listing 1 ...... retain tiles with u_i >= tau (tau = 0.37)
   Section 2.3, Stage 2, Eq. 2 ......... U_i(c) = A_i(c) - lambda E_c,
                                          A_i(c) = p_i a+_c + (1 - p_i) a-_c, c* = argmax
-  Section 2.3, Stage 2 ................ keep each retained tile's dominant tokens
+  Section 2.3, Stage 2 ................ keep each retained tile's dominant tokens and merge
+                                         the remainder into contextual tokens (VisionZip)
   Section 2.1 ......................... decoder prefill over [system | vision | query],
                                          the KV cache it builds, the last-token logits
                                          and the decode step that follows it
@@ -42,6 +43,13 @@ Readings of points the paper leaves open (each also used by the CUDA path):
   * Utility in fp32 as ((p * a+) + ((1 - p) * a-)) - (lambda * E); C ascending,
     ties to the lower index (the cheaper budget).
   * Top-b: the b largest r, ties to the lower token index, listed ascending.
+  * Merge (policy ctx_num > 0; the paper uses VisionZip's mechanism without details): a budget
+    c < n_v holds m = floor(ctx_num c / ctx_den) contextual tokens and c - m dominant ones.  Of
+    the R tokens not selected (ascending), every floor(R / m)-th from the first is a target;
+    every other one joins the target with the largest cosine similarity (ties to the lower
+    target), in the projected-token space (the paper's encoder keys are not available); a
+    contextual token is the mean of its group, target included.  Sequence i = [S system ids |
+    c - m dominant tokens | m contextual tokens in target order | Q query ids].
   * Sequence i = [S system ids | b_i selected tokens | Q query ids], positions
     0 .. L_i - 1, tiles in ascending index order.
   * Decoder: LLaMA block, RMSNorm (eps 1e-6), rotate-half RoPE (theta 1e4),
@@ -227,17 +235,58 @@ def top_b(r32: np.ndarray, b: int) -> list:
     return sorted(order[:b])
 
 
+def contextual_count(c: int, n_v: int, policy) -> int:
+    """Contextual tokens inside a budget of c tokens (none at the full budget or without merge)."""
+    num = getattr(policy, "ctx_num", 0)
+    if num == 0 or c >= n_v:
+        return 0
+    return (num * c) // policy.ctx_den
+
+
+def merge_contextual(X_tile: torch.Tensor, dominant, m: int):
+    """VisionZip-style merge of the tokens not in `dominant`: (targets, groups, ctx fp64 [m, d]).
+    groups[j] lists target j first, then the tokens that joined it in ascending index."""
+    n_v, d = X_tile.shape
+    keep = set(int(k) for k in dominant)
+    rest = [k for k in range(n_v) if k not in keep]
+    m = min(m, len(rest))
+    if m == 0:
+        return [], [], torch.zeros(0, d, dtype=torch.float64)
+    step = len(rest) // m
+    targets = [rest[j * step] for j in range(m)]
+    x = X_tile.to(torch.float64)
+    xt = x[targets]
+    nrm = torch.sqrt((xt * xt).sum(dim=1, keepdim=True))
+    xt_hat = torch.where(nrm > 0, xt / torch.where(nrm > 0, nrm, torch.ones_like(nrm)), torch.zeros_like(xt))
+    groups = [[t] for t in targets]
+    tset = set(targets)
+    for k in rest:
+        if k in tset:
+            continue
+        sim = xt_hat @ x[k]  # cosine up to the positive factor 1 / ||x_k||
+        best = 0
+        for j in range(1, m):
+            if float(sim[j]) > float(sim[best]):
+                best = j
+        groups[best].append(k)
+    ctx = torch.stack([x[g].mean(dim=0) for g in groups])
+    return targets, groups, ctx
+
+
 # ------------------------------------------------------------------------------------------
 # a8  packing into per-tile sequences [system | selected vision tokens | query]
 # ------------------------------------------------------------------------------------------
 
-def pack(X, embed, kept, sel, sys_ids, query_ids):
-    """Returns (H0 bf16 [T, d], cu_seqlens [n+1], positions [T])."""
+def pack(X, embed, kept, sel, sys_ids, query_ids, ctx=None):
+    """Returns (H0 bf16 [T, d], cu_seqlens [n+1], positions [T]).  ctx: per kept tile its
+    contextual tokens (fp64 [m, d]), placed after the dominant ones."""
     rows, cu, pos = [], [0], []
     sys_rows = embed[list(sys_ids)].to(torch.bfloat16)
     q_rows = embed[list(query_ids)].to(torch.bfloat16)
-    for i, idx in zip(kept, sel):
+    for n, (i, idx) in enumerate(zip(kept, sel)):
         vis = X[i][list(idx)].to(torch.bfloat16)
+        if ctx is not None and len(ctx[n]):
+            vis = torch.cat([vis, ctx[n].to(torch.bfloat16)], dim=0)
         seq = torch.cat([sys_rows, vis, q_rows], dim=0)
         rows.append(seq)
         cu.append(cu[-1] + seq.shape[0])
@@ -403,7 +452,10 @@ class Selection:
     kept: list
     p: np.ndarray              # [n_kept] fp32
     budgets: list              # [n_kept]
-    sel: list                  # per kept tile, ascending token indices
+    sel: list                  # per kept tile, ascending dominant token indices
+    ctx_targets: list = None   # per kept tile, the contextual tokens' targets (merge only)
+    ctx_groups: list = None
+    ctx: list = None           # per kept tile, fp64 [m, d] contextual tokens
 
 
 def decide(r32, s32, G, m, policy, p_ext=None):
@@ -417,7 +469,8 @@ def decide(r32, s32, G, m, policy, p_ext=None):
     else:
         p = np.array([F32(p_ext[i]) for i in kept], dtype=F32)
     bud = [budget(float(pi), policy) for pi in p]
-    sel = [top_b(r32[i], b) for i, b in zip(kept, bud)]
+    n_v = r32.shape[1]
+    sel = [top_b(r32[i], b - contextual_count(b, n_v, policy)) for i, b in zip(kept, bud)]
     return nbr, st, u, kept, p, bud, sel
 
 
@@ -428,4 +481,12 @@ def select(X, embed, query_ids, bg_ids, m, policy, p_ext=None, templates=None) -
     r32, s32 = to_f32(r64), to_f32(s64)
     G = similarity(V)
     nbr, st, u, kept, p, bud, sel = decide(r32, s32, G, m, policy, p_ext)
-    return Selection(t, B, r64, V, s64, r32, s32, G, nbr, st, u, kept, p, bud, sel)
+    out = Selection(t, B, r64, V, s64, r32, s32, G, nbr, st, u, kept, p, bud, sel)
+    if getattr(policy, "ctx_num", 0):
+        n_v = X.shape[1]
+        merged = [merge_contextual(X[i], idx, contextual_count(b, n_v, policy))
+                  for i, idx, b in zip(kept, sel, bud)]
+        out.ctx_targets = [mg[0] for mg in merged]
+        out.ctx_groups = [mg[1] for mg in merged]
+        out.ctx = [mg[2] for mg in merged]
+    return out

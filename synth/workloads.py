@@ -65,6 +65,10 @@ class Policy:
     alpha_neg: tuple
     energy: tuple
     lam: float
+    # Contextual tokens inside a budget c < n_v: floor(ctx_num c / ctx_den) of the c tokens are
+    # merged from the unselected ones (Stage 2, VisionZip's mechanism); ctx_num = 0 selects only.
+    ctx_num: int = 0
+    ctx_den: int = 64
 
 
 RIFT_POLICY = Policy(tau=0.37, C=(72, 144, 288, 432, 576),
@@ -72,6 +76,8 @@ RIFT_POLICY = Policy(tau=0.37, C=(72, 144, 288, 432, 576),
                      alpha_neg=(0.50, 0.68, 0.84, 0.868, 0.89),
                      energy=(0.28, 0.40, 0.62, 0.82, 1.00), lam=0.15)
 RIFT_POLICY_SKEW = replace(RIFT_POLICY, lam=0.10)
+# VisionZip's split of a budget into dominant and contextual tokens (54 + 10 of 64)
+RIFT_POLICY_MERGE = replace(RIFT_POLICY, ctx_num=10, ctx_den=64)
 # tau = 0 keeps every tile (u >= 0 always); C = {576} gives every tile its full budget.
 KEEP_ALL = Policy(tau=0.0, C=(576,), alpha_pos=(1.0,), alpha_neg=(1.0,), energy=(0.0,), lam=0.0)
 

@@ -471,3 +471,114 @@ def test_logits_select_rows_of_the_output_matrix():
     assert not torch.equal(h[:, perm], h[:, torch.argsort(perm)])
     W2 = torch.randn(5, d, generator=torch.Generator().manual_seed(15), dtype=torch.float64)
     assert torch.allclose(O.logits(h[0], W2), torch.stack([W2[r] @ h[0] for r in range(5)]), atol=1e-14)
+
+
+# ------------------------------------- contextual-token merge (Stage 2: VisionZip's mechanism)
+
+def test_contextual_count_matches_visionzip_splits():
+    P = W.RIFT_POLICY_MERGE
+    # VisionZip's LLaVA-1.5 settings: 64 = 54 + 10, 128 = 108 + 20, 192 = 162 + 30 tokens
+    assert [O.contextual_count(c, 576, P) for c in (64, 128, 192)] == [10, 20, 30]
+    assert O.contextual_count(576, 576, P) == 0              # full budget: nothing left to merge
+    assert O.contextual_count(288, 576, W.RIFT_POLICY) == 0  # merge off
+    assert [O.contextual_count(c, 576, P) for c in P.C] == [11, 22, 45, 67, 0]
+
+
+def _rest(n_v, dominant):
+    return [k for k in range(n_v) if k not in set(dominant)]
+
+
+def test_merge_recovers_planted_clusters():
+    # 12 remaining tokens (dominant ones interleaved) in 3 tight clusters of 4 consecutive
+    # remaining tokens around orthogonal directions.  With m = 3 the targets are the 1st, 5th and
+    # 9th remaining tokens, one per cluster, so the groups are the clusters and each contextual
+    # token is its cluster's mean.  A target step taken over all tokens instead of the remaining
+    # ones, or an off-by-one, puts two targets in one cluster.
+    g = torch.Generator().manual_seed(20)
+    n_v, d = 15, 6
+    dominant = [1, 5, 9]
+    rest = _rest(n_v, dominant)
+    X = 0.01 * torch.randn(n_v, d, generator=g, dtype=torch.float64)
+    for c in range(3):
+        for k in rest[4 * c:4 * c + 4]:
+            X[k, 2 * c] += 1.0 + 0.1 * c
+    targets, groups, ctx = O.merge_contextual(X, dominant, 3)
+    assert targets == [rest[0], rest[4], rest[8]]
+    assert [sorted(gr) for gr in groups] == [rest[0:4], rest[4:8], rest[8:12]]
+    for c in range(3):
+        assert torch.allclose(ctx[c], X[rest[4 * c:4 * c + 4]].mean(dim=0), atol=1e-15)
+
+
+def test_merge_special_cases():
+    g = torch.Generator().manual_seed(21)
+    X = torch.randn(10, 4, generator=g, dtype=torch.float64)
+    dominant = [2, 7]
+    rest = _rest(10, dominant)
+    t, gr, ctx = O.merge_contextual(X, dominant, len(rest))    # every remaining token a target
+    assert t == rest and torch.equal(ctx, X[rest])
+    t, gr, ctx = O.merge_contextual(X, dominant, 1)            # one target takes everything
+    assert t == [rest[0]] and torch.allclose(ctx[0], X[rest].mean(dim=0), atol=1e-15)
+    assert O.merge_contextual(X, dominant, 0)[2].shape == (0, 4)
+    assert O.merge_contextual(X, list(range(10)), 3)[2].shape == (0, 4)   # nothing left
+    assert O.merge_contextual(X, dominant, 50)[0] == rest                 # m capped at R
+
+
+@pytest.mark.parametrize("seed", [22, 23, 24])
+def test_merge_assignment_brute_force_cosine(seed):
+    g = torch.Generator().manual_seed(seed)
+    n_v, d, m = 30, 8, 5
+    X = torch.randn(n_v, d, generator=g, dtype=torch.float64)
+    dominant = sorted(torch.randperm(n_v, generator=g)[:7].tolist())
+    rest = _rest(n_v, dominant)
+    targets, groups, _ = O.merge_contextual(X, dominant, m)
+    step = len(rest) // m
+    assert targets == rest[::step][:m]
+    owner = {k: j for j, gr in enumerate(groups) for k in gr}
+    for k in rest:
+        if k in targets:
+            assert owner[k] == targets.index(k)
+            continue
+        sims = [1.0 - distance.cosine(X[k].numpy(), X[t].numpy()) for t in targets]
+        best = max(range(m), key=lambda j: (sims[j], -j))
+        assert owner[k] == best
+    # scale invariance of the assignment (positive factors on the non-target tokens)
+    Xs = X.clone()
+    for k in rest:
+        if k not in targets:
+            Xs[k] *= 0.5 + k
+    assert O.merge_contextual(Xs, dominant, m)[1] == groups
+
+
+def test_merge_ties_go_to_the_lower_target_and_mass_is_conserved():
+    # every token points the same way, so all four targets (0, 2, 4, 6) tie for every token
+    X = torch.zeros(8, 3, dtype=torch.float64)
+    X[:, 0] = torch.arange(1, 9, dtype=torch.float64)
+    _, groups, ctx = O.merge_contextual(X, [], 4)
+    assert groups == [[0, 1, 3, 5, 7], [2], [4], [6]]
+    g = torch.Generator().manual_seed(25)
+    Y = torch.randn(40, 6, generator=g, dtype=torch.float64)
+    dominant = [0, 3, 17, 39]
+    rest = _rest(40, dominant)
+    _, groups, ctx = O.merge_contextual(Y, dominant, 6)
+    assert sorted(k for gr in groups for k in gr) == rest
+    total = sum(len(gr) * ctx[j] for j, gr in enumerate(groups))
+    assert torch.allclose(total, Y[rest].sum(dim=0), atol=1e-12)
+
+
+def test_selection_with_merge_splits_every_budget():
+    from dataclasses import replace
+    wl = replace(W.TINY, policy=replace(W.TINY.policy, ctx_num=10, ctx_den=64))
+    sc = W.make_scene(wl.scene, wl.decoder.vocab)
+    sel = O.select(sc.X, sc.embed, sc.query_ids, sc.bg_ids, wl.knn_m, wl.policy)
+    n_v = wl.scene.n_v
+    for i, idx, b, ctx in zip(sel.kept, sel.sel, sel.budgets, sel.ctx):
+        m = O.contextual_count(b, n_v, wl.policy)
+        assert len(idx) == b - m and ctx.shape[0] == m
+        assert idx == O.top_b(sel.r32[i], b - m)
+    H0, cu, pos = O.pack(sc.X, sc.embed, sel.kept, sel.sel, sc.sys_ids, sc.query_ids, sel.ctx)
+    S, Q = wl.scene.S, wl.scene.Q
+    assert [cu[j + 1] - cu[j] for j in range(len(sel.kept))] == [S + b + Q for b in sel.budgets]
+    for j, (i, idx, ctx) in enumerate(zip(sel.kept, sel.sel, sel.ctx)):
+        a = cu[j] + S
+        assert torch.equal(H0[a:a + len(idx)], sc.X[i][idx].to(torch.bfloat16))
+        assert torch.equal(H0[a + len(idx):a + len(idx) + ctx.shape[0]], ctx.to(torch.bfloat16))
