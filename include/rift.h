@@ -72,7 +72,12 @@ typedef void* rift_stream_t; /* cudaStream_t */
  *   energy     profiled energy per c;  lambda  the accuracy-energy trade-off
  * U_i(c) = ((p_i * alpha_pos[c]) + ((1 - p_i) * alpha_neg[c])) - (lambda * energy[c]),
  * each operation a correctly rounded fp32 op; b_i = C[argmax_c U_i(c)], ties to the
- * lower index (the cheaper budget). */
+ * lower index (the cheaper budget).
+ *   ctx_num, ctx_den  the merge of Stage 2 (VisionZip's mechanism: keep the dominant tokens,
+ *              merge the remainder): a budget b < n_v holds floor(ctx_num b / ctx_den)
+ *              contextual tokens and b minus that many selected (dominant) tokens; ctx_num = 0
+ *              turns the merge off (every budget token is selected).  0 <= ctx_num < ctx_den.
+ *              VisionZip's split is 10 / 64. */
 typedef struct {
   float tau;
   int n_c;
@@ -81,6 +86,7 @@ typedef struct {
   float alpha_neg[RIFT_MAX_BUDGETS];
   float energy[RIFT_MAX_BUDGETS];
   float lambda;
+  int ctx_num, ctx_den;
 } rift_policy;
 
 /* A LLaMA/Vicuna-shaped decoder (Section 2.1; LLaVA-1.5-7B: 32 layers, d 4096, 32 heads
@@ -184,8 +190,9 @@ rift_status rift_score_tiles_noalloc(const void* X, rift_dtype xdt, int N, int n
  *   n_kept     out int32 [1]
  *   budgets    out int32 [N]: b_j for kept slot j (first n_kept entries)
  *   sel        out int32 [N * n_v]: kept slot j's selected token indices at sel_off[j],
- *              the b_j largest token scores (ties to the lower index), ascending
- *   sel_off    out int32 [N + 1]: exclusive prefix sum of budgets; entries j > n_kept
+ *              the s_j largest token scores (ties to the lower index), ascending, with
+ *              s_j = b_j less its contextual tokens (s_j = b_j without the merge)
+ *   sel_off    out int32 [N + 1]: exclusive prefix sum of the s_j; entries j > n_kept
  *              are set to the total
  * A NaN or Inf among the scores that are read sets RIFT_ERR_NONFINITE. */
 size_t rift_select_workspace_bytes(int N, int n_v);
@@ -196,14 +203,39 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
                                         int* sel, int* sel_off,
                                         void* ws, size_t ws_bytes, rift_stream_t stream);
 
+/* ---- a7b. Merge of the unselected tokens (Section 2.3, Stage 2: VisionZip's mechanism keeps
+ * the dominant tokens and merges the remainder) ----
+ * For kept slot j with m_j = budgets[j] - (sel_off[j+1] - sel_off[j]) contextual tokens (see
+ * rift_policy ctx_num): the R_j tokens of the tile that were not selected, in ascending index,
+ * give the targets rest[q floor(R_j / m_j)], q < m_j; every other remaining token joins the target
+ * with the largest cosine similarity to it (ties to the lower target; decided at ~fp64 accuracy),
+ * and contextual token q is the mean of its group, target included (fp32 sums in ascending token
+ * index, stored as bf16).
+ *   X, xdt, N, n_v, d   the scene (as rift_score_tiles); kept, n_kept, budgets, sel, sel_off
+ *              from rift_select_budgeted_tokens
+ *   ctx        out bf16 [max_ctx, d]: slot j's contextual tokens at rows ctx_off[j] ..
+ *   ctx_off    out int32 [N + 1]: exclusive prefix sum of the m_j; entries j > n_kept are the
+ *              total (all zero when the merge is off)
+ *   ctx_target out int32 [max_ctx]: the target token index of each contextual token
+ *   ws         rift_merge_workspace_bytes(N, n_v) bytes
+ * More than max_ctx contextual tokens set RIFT_ERR_CAPACITY (the excess is not written). */
+size_t rift_merge_workspace_bytes(int N, int n_v);
+rift_status rift_merge_contextual(const void* X, rift_dtype xdt, int N, int n_v, int d,
+                                  const int* kept, const int* n_kept, const int* budgets,
+                                  const int* sel, const int* sel_off, void* ctx, int max_ctx,
+                                  int* ctx_off, int* ctx_target, void* ws, size_t ws_bytes,
+                                  rift_stream_t stream);
+
 /* ---- a8. Ragged packing (the per-tile VLM prompt of Appendix B Step 5) ----
  *   X, xdt, N, n_v, d     as for rift_score_tiles (fp32 tokens are rounded to bf16)
  *   kept, n_kept, sel, sel_off   from rift_select_budgeted_tokens
  *   sys_ids    int32 [S] system-prompt ids;  query_ids int32 [Q] query ids
  *   embed      bf16 [vocab, d]
+ *   ctx, ctx_off  contextual tokens and offsets from rift_merge_contextual, or both NULL
  *   packed     out bf16 [max_T, d]: sequence j = [embed[sys_ids] | X[kept[j], sel_j] |
- *              embed[query_ids]], sequences back to back in kept order
- *   cu_seqlens out int32 [N + 1]: cu_seqlens[j] = j (S + Q) + sel_off[j]; entries
+ *              ctx rows ctx_off[j] .. ctx_off[j+1] | embed[query_ids]], sequences back to back
+ *              in kept order
+ *   cu_seqlens out int32 [N + 1]: cu_seqlens[j] = j (S + Q) + sel_off[j] + ctx_off[j]; entries
  *              j > n_kept are set to T
  *   positions  out int32 [max_T]: position of each packed row in its sequence (0..L_j-1)
  *   T          out int32 [1]: total packed rows
@@ -212,7 +244,7 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
                              const int* kept, const int* n_kept,
                              const int* sel, const int* sel_off,
                              const int* sys_ids, int S, const int* query_ids, int Q,
-                             const void* embed, int vocab,
+                             const void* embed, int vocab, const void* ctx, const int* ctx_off,
                              void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
                              rift_stream_t stream);
 

@@ -29,7 +29,8 @@ class RiftError(RuntimeError):
 class Policy(C.Structure):
     _fields_ = [("tau", C.c_float), ("n_c", C.c_int), ("C", C.c_int * MAX_BUDGETS),
                 ("alpha_pos", C.c_float * MAX_BUDGETS), ("alpha_neg", C.c_float * MAX_BUDGETS),
-                ("energy", C.c_float * MAX_BUDGETS), ("lam", C.c_float)]
+                ("energy", C.c_float * MAX_BUDGETS), ("lam", C.c_float), ("ctx_num", C.c_int),
+                ("ctx_den", C.c_int)]
 
 
 class Model(C.Structure):
@@ -53,8 +54,11 @@ SIGNATURES = {
     "rift_select_workspace_bytes": (_sz, [_i, _i]),
     "rift_select_budgeted_tokens": (_i, [_vp, _vp, _i, _i, _vp, C.POINTER(Policy), _vp, _vp, _vp, _vp, _vp,
                                          _vp, _vp, _sz, _vp]),
-    "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _i,
-                              _vp, _vp, _vp, _vp]),
+    "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp,
+                              _vp, _i, _vp, _vp, _vp, _vp]),
+    "rift_merge_workspace_bytes": (_sz, [_i, _i]),
+    "rift_merge_contextual": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz,
+                                   _vp]),
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
     "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "rift_decode_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i]),
@@ -121,6 +125,8 @@ def make_policy(policy) -> Policy:
         p.alpha_neg[k] = policy.alpha_neg[k]
         p.energy[k] = policy.energy[k]
     p.lam = policy.lam
+    p.ctx_num = getattr(policy, "ctx_num", 0)
+    p.ctx_den = getattr(policy, "ctx_den", 64)
     return p
 
 
@@ -171,11 +177,23 @@ def select_budgeted_tokens(token_scores, tile_s, N, n_v, p, policy: Policy, u, k
 
 
 def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, packed,
-                max_T, cu_seqlens, positions, T, stream=None):
+                max_T, cu_seqlens, positions, T, stream=None, ctx=None, ctx_off=None):
     _check(lib.rift_pack_ragged(ptr(X), xdt, N, n_v, d, ptr(kept), ptr(n_kept), ptr(sel), ptr(sel_off),
-                                ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(packed), max_T,
-                                ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),
+                                ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(ctx), ptr(ctx_off),
+                                ptr(packed), max_T, ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),
            "rift_pack_ragged")
+
+
+def merge_workspace_bytes(N, n_v) -> int:
+    return lib.rift_merge_workspace_bytes(N, n_v)
+
+
+def merge_contextual(X, xdt, N, n_v, d, kept, n_kept, budgets, sel, sel_off, ctx, max_ctx, ctx_off, ctx_target, ws,
+                     ws_bytes, stream=None):
+    _check(lib.rift_merge_contextual(ptr(X), xdt, N, n_v, d, ptr(kept), ptr(n_kept), ptr(budgets), ptr(sel),
+                                     ptr(sel_off), ptr(ctx), max_ctx, ptr(ctx_off), ptr(ctx_target), ptr(ws),
+                                     ws_bytes, stream_handle(stream)),
+           "rift_merge_contextual")
 
 
 def linear(A, W, M, N, K, epilogue, out, stream=None):

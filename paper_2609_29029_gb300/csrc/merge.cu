@@ -1,0 +1,340 @@
+// Merge of the unselected tokens into contextual tokens on sm_103a (Section 2.3, Stage 2: Rift
+// uses VisionZip's mechanism to keep the dominant tokens and merge the remainder).
+//
+// For kept slot j with m_j = budgets[j] - s_j contextual tokens (s_j selected tokens):
+//   merge_plan_kernel     m_j (capped at the R_j unselected tokens) and their offsets ctx_off
+//   merge_targets_kernel  the unselected tokens in ascending index, the targets (every
+//                         floor(R_j / m_j)-th of them from the first) and the targets' norms
+//   merge_assign_kernel   per 64 unselected tokens x 64 targets: fp32 dot products in 32-term
+//                         chunks, a running top 2 per token; the two are recomputed as float-float
+//                         sums (good to ~2^-44) and compared as x.t1 ||t2|| vs x.t2 ||t1|| in fp64,
+//                         so the decision is the cosine argmax of the exact arithmetic (ties to
+//                         the lower target)
+//   merge_mean_kernel     per contextual token: its group's sum in ascending token index
+//                         (fp32), divided by the group size, stored as bf16
+#include "rift_internal.h"
+
+namespace rift {
+
+__device__ unsigned int g_err_merge;
+
+unsigned int read_clear_err_merge() {
+  unsigned int v = 0, z = 0;
+  cudaMemcpyFromSymbol(&v, g_err_merge, sizeof(v));
+  cudaMemcpyToSymbol(g_err_merge, &z, sizeof(z));
+  return v;
+}
+
+namespace mg {
+
+constexpr int TB = 64;     // tokens and targets per block of the similarity pass
+constexpr int KC = 32;     // d-chunk
+
+template <typename XT>
+__device__ __forceinline__ float load_x(const XT* p) {
+  if constexpr (sizeof(XT) == 2)
+    return bf16_bits_to_float(*reinterpret_cast<const uint16_t*>(p));
+  else
+    return *p;
+}
+
+// Float-float accumulation of a.b over d terms by one warp (TwoProduct with an FMA, TwoSum),
+// then the lanes' pairs summed in fp64.
+template <typename XT>
+__device__ double ff_dot(const XT* a, const XT* b, int d, int lane) {
+  float hi = 0.f, lo = 0.f;
+  for (int k = lane; k < d; k += 32) {
+    const float x = load_x(a + k), y = load_x(b + k);
+    const float p = __fmul_rn(x, y);
+    const float pe = fmaf(x, y, -p);
+    const float s = __fadd_rn(hi, p);
+    const float bb = __fsub_rn(s, hi);
+    const float er = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(p, bb));
+    hi = s;
+    lo = __fadd_rn(lo, __fadd_rn(er, pe));
+  }
+  double acc = (double)hi + (double)lo;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  return acc;
+}
+
+// m_j = min(budgets[j] - s_j, n_v - s_j) and its exclusive prefix sum over the kept slots.  If
+// the total exceeds max_ctx, RIFT_EBIT_CAPACITY is set and every m_j is taken as 0 (no contextual
+// row is then written or read).
+__global__ void __launch_bounds__(1024) merge_plan_kernel(const int* __restrict__ n_kept,
+                                                          const int* __restrict__ budgets,
+                                                          const int* __restrict__ sel_off, int N, int n_v,
+                                                          int max_ctx, int* __restrict__ ctx_off) {
+  __shared__ int sh[33];
+  const int n = *n_kept;
+  auto count = [&](int j) {
+    const int s = sel_off[j + 1] - sel_off[j];
+    return max(0, min(budgets[j] - s, n_v - s));
+  };
+  int total_all = 0;
+  for (int c0 = 0; c0 < n; c0 += blockDim.x) {
+    const int j = c0 + threadIdx.x;
+    int total;
+    block_excl_scan(j < n ? count(j) : 0, sh, &total);
+    total_all += total;
+  }
+  const bool fits = total_all <= max_ctx;
+  if (threadIdx.x == 0 && !fits) atomicOr(&g_err_merge, RIFT_EBIT_CAPACITY);
+  int base = 0;
+  for (int c0 = 0; c0 < n; c0 += blockDim.x) {
+    const int j = c0 + threadIdx.x;
+    const int m = (j < n && fits) ? count(j) : 0;
+    int total;
+    const int pos = block_excl_scan(m, sh, &total);
+    if (j < n) ctx_off[j] = base + pos;
+    base += total;
+  }
+  for (int j = n + threadIdx.x; j <= N; j += blockDim.x) ctx_off[j] = base;
+}
+
+// One CTA per kept slot: rest[j][0 .. R) = the unselected tokens in ascending index, the targets
+// (written to ctx_target) and their norms (tnorm, fp64 from a float-float sum of squares).
+template <typename XT>
+__global__ void __launch_bounds__(256) merge_targets_kernel(const XT* __restrict__ X, int n_v, int d,
+                                                            const int* __restrict__ kept,
+                                                            const int* __restrict__ n_kept,
+                                                            const int* __restrict__ sel,
+                                                            const int* __restrict__ sel_off,
+                                                            const int* __restrict__ ctx_off, int max_ctx,
+                                                            int* __restrict__ rest, int* __restrict__ ctx_target,
+                                                            double* __restrict__ tnorm) {
+  __shared__ unsigned char chosen[RIFT_MAX_NV];
+  __shared__ int sh[33];
+  const int j = blockIdx.x;
+  if (j >= *n_kept) return;
+  const int so = sel_off[j], s = sel_off[j + 1] - so;
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  for (int k = threadIdx.x; k < n_v; k += blockDim.x) chosen[k] = 0;
+  __syncthreads();
+  for (int q = threadIdx.x; q < s; q += blockDim.x) {
+    const int k = sel[so + q];
+    if (k >= 0 && k < n_v) chosen[k] = 1;
+  }
+  __syncthreads();
+  int* rj = rest + (size_t)j * n_v;
+  int base = 0;
+  for (int c0 = 0; c0 < n_v; c0 += blockDim.x) {
+    const int k = c0 + threadIdx.x;
+    const int f = (k < n_v && !chosen[k]) ? 1 : 0;
+    int total;
+    const int pos = block_excl_scan(f, sh, &total);
+    if (f) rj[base + pos] = k;
+    base += total;
+  }
+  __syncthreads();
+  const int R = base;
+  if (m == 0 || R == 0) return;
+  const int step = R / m;
+  const XT* Xt = X + (size_t)kept[j] * n_v * d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int q = warp; q < m; q += blockDim.x / 32) {
+    const int t = rj[q * step];
+    const double nn = ff_dot(Xt + (size_t)t * d, Xt + (size_t)t * d, d, lane);
+    if (lane == 0 && co + q < max_ctx) {
+      ctx_target[co + q] = t;
+      tnorm[co + q] = sqrt(nn);
+    }
+  }
+}
+
+// Grid (kept slot, block of TB unselected tokens).  assign[j][a] = target index of rest[a].
+template <typename XT>
+__global__ void __launch_bounds__(256) merge_assign_kernel(const XT* __restrict__ X, int n_v, int d,
+                                                           const int* __restrict__ kept,
+                                                           const int* __restrict__ n_kept,
+                                                           const int* __restrict__ sel_off,
+                                                           const int* __restrict__ ctx_off, int max_ctx,
+                                                           const int* __restrict__ rest,
+                                                           const int* __restrict__ ctx_target,
+                                                           const double* __restrict__ tnorm,
+                                                           int* __restrict__ assign) {
+  __shared__ float As[KC][TB + 4];
+  __shared__ float Bs[KC][TB + 4];
+  __shared__ float best_v[TB][2];
+  __shared__ int best_j[TB][2];
+  __shared__ float inv_n[TB];
+  const int j = blockIdx.x;
+  if (j >= *n_kept) return;
+  const int s = sel_off[j + 1] - sel_off[j];
+  const int R = n_v - s;
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  const int a0 = blockIdx.y * TB;
+  if (m == 0 || a0 >= R || co + m > max_ctx) return;
+  const int* rj = rest + (size_t)j * n_v;
+  const XT* Xt = X + (size_t)kept[j] * n_v * d;
+  const int tid = threadIdx.x, ti = tid >> 4, tj = tid & 15;
+  if (tid < TB) {
+    best_v[tid][0] = best_v[tid][1] = -INFINITY;
+    best_j[tid][0] = best_j[tid][1] = -1;
+  }
+  for (int b0 = 0; b0 < m; b0 += TB) {
+    if (tid < TB) {
+      const double nn = b0 + tid < m ? tnorm[co + b0 + tid] : 0.0;
+      inv_n[tid] = nn > 0.0 ? (float)(1.0 / nn) : 0.f;  // a zero target has similarity 0
+    }
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < d; k0 += KC) {
+      for (int q = tid; q < TB * KC; q += 256) {
+        const int row = q / KC, c = q % KC;
+        const int a = a0 + row, b = b0 + row;
+        As[c][row] = a < R ? load_x(Xt + (size_t)rj[a] * d + k0 + c) : 0.f;
+        Bs[c][row] = b < m ? load_x(Xt + (size_t)ctx_target[co + b] * d + k0 + c) : 0.f;
+      }
+      __syncthreads();
+      float part[4][4] = {};
+#pragma unroll 8
+      for (int k = 0; k < KC; ++k) {
+        const float4 av = *reinterpret_cast<const float4*>(&As[k][ti * 4]);
+        const float4 bv = *reinterpret_cast<const float4*>(&Bs[k][tj * 4]);
+        const float aa[4] = {av.x, av.y, av.z, av.w}, bb[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) part[r][c] = fmaf(aa[r], bb[c], part[r][c]);
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
+      __syncthreads();
+    }
+    // running top 2 per token: thread (ti, tj) offers its 4 x 4 candidates row by row
+    for (int w = 0; w < 16; ++w) {
+      if (tj == w) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int row = ti * 4 + r;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const int b = b0 + tj * 4 + c;
+            if (b >= m) continue;
+            const float v = acc[r][c] * inv_n[tj * 4 + c];
+            if (v > best_v[row][0] || (v == best_v[row][0] && b < best_j[row][0])) {
+              best_v[row][1] = best_v[row][0];
+              best_j[row][1] = best_j[row][0];
+              best_v[row][0] = v;
+              best_j[row][0] = b;
+            } else if (v > best_v[row][1] || (v == best_v[row][1] && b < best_j[row][1])) {
+              best_v[row][1] = v;
+              best_j[row][1] = b;
+            }
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // decide between the top two at ~fp64 accuracy: x.t1 / ||t1|| vs x.t2 / ||t2||
+  const int warp = tid >> 5, lane = tid & 31;
+  for (int row = warp; row < TB; row += 8) {
+    const int a = a0 + row;
+    if (a >= R) break;
+    const int k = rj[a];
+    int choice = best_j[row][0];
+    const int j2 = best_j[row][1];
+    if (j2 >= 0) {
+      const int t1 = ctx_target[co + choice], t2 = ctx_target[co + j2];
+      const double d1 = ff_dot(Xt + (size_t)k * d, Xt + (size_t)t1 * d, d, lane);
+      const double d2 = ff_dot(Xt + (size_t)k * d, Xt + (size_t)t2 * d, d, lane);
+      const double n1 = tnorm[co + choice], n2 = tnorm[co + j2];
+      const double s1 = n1 > 0.0 ? d1 / n1 : 0.0, s2 = n2 > 0.0 ? d2 / n2 : 0.0;
+      if (s2 > s1 || (s2 == s1 && j2 < choice)) choice = j2;
+    }
+    if (lane == 0) assign[(size_t)j * n_v + a] = choice;
+  }
+}
+
+// Grid (kept slot, y): CTA (j, y) forms contextual tokens q = y, y + gridDim.y, ... of slot j.
+// Its members are scanned in ascending token index (the target at its own index), every thread
+// summing MV of the head dims in fp32; the mean is stored as bf16.
+constexpr int MT = 256, MV = RIFT_MERGE_MAX_D / MT;
+template <typename XT>
+__global__ void __launch_bounds__(MT) merge_mean_kernel(const XT* __restrict__ X, int n_v, int d,
+                                                        const int* __restrict__ kept, const int* __restrict__ n_kept,
+                                                        const int* __restrict__ sel_off,
+                                                        const int* __restrict__ ctx_off, int max_ctx,
+                                                        const int* __restrict__ rest,
+                                                        const int* __restrict__ assign, uint16_t* __restrict__ ctx) {
+  const int j = blockIdx.x;
+  if (j >= *n_kept) return;
+  const int R = n_v - (sel_off[j + 1] - sel_off[j]);
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  if (m == 0 || co + m > max_ctx) return;
+  const int step = R / m;
+  const int* rj = rest + (size_t)j * n_v;
+  const int* aj = assign + (size_t)j * n_v;
+  const XT* Xt = X + (size_t)kept[j] * n_v * d;
+  for (int q = blockIdx.y; q < m; q += gridDim.y) {
+    float acc[MV];
+#pragma unroll
+    for (int v = 0; v < MV; ++v) acc[v] = 0.f;
+    int cnt = 0;
+    for (int a = 0; a < R; ++a) {
+      const bool target = a % step == 0 && a / step < m;
+      if (target ? a / step != q : aj[a] != q) continue;
+      const XT* row = Xt + (size_t)rj[a] * d;
+#pragma unroll
+      for (int v = 0; v < MV; ++v) {
+        const int c = threadIdx.x + v * MT;
+        if (c < d) acc[v] += load_x(row + c);
+      }
+      ++cnt;
+    }
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(ctx) + (size_t)(co + q) * d;
+#pragma unroll
+    for (int v = 0; v < MV; ++v) {
+      const int c = threadIdx.x + v * MT;
+      if (c < d) out[c] = __float2bfloat16_rn(acc[v] / (float)cnt);
+    }
+  }
+}
+
+}  // namespace mg
+
+MergeLayout merge_layout(int N, int n_v) {
+  MergeLayout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
+  L.rest_off = take((size_t)N * n_v * sizeof(int));
+  L.assign_off = take((size_t)N * n_v * sizeof(int));
+  L.tnorm_off = take((size_t)N * n_v * sizeof(double));
+  L.total = off;
+  return L;
+}
+
+int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept, const int* n_kept,
+                 const int* budgets, const int* sel, const int* sel_off, uint16_t* ctx, int max_ctx, int* ctx_off,
+                 int* ctx_target, char* ws, cudaStream_t st) {
+  using namespace mg;
+  const MergeLayout L = merge_layout(N, n_v);
+  int* rest = reinterpret_cast<int*>(ws + L.rest_off);
+  int* assign = reinterpret_cast<int*>(ws + L.assign_off);
+  double* tnorm = reinterpret_cast<double*>(ws + L.tnorm_off);
+  merge_plan_kernel<<<1, 1024, 0, st>>>(n_kept, budgets, sel_off, N, n_v, max_ctx, ctx_off);
+  const dim3 ga(N, (n_v + TB - 1) / TB), gm(N, 16);
+  if (xdt == RIFT_BF16) {
+    const uint16_t* x = static_cast<const uint16_t*>(X);
+    merge_targets_kernel<uint16_t><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
+                                                      ctx_target, tnorm);
+    merge_assign_kernel<uint16_t><<<ga, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
+                                                      ctx_target, tnorm, assign);
+    merge_mean_kernel<uint16_t><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest, assign,
+                                                   ctx);
+  } else {
+    const float* x = static_cast<const float*>(X);
+    merge_targets_kernel<float><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
+                                                   ctx_target, tnorm);
+    merge_assign_kernel<float><<<ga, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
+                                                   ctx_target, tnorm, assign);
+    merge_mean_kernel<float><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest, assign, ctx);
+  }
+  return 4;
+}
+
+}  // namespace rift

@@ -1,5 +1,5 @@
-// Ragged packing on sm_103a: one sequence per kept tile, [system | selected tokens | query],
-// back to back, with cu_seqlens and per-row positions.
+// Ragged packing on sm_103a: one sequence per kept tile, [system | selected tokens | contextual
+// tokens (when merged) | query], back to back, with cu_seqlens and per-row positions.
 //
 // Each packed row is an 8 KB (d = 4096, bf16) copy.  For bf16 tokens a CTA owns 64 rows of one
 // sequence and one thread streams them through an 8-slot shared-memory ring with bulk copies
@@ -23,13 +23,14 @@ unsigned int read_clear_err_pack() {
 constexpr int PK_ROWS = 32;
 constexpr int PK_THREADS = 256;
 
-// cu_seqlens[j] = min(j, n) (S + Q) + sel_off[min(j, n)], T = cu_seqlens[n].
-__global__ void seqlens_kernel(const int* __restrict__ n_kept, const int* __restrict__ sel_off, int N,
-                               int S, int Q, int max_T, int* __restrict__ cu, int* __restrict__ T) {
+// cu_seqlens[j] = min(j, n) (S + Q) + sel_off[min(j, n)] + ctx_off[min(j, n)], T = cu_seqlens[n].
+__global__ void seqlens_kernel(const int* __restrict__ n_kept, const int* __restrict__ sel_off,
+                               const int* __restrict__ ctx_off, int N, int S, int Q, int max_T,
+                               int* __restrict__ cu, int* __restrict__ T) {
   const int n = *n_kept;
   for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= N; j += gridDim.x * blockDim.x) {
     const int jj = min(j, n);
-    const int v = jj * (S + Q) + sel_off[jj];
+    const int v = jj * (S + Q) + sel_off[jj] + (ctx_off ? ctx_off[jj] : 0);
     cu[j] = v;
     if (j == N) {
       *T = v;
@@ -43,14 +44,16 @@ __global__ void __launch_bounds__(PK_THREADS) pack_kernel(
     const XT* __restrict__ X, int N, int n_v, int d, const int* __restrict__ kept,
     const int* __restrict__ n_kept, const int* __restrict__ sel, const int* __restrict__ sel_off,
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
-    const uint16_t* __restrict__ embed, int vocab, uint16_t* __restrict__ packed, int max_T,
-    int* __restrict__ positions) {
+    const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
+    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
   const int j = blockIdx.x;
   if (j >= *n_kept) return;
   const int so = sel_off[j];
-  const int b = sel_off[j + 1] - so;
+  const int dom = sel_off[j + 1] - so;  // selected tokens, then m contextual ones
+  const int co = ctx_off ? ctx_off[j] : 0, m = ctx_off ? ctx_off[j + 1] - co : 0;
+  const int b = dom + m;
   const int L = S + b + Q;
-  const int base = j * (S + Q) + so;
+  const int base = j * (S + Q) + so + co;
   const int tile = kept[j];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int r_end = min(L, (blockIdx.y + 1) * PK_ROWS);
@@ -69,6 +72,9 @@ __global__ void __launch_bounds__(PK_THREADS) pack_kernel(
         continue;
       }
       const uint4* src = reinterpret_cast<const uint4*>(embed + (size_t)id * d);
+      for (int q = lane; q < nv8; q += 32) out[q] = src[q];
+    } else if (r >= S + dom) {
+      const uint4* src = reinterpret_cast<const uint4*>(ctx + (size_t)(co + r - S - dom) * d);
       for (int q = lane; q < nv8; q += 32) out[q] = src[q];
     } else {
       const int k = sel[so + r - S];
@@ -125,16 +131,18 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
     const uint16_t* __restrict__ X, int N, int n_v, int d, const int* __restrict__ kept,
     const int* __restrict__ n_kept, const int* __restrict__ sel, const int* __restrict__ sel_off,
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
-    const uint16_t* __restrict__ embed, int vocab, uint16_t* __restrict__ packed, int max_T,
-    int* __restrict__ positions) {
+    const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
+    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
   extern __shared__ __align__(128) uint8_t ring[];
   __shared__ __align__(8) uint64_t bars[PKB_SLOTS];
   const int j = blockIdx.x;
   if (j >= *n_kept) return;
   const int so = sel_off[j];
-  const int b = sel_off[j + 1] - so;
+  const int dom = sel_off[j + 1] - so;  // selected tokens, then m contextual ones
+  const int co = ctx_off ? ctx_off[j] : 0, m = ctx_off ? ctx_off[j + 1] - co : 0;
+  const int b = dom + m;
   const int L = S + b + Q;
-  const int base = j * (S + Q) + so;
+  const int base = j * (S + Q) + so + co;
   const int tile = kept[j];
   const int r0 = blockIdx.y * PKB_ROWS;
   const int n = min(L - r0, PKB_ROWS);
@@ -152,6 +160,7 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
       if (id < 0 || id >= vocab) { atomicOr(&g_err_pack, RIFT_EBIT_BADID); return nullptr; }
       return embed + (size_t)id * d;
     }
+    if (r >= S + dom) return ctx + (size_t)(co + r - S - dom) * d;
     const int k = sel[so + r - S];
     if (k < 0 || k >= n_v || tile < 0 || tile >= N) { atomicOr(&g_err_pack, RIFT_EBIT_BADID); return nullptr; }
     return X + ((size_t)tile * n_v + k) * d;
@@ -208,9 +217,10 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
 
 void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
                  const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
-                 const int* query_ids, int Q, const void* embed, int vocab, void* packed, int max_T,
-                 int* cu_seqlens, int* positions, int* T, cudaStream_t st) {
-  seqlens_kernel<<<(N + 1 + 255) / 256, 256, 0, st>>>(n_kept, sel_off, N, S, Q, max_T, cu_seqlens, T);
+                 const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
+                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, cudaStream_t st) {
+  seqlens_kernel<<<(N + 1 + 255) / 256, 256, 0, st>>>(n_kept, sel_off, ctx_off, N, S, Q, max_T, cu_seqlens, T);
+  const uint16_t* cx = static_cast<const uint16_t*>(ctx);
   const int max_L = S + n_v + Q;
   dim3 grid(N, (max_L + PK_ROWS - 1) / PK_ROWS);
   if (xdt == RIFT_BF16) {
@@ -223,11 +233,11 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
     dim3 gb(N, (max_L + PKB_ROWS - 1) / PKB_ROWS);
     pack_bulk_kernel<<<gb, 64, smem, st>>>(
         static_cast<const uint16_t*>(X), N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q,
-        static_cast<const uint16_t*>(embed), vocab, static_cast<uint16_t*>(packed), max_T, positions);
+        static_cast<const uint16_t*>(embed), vocab, cx, ctx_off, static_cast<uint16_t*>(packed), max_T, positions);
   } else
     pack_kernel<float><<<grid, PK_THREADS, 0, st>>>(
         static_cast<const float*>(X), N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q,
-        static_cast<const uint16_t*>(embed), vocab, static_cast<uint16_t*>(packed), max_T, positions);
+        static_cast<const uint16_t*>(embed), vocab, cx, ctx_off, static_cast<uint16_t*>(packed), max_T, positions);
 }
 
 }  // namespace rift

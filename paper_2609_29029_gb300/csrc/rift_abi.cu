@@ -98,7 +98,7 @@ rift_status rift_profile_read(double* ms, long long* launches, int n_classes) {
 
 long long rift_launch_count(void) { return g_launches.load(); }
 
-int rift_abi_version(void) { return 2; }
+int rift_abi_version(void) { return 3; }
 
 const char* rift_status_string(rift_status s) {
   switch (s) {
@@ -117,7 +117,7 @@ const char* rift_status_string(rift_status s) {
 rift_status rift_sync_status(rift_stream_t stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return RIFT_ERR_CUDA;
   unsigned int f = read_clear_err_score() | read_clear_err_select() | read_clear_err_pack() |
-                   read_clear_err_prefill() | read_clear_err_gemm() | read_clear_err_attn();
+                   read_clear_err_prefill() | read_clear_err_gemm() | read_clear_err_attn() | read_clear_err_merge();
   if (cudaGetLastError() != cudaSuccess) return RIFT_ERR_CUDA;
   if (f & RIFT_EBIT_BADID) return RIFT_ERR_BAD_ID;
   if (f & RIFT_EBIT_NONFINITE) return RIFT_ERR_NONFINITE;
@@ -190,6 +190,7 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
       return RIFT_ERR_INVALID;
   }
   if (!std::isfinite(pol.lambda)) return RIFT_ERR_INVALID;
+  if (pol.ctx_num < 0 || pol.ctx_den < 1 || pol.ctx_num >= pol.ctx_den) return RIFT_ERR_INVALID;
   prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
   launch_select(token_scores, tile_s, N, n_v, p, pol, u, kept, n_kept, budgets, sel, sel_off,
                 static_cast<cudaStream_t>(stream));
@@ -200,8 +201,9 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
 
 rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
                              const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
-                             const int* query_ids, int Q, const void* embed, int vocab, void* packed, int max_T,
-                             int* cu_seqlens, int* positions, int* T, rift_stream_t stream) {
+                             const int* query_ids, int Q, const void* embed, int vocab, const void* ctx,
+                             const int* ctx_off, void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
+                             rift_stream_t stream) {
   if (!dims_ok(N, n_v, d) || !X || !kept || !n_kept || !sel || !sel_off || !embed || !packed || !cu_seqlens ||
       !positions || !T)
     return RIFT_ERR_INVALID;
@@ -209,10 +211,34 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
   if (S < 0 || Q < 0 || (S > 0 && !sys_ids) || (Q > 0 && !query_ids) || vocab < 1 || max_T < 0)
     return RIFT_ERR_INVALID;
   if (!aligned16(X) || !aligned16(embed) || !aligned16(packed)) return RIFT_ERR_INVALID;
+  if ((ctx == nullptr) != (ctx_off == nullptr) || (ctx && !aligned16(ctx))) return RIFT_ERR_INVALID;
   prof_begin(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream));
-  launch_pack(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, packed,
-              max_T, cu_seqlens, positions, T, static_cast<cudaStream_t>(stream));
+  launch_pack(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, ctx, ctx_off,
+              packed, max_T, cu_seqlens, positions, T, static_cast<cudaStream_t>(stream));
   prof_end(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream), 2);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_merge_workspace_bytes(int N, int n_v) {
+  if (N < 1 || N > RIFT_MAX_TILES || n_v < 1 || n_v > RIFT_MAX_NV) return 0;
+  return merge_layout(N, n_v).total;
+}
+
+rift_status rift_merge_contextual(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
+                                  const int* n_kept, const int* budgets, const int* sel, const int* sel_off, void* ctx,
+                                  int max_ctx, int* ctx_off, int* ctx_target, void* ws, size_t ws_bytes,
+                                  rift_stream_t stream) {
+  if (!dims_ok(N, n_v, d) || !X || !kept || !n_kept || !budgets || !sel || !sel_off || !ctx_off || !ctx_target ||
+      max_ctx < 0 || (max_ctx > 0 && !ctx))
+    return RIFT_ERR_INVALID;
+  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
+  if (!aligned16(X) || (ctx && !aligned16(ctx))) return RIFT_ERR_INVALID;
+  if (!ws_ok(ws, ws_bytes, merge_layout(N, n_v).total)) return RIFT_ERR_INVALID;
+  prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
+  const int nk = launch_merge(X, xdt, N, n_v, d, kept, n_kept, budgets, sel, sel_off, static_cast<uint16_t*>(ctx),
+                              max_ctx, ctx_off, ctx_target, static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream), nk);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
 }

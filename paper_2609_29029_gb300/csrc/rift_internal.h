@@ -37,11 +37,23 @@ void launch_select(const float* token_scores, const float* tile_s, int N, int n_
                    const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
                    int* sel_off, cudaStream_t st);
 
+// ---- merge.cu ----
+struct MergeLayout {
+  size_t rest_off, assign_off, tnorm_off, total;
+};
+#define RIFT_MERGE_MAX_D 8192
+MergeLayout merge_layout(int N, int n_v);
+unsigned int read_clear_err_merge();
+// Returns the number of kernels launched.
+int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept, const int* n_kept,
+                 const int* budgets, const int* sel, const int* sel_off, uint16_t* ctx, int max_ctx, int* ctx_off,
+                 int* ctx_target, char* ws, cudaStream_t st);
+
 // ---- pack.cu ----
 void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
                  const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
-                 const int* query_ids, int Q, const void* embed, int vocab, void* packed, int max_T,
-                 int* cu_seqlens, int* positions, int* T, cudaStream_t st);
+                 const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
+                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, cudaStream_t st);
 
 // ---- prefill (prefill.cu, gemm.cu, attention.cu) ----
 struct PrefillLayout {

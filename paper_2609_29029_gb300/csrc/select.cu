@@ -25,7 +25,7 @@ unsigned int read_clear_err_select() {
 constexpr int PB_THREADS = 1024;
 
 __global__ void __launch_bounds__(PB_THREADS) prune_budget_kernel(
-    const float* __restrict__ s, int N, const float* __restrict__ p_ext, rift_policy pol,
+    const float* __restrict__ s, int N, int n_v, const float* __restrict__ p_ext, rift_policy pol,
     float* __restrict__ u, int* __restrict__ kept, int* __restrict__ n_kept,
     int* __restrict__ budgets, int* __restrict__ sel_off) {
   __shared__ float rmin[32], rmax[32];
@@ -97,6 +97,9 @@ __global__ void __launch_bounds__(PB_THREADS) prune_budget_kernel(
       }
       b = pol.C[best];
       budgets[j] = b;
+      // with the merge on, c - floor(ctx_num c / ctx_den) of the c tokens are selected (the
+      // rest of the budget is contextual tokens); the full budget selects every token
+      if (pol.ctx_num > 0 && b < n_v) b -= (pol.ctx_num * b) / pol.ctx_den;
     }
     int total;
     int pos = block_excl_scan(b, sh, &total);
@@ -130,7 +133,7 @@ __global__ void __launch_bounds__(TB_THREADS) topb_kernel(const float* __restric
   if (j >= *n_kept) return;
   const int tid = threadIdx.x, lane = tid & 31;
   const int tile = kept[j];
-  const int b = budgets[j];
+  const int b = sel_off[j + 1] - sel_off[j];  // tokens to select (the budget less its contextual tokens)
   uint32_t key[TB_KPT];
   bool valid[TB_KPT];
   bool bad = false;
@@ -209,7 +212,7 @@ __global__ void __launch_bounds__(TB_THREADS) topb_kernel(const float* __restric
 void launch_select(const float* token_scores, const float* tile_s, int N, int n_v, const float* p,
                    const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
                    int* sel_off, cudaStream_t st) {
-  prune_budget_kernel<<<1, PB_THREADS, 0, st>>>(tile_s, N, p, pol, u, kept, n_kept, budgets, sel_off);
+  prune_budget_kernel<<<1, PB_THREADS, 0, st>>>(tile_s, N, n_v, p, pol, u, kept, n_kept, budgets, sel_off);
   topb_kernel<<<N, TB_THREADS, 0, st>>>(token_scores, n_v, kept, n_kept, budgets, sel_off, sel);
 }
 

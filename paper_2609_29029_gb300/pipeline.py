@@ -88,6 +88,9 @@ class ScenePipeline:
         self.knn_m = knn_m
         self.m = min(knn_m, N - 1)
         self.policy = abi.make_policy(policy)
+        # contextual tokens (the merge of Stage 2): at most floor(ctx_num c / ctx_den) per tile
+        num, den = getattr(policy, "ctx_num", 0), getattr(policy, "ctx_den", 64)
+        self.max_m = max([(num * c) // den for c in policy.C if c < n_v] + [0]) if num else 0
         self.model = model
         self.max_T = max_T if max_T is not None else N * (S + n_v + Q)
         self.max_len = S + n_v + Q
@@ -110,6 +113,12 @@ class ScenePipeline:
         self.positions = torch.empty(max(self.max_T, 1), **i32)
         self.T = torch.zeros(1, **i32)
         self.counts_host = torch.zeros(2, dtype=torch.int32, pin_memory=True)
+        self.max_ctx = N * self.max_m
+        self.ctx = torch.empty(max(self.max_ctx, 1), d, dtype=torch.bfloat16, device=dev) if self.max_m else None
+        self.ctx_off = torch.zeros(N + 1, **i32) if self.max_m else None
+        self.ctx_target = torch.empty(max(self.max_ctx, 1), **i32) if self.max_m else None
+        self.ws_merge_bytes = abi.merge_workspace_bytes(N, n_v) if self.max_m else 0
+        self.ws_merge = torch.empty(self.ws_merge_bytes, dtype=torch.uint8, device=dev) if self.max_m else None
         self.ws_score_bytes = abi.score_workspace_bytes(N, n_v, d, M)
         self.ws_score = torch.empty(self.ws_score_bytes, dtype=torch.uint8, device=dev)
         self.ws_prefill = None
@@ -135,11 +144,19 @@ class ScenePipeline:
         abi.select_budgeted_tokens(self.token_scores, self.tile_s, self.N, self.n_v, p, self.policy, self.u,
                                    self.kept, self.n_kept, self.budgets, self.sel, self.sel_off, None, 0, stream)
 
+    def merge(self, X, stream=None):
+        """a7b (when the policy merges): the contextual tokens of every kept tile."""
+        abi.merge_contextual(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.budgets, self.sel,
+                             self.sel_off, self.ctx, self.max_ctx, self.ctx_off, self.ctx_target, self.ws_merge,
+                             self.ws_merge_bytes, stream)
+
     def pack(self, X, embed, sys_ids, query_ids, stream=None):
         """a8: the packed batch, cu_seqlens and positions."""
+        if self.max_m:
+            self.merge(X, stream)
         abi.pack_ragged(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.sel, self.sel_off,
                         sys_ids, self.S, query_ids, self.Q, embed, embed.shape[0], self.packed, self.max_T,
-                        self.cu, self.positions, self.T, stream)
+                        self.cu, self.positions, self.T, stream, ctx=self.ctx, ctx_off=self.ctx_off)
 
     def read_counts(self, stream=None):
         """Sync, check device error flags and read (n_kept, T) back to the host."""

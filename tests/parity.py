@@ -104,9 +104,10 @@ def margins(sel: O.Selection, wl) -> dict:
             wb = min(wb, (U[0] - U[1]) / EPS_U)
     out["budget"] = wb
     wt, amb = np.inf, []
-    for j, (i, b) in enumerate(zip(sel.kept, sel.budgets)):
+    for j, (i, idx) in enumerate(zip(sel.kept, sel.sel)):
+        b = len(idx)  # the selected tokens: the budget less its contextual tokens when merging
         r = np.sort(sel.r32[i].astype(np.float64))[::-1]
-        if b < len(r):
+        if 0 < b < len(r):
             mj = (r[b - 1] - r[b]) / (EPS_R * np.abs(r).max())
             wt = min(wt, mj)
             if mj < 1.0:

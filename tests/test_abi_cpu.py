@@ -31,7 +31,7 @@ def test_library_exports_every_declared_symbol(riftlib):
 def test_status_strings(riftlib):
     assert riftlib.status_string(0) == "ok"
     assert riftlib.status_string(riftlib.RIFT_ERR_CAPACITY) == "output capacity exceeded"
-    assert riftlib.abi_version() == 2
+    assert riftlib.abi_version() == 3
 
 
 FAKE = 0x10000  # a 16-byte aligned non-null address; validation rejects before using it
@@ -95,10 +95,14 @@ def test_select_rejects_bad_policies(riftlib):
 def test_pack_and_prefill_reject_bad_arguments(riftlib):
     lib = riftlib.lib
     INV = riftlib.RIFT_ERR_INVALID
-    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, None, 8, FAKE, 16, FAKE, 1000, FAKE,
-                                100, FAKE, FAKE, FAKE, 0) == INV  # S > 0 without ids
-    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000,
-                                FAKE + 2, 100, FAKE, FAKE, FAKE, 0) == INV  # misaligned output
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, None, 8, FAKE, 16, FAKE, 1000, None,
+                                None, FAKE, 100, FAKE, FAKE, FAKE, 0) == INV  # S > 0 without ids
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000, None,
+                                None, FAKE + 2, 100, FAKE, FAKE, FAKE, 0) == INV  # misaligned output
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000, FAKE,
+                                None, FAKE, 100, FAKE, FAKE, FAKE, 0) == INV  # contextual rows without offsets
+    assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000, FAKE + 8,
+                                FAKE, FAKE, 100, FAKE, FAKE, FAKE, 0) == INV  # misaligned contextual rows
     m = riftlib.Model()
     m.n_layers, m.d, m.n_heads, m.head_dim, m.ffn, m.eps, m.rope_theta = 2, 256, 4, 64, 688, 1e-6, 1e4
     assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0  # null weight arrays
@@ -155,3 +159,27 @@ def test_query_prep_rejects_bad_arguments(riftlib):
     assert lib.rift_query_prep(FAKE, 1000, 256, FAKE, 0, 16, FAKE, 8, FAKE, FAKE, 0) == INV
     assert lib.rift_query_prep(FAKE, 1000, 256, FAKE, 1, 16, None, 8, FAKE, FAKE, 0) == INV
     assert lib.rift_query_prep(FAKE, 1000, 200, FAKE, 1, 16, FAKE, 8, FAKE, FAKE, 0) == INV
+
+
+def test_merge_and_policy_reject_bad_arguments(riftlib):
+    lib = riftlib.lib
+    INV = riftlib.RIFT_ERR_INVALID
+    ws = lib.rift_merge_workspace_bytes(4, 576)
+    assert ws > 0 and lib.rift_merge_workspace_bytes(0, 576) == 0 and lib.rift_merge_workspace_bytes(4, 2000) == 0
+
+    def call(**kw):
+        a = dict(X=FAKE, xdt=1, N=4, n_v=576, d=256, kept=FAKE, nk=FAKE, bud=FAKE, sel=FAKE, off=FAKE, ctx=FAKE,
+                 max_ctx=100, coff=FAKE, tgt=FAKE, ws=FAKE, wsb=ws)
+        a.update(kw)
+        return lib.rift_merge_contextual(a["X"], a["xdt"], a["N"], a["n_v"], a["d"], a["kept"], a["nk"], a["bud"],
+                                         a["sel"], a["off"], a["ctx"], a["max_ctx"], a["coff"], a["tgt"], a["ws"],
+                                         a["wsb"], 0)
+
+    assert call(X=None) == INV and call(coff=None) == INV and call(tgt=None) == INV
+    assert call(ctx=None) == INV and call(max_ctx=-1) == INV and call(ctx=FAKE + 4) == INV
+    assert call(wsb=ws - 1) == INV and call(xdt=5) == INV and call(d=100) == INV
+    # policy: 0 <= ctx_num < ctx_den
+    for num, den in ((-1, 64), (64, 64), (1, 0)):
+        pol = _policy(riftlib, ctx_num=num, ctx_den=den)
+        assert lib.rift_select_budgeted_tokens(FAKE, FAKE, 4, 576, None, C.byref(pol), FAKE, FAKE, FAKE, FAKE,
+                                               FAKE, FAKE, None, 0, 0) == INV
