@@ -44,7 +44,7 @@ def parse():
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
-    ap.add_argument("--kernel-case", choices=["prefill", "score", "decode"],
+    ap.add_argument("--kernel-case", choices=["prefill", "score", "decode", "merge"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
                          "'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); each runs 3 times")
     return ap.parse_args()
@@ -410,6 +410,17 @@ def kernel_case(name: str):
         for _ in range(3):
             hid = H0.clone()
             abi.prefill_layers(dm.struct, hid, T, cu, len(lens), 635, pos, ws, need)
+        abi.sync_status()
+    elif name == "merge":
+        # the 400-tile scene's selection with Stage 2's merge, three times
+        wl = W.RIFT400_MERGE
+        s = wl.scene
+        sc = W.make_scene(s, wl.decoder.vocab, dev)
+        pipe = ScenePipeline(s.N, s.n_v, s.d, s.x_dtype, s.M, s.S, s.Q, wl.knn_m, wl.policy, device=dev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        for _ in range(3):
+            pipe.select(sc.X, sc.embed, torch.tensor(sc.query_ids, **i32), torch.tensor(sc.bg_ids, **i32))
+            pipe.merge(sc.X)
         abi.sync_status()
     elif name == "decode":
         # 4 layers of the 7B shape, 73 sequences of 130..635 cached rows (about the retained set

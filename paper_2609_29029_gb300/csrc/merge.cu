@@ -10,8 +10,9 @@
 //                         sums (good to ~2^-44) and compared as x.t1 ||t2|| vs x.t2 ||t1|| in fp64,
 //                         so the decision is the cosine argmax of the exact arithmetic (ties to
 //                         the lower target)
-//   merge_mean_kernel     per contextual token: its group's sum in ascending token index
-//                         (fp32), divided by the group size, stored as bf16
+//   merge_groups_kernel   the groups as member lists in ascending token index (counting sort)
+//   merge_mean_kernel     per contextual token: the fp32 sum of its members' rows in that order,
+//                         divided by the group size, stored as bf16
 #include "rift_internal.h"
 
 namespace rift {
@@ -28,7 +29,7 @@ unsigned int read_clear_err_merge() {
 namespace mg {
 
 constexpr int TB = 64;     // tokens and targets per block of the similarity pass
-constexpr int KC = 32;     // d-chunk
+constexpr int KC = 32;     // d-chunk staged per step (summed in 32-term sub-chunks)
 
 template <typename XT>
 __device__ __forceinline__ float load_x(const XT* p) {
@@ -38,20 +39,36 @@ __device__ __forceinline__ float load_x(const XT* p) {
     return *p;
 }
 
-// Float-float accumulation of a.b over d terms by one warp (TwoProduct with an FMA, TwoSum),
-// then the lanes' pairs summed in fp64.
+// Eight consecutive elements of a row (16-byte aligned) as floats.
+template <typename XT>
+__device__ __forceinline__ void load8(const XT* p, float (&v)[8]) {
+  if constexpr (sizeof(XT) == 2) {
+    unpack_bf16x8(*reinterpret_cast<const uint4*>(p), v);
+  } else {
+    const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+}
+
+// Float-float accumulation of a.b over d terms (d % 256 == 0) by one warp (TwoProduct with an
+// FMA, TwoSum), eight elements per lane and step, then the lanes' pairs summed in fp64.
 template <typename XT>
 __device__ double ff_dot(const XT* a, const XT* b, int d, int lane) {
   float hi = 0.f, lo = 0.f;
-  for (int k = lane; k < d; k += 32) {
-    const float x = load_x(a + k), y = load_x(b + k);
-    const float p = __fmul_rn(x, y);
-    const float pe = fmaf(x, y, -p);
-    const float s = __fadd_rn(hi, p);
-    const float bb = __fsub_rn(s, hi);
-    const float er = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(p, bb));
-    hi = s;
-    lo = __fadd_rn(lo, __fadd_rn(er, pe));
+  for (int k = lane * 8; k < d; k += 256) {
+    float x[8], y[8];
+    load8(a + k, x);
+    load8(b + k, y);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float p = __fmul_rn(x[e], y[e]);
+      const float pe = fmaf(x[e], y[e], -p);
+      const float s = __fadd_rn(hi, p);
+      const float bb = __fsub_rn(s, hi);
+      const float er = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(p, bb));
+      hi = s;
+      lo = __fadd_rn(lo, __fadd_rn(er, pe));
+    }
   }
   double acc = (double)hi + (double)lo;
 #pragma unroll
@@ -154,17 +171,18 @@ __global__ void __launch_bounds__(256) merge_assign_kernel(const XT* __restrict_
                                                            const int* __restrict__ ctx_target,
                                                            const double* __restrict__ tnorm,
                                                            int* __restrict__ assign) {
-  __shared__ float As[KC][TB + 4];
-  __shared__ float Bs[KC][TB + 4];
+  extern __shared__ float ab_sm[];  // As[KC][TB + 4], Bs[KC][TB + 4]
+  float (*As)[TB + 4] = reinterpret_cast<float (*)[TB + 4]>(ab_sm);
+  float (*Bs)[TB + 4] = reinterpret_cast<float (*)[TB + 4]>(ab_sm + KC * (TB + 4));
   __shared__ float best_v[TB][2];
   __shared__ int best_j[TB][2];
   __shared__ float inv_n[TB];
-  const int j = blockIdx.x;
+  const int j = blockIdx.y;  // the token blocks of one slot are adjacent: its target rows stay in L2
   if (j >= *n_kept) return;
   const int s = sel_off[j + 1] - sel_off[j];
   const int R = n_v - s;
   const int co = ctx_off[j], m = ctx_off[j + 1] - co;
-  const int a0 = blockIdx.y * TB;
+  const int a0 = blockIdx.x * TB;
   if (m == 0 || a0 >= R || co + m > max_ctx) return;
   const int* rj = rest + (size_t)j * n_v;
   const XT* Xt = X + (size_t)kept[j] * n_v * d;
@@ -179,29 +197,52 @@ __global__ void __launch_bounds__(256) merge_assign_kernel(const XT* __restrict_
       inv_n[tid] = nn > 0.0 ? (float)(1.0 / nn) : 0.f;  // a zero target has similarity 0
     }
     float acc[4][4] = {};
-    for (int k0 = 0; k0 < d; k0 += KC) {
-      for (int q = tid; q < TB * KC; q += 256) {
-        const int row = q / KC, c = q % KC;
-        const int a = a0 + row, b = b0 + row;
-        As[c][row] = a < R ? load_x(Xt + (size_t)rj[a] * d + k0 + c) : 0.f;
-        Bs[c][row] = b < m ? load_x(Xt + (size_t)ctx_target[co + b] * d + k0 + c) : 0.f;
+    // 64 rows x KC columns per operand and chunk: four 8-column groups per thread and operand,
+    // kept packed while the next chunk's loads are in flight
+    const int srow = tid >> 2, scol = (tid & 3) * 8;
+    const XT* pa = a0 + srow < R ? Xt + (size_t)rj[a0 + srow] * d + scol : nullptr;
+    const XT* pb = b0 + srow < m ? Xt + (size_t)ctx_target[co + b0 + srow] * d + scol : nullptr;
+    constexpr int NG = KC / 32;  // 8-column groups per thread and operand
+    float va[NG][8], vb[NG][8];
+    auto fetch = [&](int k0) {
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) va[g][e] = vb[g][e] = 0.f;
+        if (k0 + 32 * g >= d) continue;  // d % 32 == 0: a group is wholly inside the row or past it
+        if (pa) load8(pa + k0 + 32 * g, va[g]);
+        if (pb) load8(pb + k0 + 32 * g, vb[g]);
       }
+    };
+    fetch(0);
+    for (int k0 = 0; k0 < d; k0 += KC) {
+#pragma unroll
+      for (int g = 0; g < NG; ++g)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          As[32 * g + scol + e][srow] = va[g][e];
+          Bs[32 * g + scol + e][srow] = vb[g][e];
+        }
       __syncthreads();
-      float part[4][4] = {};
+      if (k0 + KC < d) fetch(k0 + KC);
+#pragma unroll 1
+      for (int kc = 0; kc < KC; kc += 32) {
+        float part[4][4] = {};
 #pragma unroll 8
-      for (int k = 0; k < KC; ++k) {
-        const float4 av = *reinterpret_cast<const float4*>(&As[k][ti * 4]);
-        const float4 bv = *reinterpret_cast<const float4*>(&Bs[k][tj * 4]);
-        const float aa[4] = {av.x, av.y, av.z, av.w}, bb[4] = {bv.x, bv.y, bv.z, bv.w};
+        for (int k = kc; k < kc + 32; ++k) {
+          const float4 av = *reinterpret_cast<const float4*>(&As[k][ti * 4]);
+          const float4 bv = *reinterpret_cast<const float4*>(&Bs[k][tj * 4]);
+          const float aa[4] = {av.x, av.y, av.z, av.w}, bb[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+          for (int r = 0; r < 4; ++r)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) part[r][c] = fmaf(aa[r], bb[c], part[r][c]);
+        }
 #pragma unroll
         for (int r = 0; r < 4; ++r)
 #pragma unroll
-          for (int c = 0; c < 4; ++c) part[r][c] = fmaf(aa[r], bb[c], part[r][c]);
+          for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
       }
-#pragma unroll
-      for (int r = 0; r < 4; ++r)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
       __syncthreads();
     }
     // running top 2 per token: thread (ti, tj) offers its 4 x 4 candidates row by row
@@ -250,17 +291,16 @@ __global__ void __launch_bounds__(256) merge_assign_kernel(const XT* __restrict_
   }
 }
 
-// Grid (kept slot, y): CTA (j, y) forms contextual tokens q = y, y + gridDim.y, ... of slot j.
-// Its members are scanned in ascending token index (the target at its own index), every thread
-// summing MV of the head dims in fp32; the mean is stored as bf16.
-constexpr int MT = 256, MV = RIFT_MERGE_MAX_D / MT;
-template <typename XT>
-__global__ void __launch_bounds__(MT) merge_mean_kernel(const XT* __restrict__ X, int n_v, int d,
-                                                        const int* __restrict__ kept, const int* __restrict__ n_kept,
-                                                        const int* __restrict__ sel_off,
-                                                        const int* __restrict__ ctx_off, int max_ctx,
-                                                        const int* __restrict__ rest,
-                                                        const int* __restrict__ assign, uint16_t* __restrict__ ctx) {
+// One CTA per kept slot: the slot's groups as member lists, ascending token index within each
+// group (targets at their own index): gstart[j][q] .. gstart[j][q+1] in memb[j].  A counting sort
+// whose placement pass runs in token order on one thread.
+__global__ void __launch_bounds__(256) merge_groups_kernel(int n_v, const int* __restrict__ n_kept,
+                                                           const int* __restrict__ sel_off,
+                                                           const int* __restrict__ ctx_off, int max_ctx,
+                                                           const int* __restrict__ rest,
+                                                           const int* __restrict__ assign, int* __restrict__ memb,
+                                                           int* __restrict__ gstart) {
+  __shared__ int cnt[RIFT_MAX_NV + 1];
   const int j = blockIdx.x;
   if (j >= *n_kept) return;
   const int R = n_v - (sel_off[j + 1] - sel_off[j]);
@@ -269,28 +309,73 @@ __global__ void __launch_bounds__(MT) merge_mean_kernel(const XT* __restrict__ X
   const int step = R / m;
   const int* rj = rest + (size_t)j * n_v;
   const int* aj = assign + (size_t)j * n_v;
+  auto group = [&](int a) { return (a % step == 0 && a / step < m) ? a / step : aj[a]; };
+  for (int q = threadIdx.x; q <= m; q += blockDim.x) cnt[q] = 0;
+  __syncthreads();
+  for (int a = threadIdx.x; a < R; a += blockDim.x) atomicAdd(&cnt[group(a)], 1);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int* gs = gstart + (size_t)j * (n_v + 1);
+    int acc = 0;
+    for (int q = 0; q < m; ++q) {  // cnt becomes each group's next free slot
+      const int c = cnt[q];
+      gs[q] = acc;
+      cnt[q] = acc;
+      acc += c;
+    }
+    gs[m] = acc;
+    int* mj = memb + (size_t)j * n_v;
+    for (int a = 0; a < R; ++a) mj[cnt[group(a)]++] = rj[a];
+  }
+}
+
+// Grid (kept slot, y), 256 threads: contextual token q = y, y + gridDim.y, ... is the mean of its
+// group's rows, summed in fp32 in member order (ascending index), each thread owning d / 256 of
+// the columns; stored as bf16.
+constexpr int MT = 256, MV = RIFT_MERGE_MAX_D / (MT * 8);
+template <typename XT>
+__global__ void __launch_bounds__(MT) merge_mean_kernel(const XT* __restrict__ X, int n_v, int d,
+                                                        const int* __restrict__ kept, const int* __restrict__ n_kept,
+                                                        const int* __restrict__ ctx_off, int max_ctx,
+                                                        const int* __restrict__ memb, const int* __restrict__ gstart,
+                                                        uint16_t* __restrict__ ctx) {
+  const int j = blockIdx.x;
+  if (j >= *n_kept) return;
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  if (m == 0 || co + m > max_ctx) return;
+  const int* gs = gstart + (size_t)j * (n_v + 1);
+  const int* mj = memb + (size_t)j * n_v;
   const XT* Xt = X + (size_t)kept[j] * n_v * d;
   for (int q = blockIdx.y; q < m; q += gridDim.y) {
-    float acc[MV];
+    const int g0 = gs[q], g1 = gs[q + 1];
+    float acc[MV][8];
 #pragma unroll
-    for (int v = 0; v < MV; ++v) acc[v] = 0.f;
-    int cnt = 0;
-    for (int a = 0; a < R; ++a) {
-      const bool target = a % step == 0 && a / step < m;
-      if (target ? a / step != q : aj[a] != q) continue;
-      const XT* row = Xt + (size_t)rj[a] * d;
+    for (int v = 0; v < MV; ++v)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[v][e] = 0.f;
+    for (int g = g0; g < g1; ++g) {
+      const XT* row = Xt + (size_t)mj[g] * d;
 #pragma unroll
       for (int v = 0; v < MV; ++v) {
-        const int c = threadIdx.x + v * MT;
-        if (c < d) acc[v] += load_x(row + c);
+        const int c = (threadIdx.x + v * MT) * 8;
+        if (c < d) {
+          float x[8];
+          load8(row + c, x);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[v][e] += x[e];
+        }
       }
-      ++cnt;
     }
-    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(ctx) + (size_t)(co + q) * d;
+    const float inv = 1.f / (float)(g1 - g0);
 #pragma unroll
     for (int v = 0; v < MV; ++v) {
-      const int c = threadIdx.x + v * MT;
-      if (c < d) out[c] = __float2bfloat16_rn(acc[v] / (float)cnt);
+      const int c = (threadIdx.x + v * MT) * 8;
+      if (c < d) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) w[e] = pack_bf16x2(acc[v][2 * e] * inv, acc[v][2 * e + 1] * inv);
+        *reinterpret_cast<uint4*>(ctx + (size_t)(co + q) * d + c) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
     }
   }
 }
@@ -304,6 +389,8 @@ MergeLayout merge_layout(int N, int n_v) {
   L.rest_off = take((size_t)N * n_v * sizeof(int));
   L.assign_off = take((size_t)N * n_v * sizeof(int));
   L.tnorm_off = take((size_t)N * n_v * sizeof(double));
+  L.memb_off = take((size_t)N * n_v * sizeof(int));
+  L.gstart_off = take((size_t)N * (n_v + 1) * sizeof(int));
   L.total = off;
   return L;
 }
@@ -316,25 +403,39 @@ int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
   int* rest = reinterpret_cast<int*>(ws + L.rest_off);
   int* assign = reinterpret_cast<int*>(ws + L.assign_off);
   double* tnorm = reinterpret_cast<double*>(ws + L.tnorm_off);
+  int* memb = reinterpret_cast<int*>(ws + L.memb_off);
+  int* gstart = reinterpret_cast<int*>(ws + L.gstart_off);
   merge_plan_kernel<<<1, 1024, 0, st>>>(n_kept, budgets, sel_off, N, n_v, max_ctx, ctx_off);
-  const dim3 ga(N, (n_v + TB - 1) / TB), gm(N, 16);
+  const dim3 ga((n_v + TB - 1) / TB, N), gm(N, 32);
+  const size_t ab_bytes = 2 * (size_t)KC * (TB + 4) * sizeof(float);
   if (xdt == RIFT_BF16) {
     const uint16_t* x = static_cast<const uint16_t*>(X);
     merge_targets_kernel<uint16_t><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
                                                       ctx_target, tnorm);
-    merge_assign_kernel<uint16_t><<<ga, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
+    static bool attr16 = false;
+    if (!attr16) {
+      cudaFuncSetAttribute(merge_assign_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ab_bytes);
+      attr16 = true;
+    }
+    merge_assign_kernel<uint16_t><<<ga, 256, ab_bytes, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
                                                       ctx_target, tnorm, assign);
-    merge_mean_kernel<uint16_t><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest, assign,
-                                                   ctx);
+    merge_groups_kernel<<<N, 256, 0, st>>>(n_v, n_kept, sel_off, ctx_off, max_ctx, rest, assign, memb, gstart);
+    merge_mean_kernel<uint16_t><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, ctx_off, max_ctx, memb, gstart, ctx);
   } else {
     const float* x = static_cast<const float*>(X);
     merge_targets_kernel<float><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
                                                    ctx_target, tnorm);
-    merge_assign_kernel<float><<<ga, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
+    static bool attr32 = false;
+    if (!attr32) {
+      cudaFuncSetAttribute(merge_assign_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ab_bytes);
+      attr32 = true;
+    }
+    merge_assign_kernel<float><<<ga, 256, ab_bytes, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
                                                    ctx_target, tnorm, assign);
-    merge_mean_kernel<float><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest, assign, ctx);
+    merge_groups_kernel<<<N, 256, 0, st>>>(n_v, n_kept, sel_off, ctx_off, max_ctx, rest, assign, memb, gstart);
+    merge_mean_kernel<float><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, ctx_off, max_ctx, memb, gstart, ctx);
   }
-  return 4;
+  return 5;
 }
 
 }  // namespace rift

@@ -39,7 +39,7 @@ void launch_select(const float* token_scores, const float* tile_s, int N, int n_
 
 // ---- merge.cu ----
 struct MergeLayout {
-  size_t rest_off, assign_off, tnorm_off, total;
+  size_t rest_off, assign_off, tnorm_off, memb_off, gstart_off, total;
 };
 #define RIFT_MERGE_MAX_D 8192
 MergeLayout merge_layout(int N, int n_v);

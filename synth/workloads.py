@@ -140,7 +140,11 @@ RIFT1600 = Workload(
     LLAVA7B, RIFT_POLICY_SKEW, knn_m=6,
     description="1600 tiles, Pareto(1.5) planted strengths on every tile, elastic budgets with lambda=0.10")
 
-WORKLOADS = {w.name: w for w in (TINY, EXH16, EXH400, RIFT400, RIFT1600)}
+RIFT400_MERGE = replace(RIFT400, name="rift400_7b_merge", policy=RIFT_POLICY_MERGE,
+                        description="the rift400_7b query with Stage 2's merge: each budget holds "
+                                    "floor(10 c / 64) contextual tokens merged from the unselected ones")
+
+WORKLOADS = {w.name: w for w in (TINY, EXH16, EXH400, RIFT400, RIFT1600, RIFT400_MERGE)}
 SWEEP_N = (100, 400, 1600, 6400)
 
 
