@@ -142,6 +142,29 @@ def to_f32(x) -> np.ndarray:
     return np.asarray(x, dtype=np.float64).astype(F32)
 
 
+def quadrant_scores(X_tile: torch.Tensor, t, B) -> torch.Tensor:
+    """Eq. 1 of the four quadrants of the tile's token grid (Section 2.3, Stage 2: a predictor
+    feature): tokens k = row * g + col of the g x g grid (n_v = g^2, g even) split into rows
+    < g/2 or not and columns < g/2 or not; quadrant order top-left, top-right, bottom-left,
+    bottom-right; each scored as l2norm(mean of its tokens), fp64 [4]."""
+    n_v = X_tile.shape[0]
+    g = int(round(math.sqrt(n_v)))
+    if g * g != n_v or g % 2:
+        raise OracleError("quadrants need an even square token grid")
+    h = g // 2
+    x = X_tile.to(torch.float64).view(g, g, -1)
+    quads = [x[:h, :h], x[:h, h:], x[h:, :h], x[h:, h:]]
+    V = torch.stack([l2norm(q.reshape(-1, q.shape[-1]).sum(dim=0)) for q in quads])
+    return margin(V, t, B)
+
+
+def token_stats(r_tile) -> tuple:
+    """(max, mean, population standard deviation) of a tile's token scores, in fp64."""
+    r = np.asarray(r_tile, dtype=np.float64)
+    mean = float(r.sum() / r.size)
+    return float(r.max()), mean, float(math.sqrt(((r - mean) ** 2).sum() / r.size))
+
+
 # ------------------------------------------------------------------------------------------
 # a4  kNN smoothing (Appendix B Step 2; Listing 1 comment: smoothed with the 6 most similar tiles)
 # ------------------------------------------------------------------------------------------

@@ -582,3 +582,50 @@ def test_selection_with_merge_splits_every_budget():
         a = cu[j] + S
         assert torch.equal(H0[a:a + len(idx)], sc.X[i][idx].to(torch.bfloat16))
         assert torch.equal(H0[a + len(idx):a + len(idx) + ctx.shape[0]], ctx.to(torch.bfloat16))
+
+
+# ------------------------------- predictor features (Section 2.3, Stage 2: quadrant scores)
+
+def _tq(d=16, M=3, seed=30):
+    g = torch.Generator().manual_seed(seed)
+    t = O.l2norm(torch.randn(d, generator=g, dtype=torch.float64))
+    B = torch.stack([O.l2norm(torch.randn(d, generator=g, dtype=torch.float64)) for _ in range(M)])
+    return t, B
+
+
+def test_quadrants_of_a_uniform_tile_equal_the_tile_score():
+    t, B = _tq()
+    row = torch.randn(16, generator=torch.Generator().manual_seed(31), dtype=torch.float64)
+    X = row.repeat(36, 1)  # 6 x 6 grid, every token the same
+    q = O.quadrant_scores(X, t, B)
+    s = O.margin(O.tile_embedding(X)[None, :], t, B)[0]
+    assert torch.allclose(q, s.expand(4), atol=1e-14)
+
+
+def test_quadrants_partition_the_grid_and_follow_a_planted_patch():
+    t, B = _tq()
+    g = torch.Generator().manual_seed(32)
+    X = torch.randn(64, 16, generator=g, dtype=torch.float64)  # 8 x 8 grid
+    # the pooled tile sum is the sum of the four quadrant sums: every token in exactly one quadrant
+    grid = X.view(8, 8, 16)
+    qs = [grid[:4, :4], grid[:4, 4:], grid[4:, :4], grid[4:, 4:]]
+    assert torch.allclose(sum(q.reshape(-1, 16).sum(0) for q in qs), X.sum(0), atol=1e-12)
+    # plant the query direction on a patch inside the bottom-right quadrant (rows 5-6, cols 5-7)
+    for r in (5, 6):
+        for c in (5, 6, 7):
+            X[r * 8 + c] += 6.0 * t
+    q = O.quadrant_scores(X, t, B)
+    assert int(torch.argmax(q)) == 3
+    # a left-right mirror of the grid swaps top-left/top-right and bottom-left/bottom-right
+    Xm = X.view(8, 8, 16).flip(1).reshape(64, 16)
+    assert torch.allclose(O.quadrant_scores(Xm, t, B), q[[1, 0, 3, 2]], atol=1e-14)
+    with pytest.raises(O.OracleError):
+        O.quadrant_scores(X[:63], t, B)
+
+
+def test_token_stats_match_numpy():
+    r = np.random.default_rng(33).standard_normal(576).astype(np.float32)
+    mx, mean, std = O.token_stats(r)
+    r64 = r.astype(np.float64)
+    assert mx == float(r64.max()) and mean == pytest.approx(float(r64.mean()), abs=1e-15)
+    assert std == pytest.approx(float(r64.std()), abs=1e-14)
