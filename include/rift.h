@@ -203,6 +203,26 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
                                         int* sel, int* sel_off,
                                         void* ws, size_t ws_bytes, rift_stream_t stream);
 
+/* ---- Predictor features (Section 2.3, Stage 2: the features of the paper's p_i predictor,
+ * computed for the listed tiles, e.g. the kept ones, whose p_i the budget rule uses) ----
+ *   X, xdt, N, n_v, d   the scene; t, B, M   as for rift_score_tiles (Eq. 1's query and
+ *              background embeddings); token_scores  from rift_score_tiles
+ *   tiles      int32 [*n_tiles] tile indices (device), or NULL for every tile (slot j = tile j)
+ *   features   out fp32 [N, RIFT_N_FEATURES]: slot j = (s_TL, s_TR, s_BL, s_BR, r_max, r_mean,
+ *              r_std): Eq. 1 of each quadrant's pooled embedding (quadrants of the g x g token grid,
+ *              n_v = g^2 with g even, tokens in row-major grid order; top-left, top-right,
+ *              bottom-left, bottom-right), then the max, mean and population standard deviation
+ *              of the tile's token scores
+ *   V          out fp32 [N, d] (nullable): slot j's tile embedding, l2norm of its pooled tokens
+ *   ws         rift_features_workspace_bytes(N, d) bytes
+ * n_v not an even square returns RIFT_ERR_UNSUPPORTED. */
+#define RIFT_N_FEATURES 7
+size_t rift_features_workspace_bytes(int N, int d);
+rift_status rift_tile_features(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t,
+                               const float* B, int M, const float* token_scores, const int* tiles,
+                               const int* n_tiles, float* features, float* V, void* ws,
+                               size_t ws_bytes, rift_stream_t stream);
+
 /* ---- a7b. Merge of the unselected tokens (Section 2.3, Stage 2: VisionZip's mechanism keeps
  * the dominant tokens and merges the remainder) ----
  * For kept slot j with m_j = budgets[j] - (sel_off[j+1] - sel_off[j]) contextual tokens (see

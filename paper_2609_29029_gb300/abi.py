@@ -56,6 +56,8 @@ SIGNATURES = {
                                          _vp, _vp, _sz, _vp]),
     "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp,
                               _vp, _i, _vp, _vp, _vp, _vp]),
+    "rift_features_workspace_bytes": (_sz, [_i, _i]),
+    "rift_tile_features": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "rift_merge_workspace_bytes": (_sz, [_i, _i]),
     "rift_merge_contextual": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz,
                                    _vp]),
@@ -182,6 +184,20 @@ def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query
                                 ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(ctx), ptr(ctx_off),
                                 ptr(packed), max_T, ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),
            "rift_pack_ragged")
+
+
+N_FEATURES = 7
+
+
+def features_workspace_bytes(N, d) -> int:
+    return lib.rift_features_workspace_bytes(N, d)
+
+
+def tile_features(X, xdt, N, n_v, d, t, B, M, token_scores, tiles, n_tiles, features, V, ws, ws_bytes,
+                  stream=None):
+    _check(lib.rift_tile_features(ptr(X), xdt, N, n_v, d, ptr(t), ptr(B), M, ptr(token_scores), ptr(tiles),
+                                  ptr(n_tiles), ptr(features), ptr(V), ptr(ws), ws_bytes, stream_handle(stream)),
+           "rift_tile_features")
 
 
 def merge_workspace_bytes(N, n_v) -> int:

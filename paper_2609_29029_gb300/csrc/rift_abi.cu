@@ -220,6 +220,30 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
   return RIFT_OK;
 }
 
+size_t rift_features_workspace_bytes(int N, int d) {
+  if (N < 1 || N > RIFT_MAX_TILES || d < 64 || d > 8192 || d % 64 != 0) return 0;
+  return features_layout(N, d).total;
+}
+
+rift_status rift_tile_features(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                               int M, const float* token_scores, const int* tiles, const int* n_tiles,
+                               float* features, float* V, void* ws, size_t ws_bytes, rift_stream_t stream) {
+  if (!dims_ok(N, n_v, d) || !X || !t || !token_scores || !features) return RIFT_ERR_INVALID;
+  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
+  if (M < 0 || M > 64 || (M > 0 && !B) || (tiles == nullptr) != (n_tiles == nullptr)) return RIFT_ERR_INVALID;
+  if (!aligned16(X) || !aligned16(features) || (V && !aligned16(V))) return RIFT_ERR_INVALID;
+  if (!ws_ok(ws, ws_bytes, features_layout(N, d).total)) return RIFT_ERR_INVALID;
+  int g = 0;
+  while ((g + 1) * (g + 1) <= n_v) ++g;
+  if (g * g != n_v || g % 2 != 0) return RIFT_ERR_UNSUPPORTED;
+  prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));
+  const int nk = launch_features(X, xdt, N, n_v, d, g, t, B, M, token_scores, tiles, n_tiles, features, V,
+                                 static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream), nk);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
 size_t rift_merge_workspace_bytes(int N, int n_v) {
   if (N < 1 || N > RIFT_MAX_TILES || n_v < 1 || n_v > RIFT_MAX_NV) return 0;
   return merge_layout(N, n_v).total;

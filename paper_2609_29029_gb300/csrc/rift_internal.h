@@ -37,6 +37,15 @@ void launch_select(const float* token_scores, const float* tile_s, int N, int n_
                    const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
                    int* sel_off, cudaStream_t st);
 
+// ---- features.cu ----
+struct FeaturesLayout {
+  size_t w_off, qsum_off, total;
+};
+FeaturesLayout features_layout(int N, int d);
+int launch_features(const void* X, rift_dtype xdt, int N, int n_v, int d, int g, const float* t, const float* B, int M,
+                    const float* token_scores, const int* tiles, const int* n_tiles, float* features, float* V,
+                    char* ws, cudaStream_t st);
+
 // ---- merge.cu ----
 struct MergeLayout {
   size_t rest_off, assign_off, tnorm_off, memb_off, gstart_off, total;

@@ -144,6 +144,17 @@ class ScenePipeline:
         abi.select_budgeted_tokens(self.token_scores, self.tile_s, self.N, self.n_v, p, self.policy, self.u,
                                    self.kept, self.n_kept, self.budgets, self.sel, self.sel_off, None, 0, stream)
 
+    def features(self, X, kept_only=True, V=None, stream=None):
+        """Predictor features (quadrant Eq. 1 scores, token-score max/mean/std) of the kept tiles
+        (slot j = kept[j]) or of every tile; after select()."""
+        out = torch.empty(self.N, abi.N_FEATURES, dtype=torch.float32, device=self.device)
+        need = abi.features_workspace_bytes(self.N, self.d)
+        ws = torch.empty(need, dtype=torch.uint8, device=self.device)
+        abi.tile_features(X, self.xdt, self.N, self.n_v, self.d, self.t, self.B if self.M else None, self.M,
+                          self.token_scores, self.kept if kept_only else None, self.n_kept if kept_only else None,
+                          out, V, ws, need, stream)
+        return out
+
     def merge(self, X, stream=None):
         """a7b (when the policy merges): the contextual tokens of every kept tile."""
         abi.merge_contextual(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.budgets, self.sel,

@@ -183,3 +183,23 @@ def test_merge_and_policy_reject_bad_arguments(riftlib):
         pol = _policy(riftlib, ctx_num=num, ctx_den=den)
         assert lib.rift_select_budgeted_tokens(FAKE, FAKE, 4, 576, None, C.byref(pol), FAKE, FAKE, FAKE, FAKE,
                                                FAKE, FAKE, None, 0, 0) == INV
+
+
+def test_tile_features_reject_bad_arguments(riftlib):
+    lib = riftlib.lib
+    INV = riftlib.RIFT_ERR_INVALID
+    ws = lib.rift_features_workspace_bytes(4, 256)
+    assert ws > 0 and lib.rift_features_workspace_bytes(4, 100) == 0
+
+    def call(**kw):
+        a = dict(X=FAKE, xdt=1, N=4, n_v=576, d=256, t=FAKE, B=FAKE, M=8, r=FAKE, tiles=None, nt=None, f=FAKE,
+                 V=None, ws=FAKE, wsb=ws)
+        a.update(kw)
+        return lib.rift_tile_features(a["X"], a["xdt"], a["N"], a["n_v"], a["d"], a["t"], a["B"], a["M"], a["r"],
+                                      a["tiles"], a["nt"], a["f"], a["V"], a["ws"], a["wsb"], 0)
+
+    assert call(X=None) == INV and call(r=None) == INV and call(f=None) == INV
+    assert call(tiles=FAKE) == INV                       # a list without its count
+    assert call(M=2, B=None) == INV and call(f=FAKE + 4) == INV and call(wsb=ws - 1) == INV
+    assert call(n_v=200) == riftlib.RIFT_ERR_UNSUPPORTED  # not a square grid
+    assert call(n_v=225) == riftlib.RIFT_ERR_UNSUPPORTED  # odd side: no quadrants
