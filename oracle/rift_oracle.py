@@ -424,6 +424,23 @@ def prefill_with_cache(H0_seq: torch.Tensor, get_layer, g_final, dec):
     return rmsnorm(h, g_final.to(torch.float64), dec.eps), cache
 
 
+def extend_with_cache(H_new: torch.Tensor, cache, get_layer, g_final, dec):
+    """The rows H_new [n, d] appended after the P cached rows of a sequence (positions P ..
+    P + n - 1), each attending to the cache and causally to the new rows: their final hidden
+    states fp64 [n, d] and, per layer, their (keys after RoPE, values) fp64 [n, d].  With the
+    system prompt as the cache this is the prefill of a sequence's suffix over a shared prefix."""
+    h = H_new.to(torch.float64)
+    P = cache[0][0].shape[0]
+    pos = torch.arange(P, P + h.shape[0])
+    new = []
+    for l in range(dec.n_layers):
+        kp = cache[l][0].view(P, dec.n_heads, dec.head_dim)
+        vp = cache[l][1].view(P, dec.n_heads, dec.head_dim)
+        h, k, v = decoder_layer_cached(h, get_layer(l), dec, pos, kp, vp)
+        new.append((k.reshape(-1, dec.d), v.reshape(-1, dec.d)))
+    return rmsnorm(h, g_final.to(torch.float64), dec.eps), new
+
+
 def decode_token(x_emb: torch.Tensor, cache, get_layer, g_final, dec):
     """One decode step of one sequence: the new token's input embedding x_emb [d] at position
     P = len(cache rows), attending to the cached rows and itself.  Returns its final hidden

@@ -629,3 +629,26 @@ def test_token_stats_match_numpy():
     r64 = r.astype(np.float64)
     assert mx == float(r64.max()) and mean == pytest.approx(float(r64.mean()), abs=1e-15)
     assert std == pytest.approx(float(r64.std()), abs=1e-14)
+
+
+def test_suffix_over_a_shared_prefix_equals_the_whole_prefill():
+    # The prefix (system prompt) prefilled once and each sequence's suffix extended from its
+    # cache give the whole sequence's prefill: same suffix hidden states and cache rows.
+    dec = W.TINY_DECODER
+    layers, gf = _tiny_layers(dec)
+    g = torch.Generator().manual_seed(34)
+    prefix = torch.randn(8, dec.d, generator=g, dtype=torch.float64)
+    pre_h, pre_cache = O.prefill_with_cache(prefix, lambda l: layers[l], gf, dec)
+    for n in (1, 5, 13):
+        suffix = torch.randn(n, dec.d, generator=g, dtype=torch.float64)
+        full, full_cache = O.prefill_with_cache(torch.cat([prefix, suffix]), lambda l: layers[l], gf, dec)
+        h, new = O.extend_with_cache(suffix, pre_cache, lambda l: layers[l], gf, dec)
+        assert torch.allclose(full[:8], pre_h, rtol=0, atol=1e-12)
+        assert torch.allclose(full[8:], h, rtol=0, atol=1e-12)
+        for (k, v), (fk, fv) in zip(new, full_cache):
+            assert torch.allclose(k, fk[8:], rtol=0, atol=1e-12) and torch.allclose(v, fv[8:], rtol=0, atol=1e-12)
+    # the one-row case is the decode step
+    x = torch.randn(dec.d, generator=g, dtype=torch.float64)
+    h1, _ = O.extend_with_cache(x[None], pre_cache, lambda l: layers[l], gf, dec)
+    h2, _ = O.decode_token(x, pre_cache, lambda l: layers[l], gf, dec)
+    assert torch.equal(h1[0], h2)
