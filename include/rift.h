@@ -290,6 +290,28 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 const int* positions, void* kv_out, float* last_logits,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
 
+/* ---- Prefill over a shared system prompt (SURVEY-style extension of Section 2.1's prefill:
+ * the S system-prompt rows open every per-tile sequence at positions 0..S-1, so their hidden
+ * states and cache are the same in every sequence) ----
+ * The prompt is prefilled once and every sequence's remaining rows (its b_i vision tokens and
+ * the query; pack them with S = 0) are prefilled over the prompt's cache.  Results equal
+ * rift_prefill_layers on the full sequences (row for row, up to the fp32 summation order).
+ *   sys_ids     int32 [S] (device), embed bf16 [vocab, d]
+ *   prefix_hidden out bf16 [S, d]: the prompt's final hidden states
+ *   prefix_kv   out fp16 [n_layers][2][S][d]: the prompt's cache (the layout of kv_out)
+ *   hidden      bf16 [T, d] in/out: the suffix rows (packed with S = 0), then their final hidden
+ *               states; cu_seqlens [n_seq + 1] and positions [T] (0-based) over them
+ *   max_len     an upper bound on S + every suffix length
+ *   last_logits out fp32 [n_seq, vocab] (nullable; needs m->lm_head): each sequence's last row
+ *   ws          rift_prefill_shared_prefix_workspace_bytes(m, T, n_seq, max_len, S) bytes */
+size_t rift_prefill_shared_prefix_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len,
+                                                  int S);
+rift_status rift_prefill_shared_prefix(const rift_model* m, const int* sys_ids, int S, const void* embed,
+                                       int vocab, void* prefix_hidden, void* prefix_kv, void* hidden,
+                                       int T, const int* cu_seqlens, int n_seq, int max_len,
+                                       const int* positions, float* last_logits, void* ws,
+                                       size_t ws_bytes, rift_stream_t stream);
+
 /* ---- Decode step after the prefill (Section 2.1: decoding extends the prefilled KV cache one
  * token at a time) ----
  * One new token per sequence: sequence i's token token_ids[i] (an id into embed [vocab_embed, d]

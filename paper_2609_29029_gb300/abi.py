@@ -63,6 +63,9 @@ SIGNATURES = {
                                    _vp]),
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
     "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "rift_prefill_shared_prefix_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i, _i]),
+    "rift_prefill_shared_prefix": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _vp, _vp, _vp, _i, _vp, _i, _i, _vp, _vp,
+                                        _vp, _sz, _vp]),
     "rift_decode_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i]),
     "rift_decode_step": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _sz,
                               _vp]),
@@ -235,6 +238,18 @@ def prefill_layers(model: Model, hidden, T, cu_seqlens, n_seq, max_len, position
                                    ptr(positions), ptr(kv_out), ptr(last_logits), ptr(ws), ws_bytes,
                                    stream_handle(stream)),
            "rift_prefill_layers")
+
+
+def prefill_shared_prefix_workspace_bytes(model: Model, max_T, max_seqs, max_len, S) -> int:
+    return lib.rift_prefill_shared_prefix_workspace_bytes(C.byref(model), max_T, max_seqs, max_len, S)
+
+
+def prefill_shared_prefix(model: Model, sys_ids, S, embed, vocab, prefix_hidden, prefix_kv, hidden, T, cu_seqlens,
+                          n_seq, max_len, positions, last_logits, ws, ws_bytes, stream=None):
+    _check(lib.rift_prefill_shared_prefix(C.byref(model), ptr(sys_ids), S, ptr(embed), vocab, ptr(prefix_hidden),
+                                          ptr(prefix_kv), ptr(hidden), T, ptr(cu_seqlens), n_seq, max_len,
+                                          ptr(positions), ptr(last_logits), ptr(ws), ws_bytes, stream_handle(stream)),
+           "rift_prefill_shared_prefix")
 
 
 def decode_workspace_bytes(model: Model, n_seq, max_len) -> int:

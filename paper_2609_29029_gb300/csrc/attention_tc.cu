@@ -21,6 +21,10 @@
 // double-buffered, so the softmax of block j overlaps S_{j+1} and PV_{j-1}.  S_{j+2} is issued
 // only once PV_j (the reader of P_j in the same columns) has completed.  Every mbarrier wait is
 // bounded; on timeout the kernel sets RIFT_EBIT_TIMEOUT and every role falls through.
+//
+// With a shared prefix (S_pre > 0: a system prompt prefilled once), every item first runs over
+// the prefix's key/value blocks, loaded from their own tensor maps and masked only past S_pre, and
+// then over its own sequence's blocks, causal as above.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -219,6 +223,7 @@ __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.
 template <int HD, int KB>
 __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+                   const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int S_pre,
                    const int* __restrict__ cu, const int2* __restrict__ sched, int n_entries, int H, float scale_log2,
                    uint16_t* __restrict__ out) {
   using CF = Cfg<HD, KB>;
@@ -275,6 +280,7 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
   const uint32_t tmem = *tmem_slot;
   const int n_items = n_entries * H;
   const int d = H * HD;
+  const int np = (S_pre + KB - 1) / KB;  // prefix blocks ahead of every sequence's own
 
   // An item's sequence start, length, first row, head and number of KB-key blocks (causal:
   // keys up to the block's last valid row).  Every role reads the next item's entry while it
@@ -291,7 +297,7 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
     it.seq0 = cu[e.x];
     it.L = cu[e.x + 1] - it.seq0;
     it.q0 = e.y;
-    it.nkv = (min(it.L, it.q0 + BQ) - 1) / KB + 1;
+    it.nkv = np + (min(it.L, it.q0 + BQ) - 1) / KB + 1;
     return it;
   };
   // Counters shared by every role: g counts KB-key blocks, t counts items of this CTA.  Block g
@@ -317,14 +323,18 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
         for (int j = 0; j < cur.nkv; ++j, ++g) {
           const int s = g % NST;
           const uint32_t ph = (g / NST) & 1u;
-          const int col = (lane == 0 ? d : 2 * d) + cur.h * HD;
           const int base = lane == 0 ? K_EMPTY : V_EMPTY;
           if (!mbar_wait(BAR(base, s), ph ^ 1u, abort_flag)) { ok = false; break; }
           const uint32_t full = BAR(lane == 0 ? K_FULL : V_FULL, s);
           mbar_expect_tx(full, CF::K_BYTES);
           uint8_t* dst = (lane == 0 ? sK + s * CF::K_BYTES : sV + s * CF::V_BYTES);
-          for (int c = 0; c < HD / 64; ++c)
-            tma_load_2d(smem_u32(dst + c * KB * 128), &tm_kv, col + c * 64, cur.seq0 + j * KB, full);
+          // prefix blocks from the prefix's [S_pre, d] K / V maps (rows past S_pre read as zero),
+          // then the sequence's own rows of the qkv map
+          const bool pre = j < np;
+          const CUtensorMap* map = pre ? (lane == 0 ? &tm_pk : &tm_pv) : &tm_kv;
+          const int col = (pre ? 0 : (lane == 0 ? d : 2 * d)) + cur.h * HD;
+          const int row = pre ? j * KB : cur.seq0 + (j - np) * KB;
+          for (int c = 0; c < HD / 64; ++c) tma_load_2d(smem_u32(dst + c * KB * 128), map, col + c * 64, row, full);
         }
         ++t;
       }
@@ -413,12 +423,14 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
 #pragma unroll
         for (int c = 0; c < NC; ++c) tmem_ld32(sbase + 32u * c, sv[c]);
         tmem_wait_ld();
-        const int k0 = j * KB;
-        // Only the diagonal blocks and the block holding the sequence end need the mask: key
-        // valid iff key <= qrow and key < L (this branch is uniform over the CTA).  Within it a
-        // 32-key chunk is touched only where some row of the warp ends inside or before it.
-        if (k0 + KB - 1 > q0 || k0 + KB > L) {
-          const int lim = min(qrow, L - 1) - k0;  // last valid column of this row
+        // Own blocks: only the diagonal blocks and the block holding the sequence end need the
+        // mask, key valid iff key <= qrow and key < L (uniform over the CTA).  Prefix blocks: key
+        // valid iff key < S_pre.  Within a masked block a 32-key chunk is touched only where some
+        // row of the warp ends inside or before it.
+        const bool pre = j < np;
+        const int k0 = pre ? j * KB : (j - np) * KB;
+        if (pre ? k0 + KB > S_pre : (k0 + KB - 1 > q0 || k0 + KB > L)) {
+          const int lim = pre ? S_pre - 1 - k0 : min(qrow, L - 1) - k0;  // last valid column of this row
 #pragma unroll
           for (int c = 0; c < NC; ++c)
             if (__any_sync(0xffffffffu, lim < 32 * c + 31)) {
@@ -582,8 +594,9 @@ namespace {
 constexpr int kAttnKB = 64;
 
 template <int HD, int KB>
-int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const int* cu_seqlens, const int2* sched,
-                 int n_sched_max, int n_heads, float scale_log2, void* out, cudaStream_t st) {
+int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& mpk, const CUtensorMap& mpv,
+                 int S_pre, const int* cu_seqlens, const int2* sched, int n_sched_max, int n_heads, float scale_log2,
+                 void* out, cudaStream_t st) {
   using namespace fa;
   using CF = Cfg<HD, KB>;
   static bool attr = false;
@@ -596,40 +609,52 @@ int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const int* cu_se
   const int items = n_sched_max * n_heads;
   const int slots = CF::CTAS * sm_count();
   const int grid = items < slots ? items : slots;
-  attn_tc_kernel<HD, KB><<<grid, THREADS, CF::SMEM, st>>>(mq, mkv, cu_seqlens, sched, n_sched_max, n_heads, scale_log2,
-                                                          static_cast<uint16_t*>(out));
+  attn_tc_kernel<HD, KB><<<grid, THREADS, CF::SMEM, st>>>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max,
+                                                          n_heads, scale_log2, static_cast<uint16_t*>(out));
   return 0;
+}
+
+// fp16 [rows, cols] (row-major) as a 2-D tensor map of 64-column x box_rows boxes, 128B swizzle.
+bool make_attn_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows) {
+  auto fn = fa::encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
 
-// qkv fp16 [T, 3 H hd] (q | k | v, heads contiguous), out fp16 [T, H hd].
+// qkv fp16 [T, 3 H hd] (q | k | v, heads contiguous), out fp16 [T, H hd]; optional prefix keys and
+// values fp16 [S_pre, H hd] attended to by every sequence before its own rows.
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
-                     const int2* sched, int n_sched_max, void* out, cudaStream_t st) {
+                     const int2* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k,
+                     const void* prefix_v, int S_pre) {
   using namespace fa;
   (void)n_seq;
   if (T <= 0) return 0;
   if (head_dim != 64 && head_dim != 128) return 1;
-  auto fn = encode_fn();
-  if (!fn) return 1;
+  if (S_pre > 0 && (!prefix_k || !prefix_v)) return 1;
   const int d = n_heads * head_dim;
   // Q tiles of 128 rows and K/V tiles of kAttnKB rows, each a 64-column (128-byte) box
-  CUtensorMap maps[2];
-  const cuuint32_t rows[2] = {(cuuint32_t)BQ, (cuuint32_t)kAttnKB};
-  for (int i = 0; i < 2; ++i) {
-    cuuint64_t dims[2] = {(cuuint64_t)(3 * d), (cuuint64_t)T};
-    cuuint64_t strides[1] = {(cuuint64_t)(3 * d) * 2};
-    cuuint32_t box[2] = {64, rows[i]};
-    cuuint32_t estr[2] = {1, 1};
-    if (fn(&maps[i], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(qkv), dims, strides, box, estr,
-           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return 1;
+  CUtensorMap mq, mkv, mpk, mpv;
+  if (!make_attn_map(&mq, qkv, 3 * d, T, BQ) || !make_attn_map(&mkv, qkv, 3 * d, T, kAttnKB)) return 1;
+  if (S_pre > 0) {
+    if (!make_attn_map(&mpk, prefix_k, d, S_pre, kAttnKB) || !make_attn_map(&mpv, prefix_v, d, S_pre, kAttnKB)) return 1;
+  } else {
+    mpk = mkv;  // unused without a prefix
+    mpv = mkv;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
   if (head_dim == 128)
-    return launch_shape<128, kAttnKB>(maps[0], maps[1], cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out, st);
-  return launch_shape<64, kAttnKB>(maps[0], maps[1], cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out, st);
+    return launch_shape<128, kAttnKB>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max, n_heads, scale_log2,
+                                      out, st);
+  return launch_shape<64, kAttnKB>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out,
+                                   st);
 }
 
 }  // namespace rift

@@ -368,7 +368,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * ACC_COLS);
       if constexpr (EPI == EPI_QKV_ROPE) {
         const int half = ep.head_dim >> 1;
-        const int pos = (row < M) ? ep.positions[row] : 0;
+        const int pos = (row < M) ? ep.positions[row] + ep.pos_offset : 0;
         const bool pos_ok = pos >= 0 && pos < ep.max_len;
         if (row < M && !pos_ok) atomicOr(&g_err_gemm, RIFT_EBIT_BADID);
 #pragma unroll 1
@@ -520,7 +520,7 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits,
       float4 y = acc4(row, col);
       if (col < ep.rope_cols) {
         const int half = ep.head_dim >> 1, j = col % ep.head_dim;
-        const int pos = ep.positions[row];
+        const int pos = ep.positions[row] + ep.pos_offset;
         if (pos < 0 || pos >= ep.max_len) {
           if (j == 0) atomicOr(&g_err_gemm, RIFT_EBIT_BADID);
           continue;  // as the fused epilogue: q and k of a row without a valid position stay unwritten

@@ -172,7 +172,7 @@ static void norm_launch(int kind, int T, const void* in, float* h32, const void*
 
 int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
                    int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
-                   cudaStream_t st) {
+                   cudaStream_t st, const void* prefix_kv, int S_pre) {
   if (T == 0) return 0;
   const PrefillLayout L = prefill_layout(m, T, n_seq, max_len);
   float* h32 = reinterpret_cast<float*>(ws + L.h32_off);
@@ -196,6 +196,7 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   rope_ep.rope_cols = 2 * d;
   rope_ep.head_dim = m.head_dim;
   rope_ep.max_len = max_len;
+  rope_ep.pos_offset = S_pre;
   for (int l = 0; l < m.n_layers; ++l) {
     if (l == 0)
       norm_launch(0, T, hidden, h32, m.g_attn[0], xn, d, m.eps, st);
@@ -207,7 +208,10 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
       kv_store(qkv, T, d, kl, kl + (size_t)T * d, st);
     }
     prof_begin(RIFT_PROF_ATTN, st);
-    if (launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st)) return 1;
+    const uint16_t* pk = prefix_kv ? static_cast<const uint16_t*>(prefix_kv) + (size_t)l * 2 * S_pre * d : nullptr;
+    if (launch_attention(qkv, T, cu_seqlens, n_seq, m.n_heads, m.head_dim, sched, L.max_qblocks, att, st, pk,
+                         pk ? pk + (size_t)S_pre * d : nullptr, prefix_kv ? S_pre : 0))
+      return 1;
     prof_end(RIFT_PROF_ATTN, st, 1);
     if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st)) return 1;
     norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
@@ -222,6 +226,62 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
     norm_launch(1, n_seq, last32, nullptr, m.g_final, last16, d, m.eps, st);
     if (launch_gemm(last16, m.lm_head, n_seq, m.vocab, d, EPI_STORE_F32, last_logits, st)) return 1;
   }
+  return 0;
+}
+
+// ------------------------------------------------------------------------------------------
+// Shared-prefix prefill: the system prompt once, then every sequence's suffix over its cache
+// ------------------------------------------------------------------------------------------
+
+// prefix rows = embed[sys_ids] (bf16), cu = {0, S}, positions 0 .. S-1; a bad id sets
+// RIFT_EBIT_BADID and gives a zero row.
+__global__ void prefix_rows_kernel(const int* __restrict__ sys_ids, int S, const uint16_t* __restrict__ embed,
+                                   int vocab, int d, uint16_t* __restrict__ rows, int* __restrict__ cu,
+                                   int* __restrict__ pos) {
+  const int r = blockIdx.x;
+  const int id = sys_ids[r];
+  const bool ok = id >= 0 && id < vocab;
+  if (threadIdx.x == 0) {
+    pos[r] = r;
+    if (!ok) atomicOr(&g_err_prefill, RIFT_EBIT_BADID);
+    if (r == 0) {
+      cu[0] = 0;
+      cu[1] = S;
+    }
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(embed + (size_t)(ok ? id : 0) * d);
+  uint4* dst = reinterpret_cast<uint4*>(rows + (size_t)r * d);
+  for (int c = threadIdx.x; c < d / 8; c += blockDim.x) dst[c] = ok ? src[c] : make_uint4(0, 0, 0, 0);
+}
+
+SharedPrefixLayout shared_prefix_layout(const rift_model& m, int max_T, int max_seqs, int max_len, int S) {
+  SharedPrefixLayout L{};
+  const PrefillLayout P = prefill_layout(m, max_T > S ? max_T : S, max_seqs > 1 ? max_seqs : 1, max_len);
+  size_t off = (P.total + 255) & ~size_t(255);
+  L.prefill_bytes = P.total;
+  L.cu_off = off;
+  off += 256;
+  L.pos_off = off;
+  off += ((size_t)S * sizeof(int) + 255) & ~size_t(255);
+  L.total = off;
+  return L;
+}
+
+int launch_prefill_shared_prefix(const rift_model& m, const int* sys_ids, int S, const void* embed, int vocab,
+                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
+                                 int n_seq, int max_len, const int* positions, float* last_logits, char* ws,
+                                 cudaStream_t st) {
+  const SharedPrefixLayout L = shared_prefix_layout(m, T, n_seq, max_len, S);
+  int* cu_pre = reinterpret_cast<int*>(ws + L.cu_off);
+  int* pos_pre = reinterpret_cast<int*>(ws + L.pos_off);
+  prefix_rows_kernel<<<S, 128, 0, st>>>(sys_ids, S, static_cast<const uint16_t*>(embed), vocab, m.d,
+                                        static_cast<uint16_t*>(prefix_hidden), cu_pre, pos_pre);
+  // the prefix as one sequence, keeping its cache; then the suffixes over it (the two share the
+  // prefill workspace: they run in order on the stream)
+  if (launch_prefill(m, prefix_hidden, S, cu_pre, 1, max_len, pos_pre, prefix_kv, nullptr, ws, st)) return 1;
+  if (T > 0 && launch_prefill(m, hidden, T, cu_seqlens, n_seq, max_len, positions, nullptr, last_logits, ws, st,
+                              prefix_kv, S))
+    return 1;
   return 0;
 }
 

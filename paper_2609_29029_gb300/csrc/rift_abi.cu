@@ -311,6 +311,32 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const 
   return RIFT_OK;
 }
 
+size_t rift_prefill_shared_prefix_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len, int S) {
+  if (!model_ok(m) || max_T < 0 || max_seqs < 0 || max_len < 1 || S < 1 || S > max_len) return 0;
+  return shared_prefix_layout(*m, max_T, max_seqs, max_len, S).total;
+}
+
+rift_status rift_prefill_shared_prefix(const rift_model* m, const int* sys_ids, int S, const void* embed, int vocab,
+                                       void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
+                                       int n_seq, int max_len, const int* positions, float* last_logits, void* ws,
+                                       size_t ws_bytes, rift_stream_t stream) {
+  if (!model_ok(m) || !sys_ids || !embed || !prefix_hidden || !prefix_kv || S < 1 || vocab < 1 || T < 0 ||
+      n_seq < 0 || max_len < 1 || S > max_len)
+    return RIFT_ERR_INVALID;
+  if (T > 0 && (!hidden || !cu_seqlens || !positions || n_seq < 1)) return RIFT_ERR_INVALID;
+  if (!aligned16(embed) || !aligned16(prefix_hidden) || !aligned16(prefix_kv) || (hidden && !aligned16(hidden)) ||
+      (last_logits && !aligned16(last_logits)))
+    return RIFT_ERR_INVALID;
+  if (last_logits && !lm_head_ok(m)) return RIFT_ERR_INVALID;
+  if (!ws_ok(ws, ws_bytes, shared_prefix_layout(*m, T, n_seq, max_len, S).total)) return RIFT_ERR_INVALID;
+  if (launch_prefill_shared_prefix(*m, sys_ids, S, embed, vocab, prefix_hidden, prefix_kv, hidden, T, cu_seqlens,
+                                   n_seq, max_len, positions, last_logits, static_cast<char*>(ws),
+                                   static_cast<cudaStream_t>(stream)))
+    return RIFT_ERR_INVALID;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
 size_t rift_decode_workspace_bytes(const rift_model* m, int n_seq, int max_len) {
   if (!model_ok(m) || n_seq < 0 || max_len < 1 || max_len > 32768) return 0;
   return decode_layout(*m, n_seq, max_len).total;

@@ -70,9 +70,19 @@ struct PrefillLayout {
   int max_qblocks;
 };
 PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len);
+// prefix_kv (optional): fp16 [n_layers][2][S_pre][d] cache of a prefix shared by every sequence
+// (each sequence's rows attend to it first; their positions are positions[] + S_pre).
 int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
                    int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
-                   cudaStream_t st);
+                   cudaStream_t st, const void* prefix_kv = nullptr, int S_pre = 0);
+struct SharedPrefixLayout {
+  size_t prefill_bytes, cu_off, pos_off, total;
+};
+SharedPrefixLayout shared_prefix_layout(const rift_model& m, int max_T, int max_seqs, int max_len, int S);
+int launch_prefill_shared_prefix(const rift_model& m, const int* sys_ids, int S, const void* embed, int vocab,
+                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
+                                 int n_seq, int max_len, const int* positions, float* last_logits, char* ws,
+                                 cudaStream_t st);
 struct DecodeLayout {
   size_t h32_off, x0_off, xn_off, qkv_off, attn_off, act_off, rope_off, pos_off, dpart_off, split_off, split_bytes,
       total;
@@ -96,6 +106,7 @@ struct EpiParams {
   int rope_cols = 0;               // q and k columns: 2 d
   int head_dim = 0;
   int max_len = 0;
+  int pos_offset = 0;              // added to positions[row] (rows that follow a shared prefix)
   float out_scale = 1.f;           // EPI_STORE_F32
   // EPI_RESID_F32 with split scratch: also norm_out fp16 [M, N] = RMSNorm(C) norm_gain (bf16 [N])
   const void* norm_gain = nullptr;
@@ -114,8 +125,11 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].
 int attention_max_qblocks(int max_T, int max_seqs);
 void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st);
+// prefix_k, prefix_v (optional): fp16 [S_pre, d] keys (after RoPE) and values of a prefix that every
+// sequence attends to before its own rows.
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
-                     const int2* sched, int n_sched_max, void* out, cudaStream_t st);
+                     const int2* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k = nullptr,
+                     const void* prefix_v = nullptr, int S_pre = 0);
 unsigned int read_clear_err_attn();
 
 }  // namespace rift

@@ -161,13 +161,35 @@ class ScenePipeline:
                              self.sel_off, self.ctx, self.max_ctx, self.ctx_off, self.ctx_target, self.ws_merge,
                              self.ws_merge_bytes, stream)
 
-    def pack(self, X, embed, sys_ids, query_ids, stream=None):
-        """a8: the packed batch, cu_seqlens and positions."""
+    def pack(self, X, embed, sys_ids, query_ids, stream=None, with_system=True):
+        """a8: the packed batch, cu_seqlens and positions (without the system rows: the suffixes
+        for a shared-prefix prefill)."""
         if self.max_m:
             self.merge(X, stream)
+        S = self.S if with_system else 0
         abi.pack_ragged(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.sel, self.sel_off,
-                        sys_ids, self.S, query_ids, self.Q, embed, embed.shape[0], self.packed, self.max_T,
+                        sys_ids if S else None, S, query_ids, self.Q, embed, embed.shape[0], self.packed, self.max_T,
                         self.cu, self.positions, self.T, stream, ctx=self.ctx, ctx_off=self.ctx_off)
+
+    def run_shared_prefix(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, stream=None):
+        """The query with the system prompt prefilled once: packed suffixes (vision tokens + query)
+        prefilled over its cache.  Returns (n_kept, suffix rows); self.packed holds the suffixes'
+        final hidden states, self.prefix_hidden the prompt's."""
+        self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)
+        self.pack(X, embed, sys_ids, query_ids, stream, with_system=False)
+        n_kept, T = self.read_counts(stream)
+        m, S = self.model, self.S
+        if not hasattr(self, "prefix_hidden"):
+            self.prefix_hidden = torch.empty(S, self.d, dtype=torch.bfloat16, device=self.device)
+            self.prefix_kv = torch.empty(m.dec.n_layers, 2, S, self.d, dtype=torch.float16, device=self.device)
+        need = abi.prefill_shared_prefix_workspace_bytes(m.struct, T, n_kept, self.max_len, S)
+        if need > self.ws_prefill_bytes:
+            self.ws_prefill = torch.empty(need, dtype=torch.uint8, device=self.device)
+            self.ws_prefill_bytes = need
+        abi.prefill_shared_prefix(m.struct, sys_ids, S, embed, embed.shape[0], self.prefix_hidden, self.prefix_kv,
+                                  self.packed, T, self.cu, n_kept, self.max_len, self.positions, None,
+                                  self.ws_prefill, self.ws_prefill_bytes, stream)
+        return n_kept, T
 
     def read_counts(self, stream=None):
         """Sync, check device error flags and read (n_kept, T) back to the host."""
