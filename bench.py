@@ -41,6 +41,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-step measurement")
+    ap.add_argument("--no-shared-prefix", action="store_true", help="skip the shared-prefix measurement")
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
@@ -335,6 +336,27 @@ def sweep(steps: int, warmup: int):
         torch.cuda.empty_cache()
 
 
+def shared_prefix_measure(pipe, sc, q, bg, sy, T, stream, steps):
+    """The same scene query with the system prompt prefilled once and every sequence's suffix over
+    its cache (rift_prefill_shared_prefix): same final hidden states, fewer rows prefilled.  Kept
+    apart from the metric, whose token count it changes."""
+    def one():
+        return pipe.run_shared_prefix(sc.X, sc.embed, q, bg, sy, q, stream=stream)
+    for _ in range(2):
+        n_kept, T2 = one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        n_kept, T2 = one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    return {"ms_per_query": ms, "rows_prefilled": T2 + pipe.S, "rows_of_the_sequences": T,
+            "retained_tokens_per_s_equivalent": T / (ms / 1e3), "note": "system prompt prefilled once; "
+            "the suffixes attend to its cache"}
+
+
 def decode_measure(pipe, dm, sc, dec, n_kept, T, stream, steps):
     """The first decode step after the prefill (Section 2.1), timed on its own: the prefill runs
     once more writing its KV cache, then `steps` decode steps of one seeded token per retained
@@ -565,6 +587,7 @@ def main():
     h2d_bytes = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
     d2h = Te * s.d * 2 + 8
     decode = None if args.no_decode else decode_measure(pipe, dm, sc, dec, n_kept, T, stream, args.steps)
+    shared = None if args.no_shared_prefix else shared_prefix_measure(pipe, sc, q, bg, sy, T, stream, args.steps)
 
     if rank != 0:
         return
@@ -606,6 +629,7 @@ def main():
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h},
         "decode_step": decode,
+        "shared_prefix": shared,
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
