@@ -41,16 +41,10 @@ namespace tc {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
-constexpr int B_BYTES = BN * BK * 2;  // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int THREADS = 192;
-constexpr int ACC_COLS = BN;        // fp32 accumulator columns per buffer
-constexpr int TMEM_COLS = 2 * ACC_COLS;
-constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
-
-// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A fp16 (bits 7-9 = 0), B fp16
-// (bits 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+// Instruction descriptor (per kernel instance), kind::f16: D fp32 (bits 4-5 = 1), A fp16 (bits
+// 7-9 = 0), B fp16 (bits 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22, M >> 4
+// at bits 24-28.
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -114,11 +108,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accum) {
+__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accum) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accum));
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum));
 }
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
@@ -244,10 +239,16 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
   }
 }
 
-template <int EPI>
+// BN_ x STAGES_: 256 x 4 for the prefill; 128 x 6 for few-row products with the operands swapped
+// (weights as the 128-row operand, the few activation rows as the N side; EPI_STORE_F32_T).
+template <int EPI, int BN_, int STAGES_>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
                    int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride) {
+  constexpr int BN = BN_, STAGES = STAGES_;  // this instance's tile width and ring depth
+  constexpr int B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr int ACC_COLS = BN, TMEM_COLS = 2 * ACC_COLS;
+  constexpr uint32_t IDESC_T = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -345,7 +346,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t bd = smem_desc(smem_u32(sB + s * B_BYTES));
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along K per step (encoded >> 4)
-            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (k != k0 || kk != 0) ? 1u : 0u);
+            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, IDESC_T, (k != k0 || kk != 0) ? 1u : 0u);
           umma_commit(empty_bar(s));
         }
         if (ok) umma_commit(tfull_bar(b));
@@ -392,7 +393,17 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld32(taddr + c, r);
-          if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, Cu, ep.out_scale);
+          if constexpr (EPI == EPI_STORE_F32_T) {  // C[col][row] (transposed), col < N, row < M
+            const int col = n_blk * BN + c;
+            if (row < M) {
+              float* out = static_cast<float*>(Cu) + row;
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                if (col + e < N) out[(size_t)(col + e) * M] = __uint_as_float(r[e]);
+            }
+          } else {
+            if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, Cu, ep.out_scale);
+          }
         }
       }
       fence_before();
@@ -448,21 +459,22 @@ static int sm_count() {
   return n;
 }
 
-template <int EPI>
+template <int EPI, int BN_ = BN, int STAGES_ = STAGES>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
                   cudaStream_t st, int splits = 1) {
+  constexpr size_t smem = (size_t)STAGES_ * (A_BYTES + BN_ * BK * 2) + 1024 + 256;
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM);
+    cudaFuncSetAttribute(gemm_tc_kernel<EPI, BN_, STAGES_>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     attr = true;
   }
-  const int units = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * splits;
+  const int units = ((M + BM - 1) / BM) * ((N + BN_ - 1) / BN_) * splits;
   const int grid = units < sm_count() ? units : sm_count();
   // Band height: as many M-tiles as keep the band's A rows within ~48 MB of L2 (8..64), so each
   // weight tile is streamed from DRAM once per band.
   int group_m = (int)((48u << 20) / ((size_t)BM * K * 2));
   group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM, st>>>(a, b, M, N, K, C, ep, group_m, splits, (size_t)M * N);
+  gemm_tc_kernel<EPI, BN_, STAGES_><<<grid, THREADS, smem, st>>>(a, b, M, N, K, C, ep, group_m, splits, (size_t)M * N);
   return 0;
 }
 
@@ -584,23 +596,48 @@ __global__ void __launch_bounds__(256) splitk_resid_norm_kernel(const float* __r
 // Split count for an M x N x K product whose tiles leave SMs idle: the K-slice count (1..16, at
 // least 4 K-blocks a slice, partials within the workspace) that minimises the makespan, i.e. the
 // rounds of units over the SMs times the K-blocks of a slice.  1 = no split.
-static int choose_splits(int M, int N, int K, size_t ws_bytes) {
+// With `unit_cost` > 0 (the swapped few-row path, whose units always store partials) every slice
+// count is weighed, each unit costing its K-blocks plus unit_cost K-blocks' worth of traffic and
+// overhead; otherwise only products whose tiles leave SMs idle are split.
+static int choose_splits(int M, int N, int K, size_t ws_bytes, int bn = BN, double unit_cost = 0.0) {
   const int sms = sm_count();
-  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN), kt = (K + BK - 1) / BK;
-  if (tiles >= sms) return 1;
+  const int tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn), kt = (K + BK - 1) / BK;
+  if (tiles >= sms && unit_cost == 0.0) return 1;
   int best = 1;
-  long best_cost = (long)((tiles + sms - 1) / sms) * kt;
+  double best_cost = (double)((tiles + sms - 1) / sms) * (kt + unit_cost);
   for (int s = 2; s <= 16 && kt / s >= 4; ++s) {
     if ((size_t)s * M * N * sizeof(float) > ws_bytes) break;
     const int per = (kt + s - 1) / s;
     const int se = (kt + per - 1) / per;  // every slice non-empty
-    const long cost = (long)((tiles * se + sms - 1) / sms) * per;
+    const double cost = (double)((tiles * se + sms - 1) / sms) * (per + unit_cost);
     if (cost < best_cost) {
       best_cost = cost;
       best = se;
     }
   }
   return best;
+}
+
+// The slices' partial products [splits][M][N] summed in slice order with the epilogue epi (a
+// residual product with ep.norm_out also applies the following RMSNorm).
+static int reduce_slices(const float* part, int splits, int M, int N, int epi, void* C, const EpiParams& ep,
+                         cudaStream_t st) {
+  if (epi == EPI_RESID_F32 && ep.norm_out) {
+    splitk_resid_norm_kernel<<<M, 256, 0, st>>>(part, splits, M, N, static_cast<float*>(C),
+                                                 static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out);
+    return 0;
+  }
+  const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N) / 4;
+  const int grid = (int)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048);
+  switch (epi) {
+    case EPI_STORE_BF16: splitk_reduce_kernel<EPI_STORE_BF16><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    case EPI_RESID_F32: splitk_reduce_kernel<EPI_RESID_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    case EPI_SWIGLU: splitk_reduce_kernel<EPI_SWIGLU><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    case EPI_QKV_ROPE: splitk_reduce_kernel<EPI_QKV_ROPE><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    case EPI_STORE_F32: splitk_reduce_kernel<EPI_STORE_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    default: return 1;
+  }
+  return 0;
 }
 
 }  // namespace tc
@@ -614,6 +651,19 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
   if (epi == EPI_QKV_ROPE && (N % 64 != 0 || (ep.head_dim != 64 && ep.head_dim != 128) || !ep.positions || !ep.rope))
     return 1;
+  // Few rows (<= 128, with scratch: the decode step): the operands swapped so that the weights
+  // stream as the 128-row operand in 128-row tiles and the rows sit on the N side (128 wide); the
+  // slices' fp32 partials are stored transposed ([M, N] as the reductions below read them).
+  if (split_ws && M <= 128 && (size_t)M * N * sizeof(float) <= split_ws_bytes) {
+    constexpr int SW_BN = 128, SW_STAGES = 6;
+    CUtensorMap mw, mx;
+    if (!make_map(&mw, B, (uint64_t)K, (uint64_t)N, BM) || !make_map(&mx, A, (uint64_t)K, (uint64_t)M, SW_BN)) return 1;
+    // a unit's partials (M x 128 fp32, written and read back) cost M / 16 K-blocks of weight
+    // traffic; its fill and drain about 1.5 more
+    const int splits = choose_splits(N, M, K, split_ws_bytes, SW_BN, M / 16.0 + 1.5);
+    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits)) return 1;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st);
+  }
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
   // The residual product with a following RMSNorm (ep.norm_out) always goes through the
@@ -623,23 +673,7 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
   if (splits > 1 || fuse_norm) {
     if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits)) return 1;
-    const float* part = static_cast<const float*>(split_ws);
-    if (fuse_norm) {
-      splitk_resid_norm_kernel<<<M, 256, 0, st>>>(part, splits, M, N, static_cast<float*>(C),
-                                                   static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out);
-      return 0;
-    }
-    const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N) / 4;
-    const int grid = (int)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048);
-    switch (epi) {
-      case EPI_STORE_BF16: splitk_reduce_kernel<EPI_STORE_BF16><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-      case EPI_RESID_F32: splitk_reduce_kernel<EPI_RESID_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-      case EPI_SWIGLU: splitk_reduce_kernel<EPI_SWIGLU><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-      case EPI_QKV_ROPE: splitk_reduce_kernel<EPI_QKV_ROPE><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-      case EPI_STORE_F32: splitk_reduce_kernel<EPI_STORE_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-      default: return 1;
-    }
-    return 0;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st);
   }
   switch (epi) {
     case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, ep, st);

@@ -98,7 +98,8 @@ enum GemmEpilogue {
   EPI_RESID_F32 = 1,   // R fp32 [M, N] += acc
   EPI_SWIGLU = 2,      // N = 2F interleaved in 16-column groups; C fp16 [M, F] = silu(g) * u
   EPI_QKV_ROPE = 3,    // C fp16 [M, N]; columns < rope_cols get rotate-half RoPE at positions[row]
-  EPI_STORE_F32 = 4    // C fp32 [M, N] = acc * out_scale
+  EPI_STORE_F32 = 4,   // C fp32 [M, N] = acc * out_scale
+  EPI_STORE_F32_T = 5  // C fp32 [N, M] = acc (transposed; the swapped few-row products)
 };
 struct EpiParams {
   const int* positions = nullptr;  // [M] position of each row (EPI_QKV_ROPE)
