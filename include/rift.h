@@ -366,6 +366,13 @@ rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens,
 #define RIFT_PROF_SELECT 5    /* prune, budgets, top-b */
 #define RIFT_PROF_PACK 6      /* ragged packing */
 #define RIFT_PROF_CLASSES 7
+/* ---- Diagnostics ----
+ * Enqueues a kernel whose pipeline wait can never complete (an mbarrier no one arrives at),
+ * through the same bounded wait as the library's kernels: after ~4 s it gives up, and the next
+ * rift_sync_status returns RIFT_ERR_TIMEOUT with the context still usable.  A check of the
+ * failure path, not of any result. */
+rift_status rift_check_wait_timeout(rift_stream_t stream);
+
 /* rift_profile_enable(1) starts recording a pair of CUDA events on the launch stream around
  * every kernel launch of the classes above (0 stops).  rift_profile_read waits for the recorded
  * events, writes per-class totals (ms[c] in milliseconds, launches[c]) for n_classes classes and

@@ -73,6 +73,7 @@ SIGNATURES = {
     "rift_linear": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
     "rift_attention_workspace_bytes": (_sz, [_i, _i]),
     "rift_attention_varlen": (_i, [_vp, _i, _vp, _i, _i, _i, _vp, _vp, _sz, _vp]),
+    "rift_check_wait_timeout": (_i, [_vp]),
     "rift_profile_enable": (None, [_i]),
     "rift_profile_read": (_i, [C.POINTER(C.c_double), C.POINTER(C.c_longlong), _i]),
     "rift_launch_count": (C.c_longlong, []),
@@ -262,6 +263,10 @@ def decode_step(model: Model, kv_cache, T, cu_seqlens, n_seq, max_len, token_ids
                                 ptr(embed), vocab_embed, ptr(hidden_out), ptr(kv_new), ptr(logits), ptr(ws), ws_bytes,
                                 stream_handle(stream)),
            "rift_decode_step")
+
+
+def check_wait_timeout(stream=None):
+    _check(lib.rift_check_wait_timeout(stream_handle(stream)), "rift_check_wait_timeout")
 
 
 def profile_enable(on: bool):

@@ -618,6 +618,19 @@ static int choose_splits(int M, int N, int K, size_t ws_bytes, int bn = BN, doub
   return best;
 }
 
+// A wait that can never complete (an mbarrier nobody arrives at), through the same bounded
+// mbar_wait as the GEMM's pipeline: it gives up after ~4 s of globaltimer, sets
+// RIFT_EBIT_TIMEOUT and returns, leaving the context usable.
+__global__ void wait_timeout_check_kernel() {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  mbar_init(smem_u32(&bar), 1);
+  asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  mbar_wait(smem_u32(&bar), 0, reinterpret_cast<volatile int*>(&abort_flag));
+}
+
 // The slices' partial products [splits][M][N] summed in slice order with the epilogue epi (a
 // residual product with ep.norm_out also applies the following RMSNorm).
 static int reduce_slices(const float* part, int splits, int M, int N, int epi, void* C, const EpiParams& ep,
@@ -641,6 +654,11 @@ static int reduce_slices(const float* part, int splits, int M, int N, int epi, v
 }
 
 }  // namespace tc
+
+int launch_wait_timeout_check(cudaStream_t st) {
+  tc::wait_timeout_check_kernel<<<1, 32, 0, st>>>();
+  return 0;
+}
 
 // Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
 // the RoPE epilogue), A, B and C 16-byte aligned.

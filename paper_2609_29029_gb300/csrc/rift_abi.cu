@@ -284,6 +284,12 @@ static bool model_ok(const rift_model* m) {
   return aligned16(m->g_final);
 }
 
+rift_status rift_check_wait_timeout(rift_stream_t stream) {
+  launch_wait_timeout_check(static_cast<cudaStream_t>(stream));
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
 size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len) {
   if (!model_ok(m) || max_T < 0 || max_seqs < 0 || max_len < 1) return 0;
   return prefill_layout(*m, max_T, max_seqs, max_len).total;

@@ -121,6 +121,7 @@ int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void
                 size_t split_ws_bytes = 0);
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
                    cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0);
+int launch_wait_timeout_check(cudaStream_t st);
 
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].

@@ -63,3 +63,21 @@ def test_weights_reproducible_and_shaped():
         assert a[k].shape == s and a[k].dtype == torch.bfloat16 and torch.equal(a[k], b[k])
     assert abs(float(a["wq"].float().std()) - 0.02) < 0.002
     assert not torch.equal(a["wq"], W.make_layer(dec, 0)["wq"])
+
+
+def test_weights_file_round_trip(tmp_path):
+    from paper_2609_29029_gb300.weights import load_weights, save_weights
+    from synth import workloads as W
+    dec = W.TINY_DECODER
+    layers = [W.make_layer(dec, l) for l in range(dec.n_layers)]
+    gf, lm = W.make_final_norm(dec), W.make_lm_head(dec)
+    dims = {"n_layers": dec.n_layers, "d": dec.d, "n_heads": dec.n_heads, "head_dim": dec.head_dim, "ffn": dec.ffn,
+            "vocab": dec.vocab}
+    path = tmp_path / "tiny.rift"
+    save_weights(path, dims, layers, gf, lm)
+    dims2, layers2, gf2, lm2 = load_weights(path)
+    assert dims2 == dims
+    assert all(torch.equal(a[k], b[k]) for a, b in zip(layers, layers2) for k in a)
+    assert torch.equal(gf, gf2) and torch.equal(lm, lm2)
+    save_weights(path, dims, layers, gf)
+    assert load_weights(path)[3] is None
