@@ -83,13 +83,27 @@ __device__ __forceinline__ uint64_t globaltimer() {
   return t;
 }
 
-// Bounded wait for the phase of parity `parity`.  Returns false if the kernel is aborting or
-// the wait ran out (which starts the abort).
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.b32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase of parity `parity` (CL: acquire at cluster scope, for a barrier the
+// other CTA of the pair arrives on).  Returns false if the kernel is aborting or the wait ran out
+// (which starts the abort).
+template <bool CL = false>
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
+  auto tw = [&]() { return CL ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
+  if (tw()) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 0; i < RIFT_SPIN_LIMIT; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (tw()) return true;
     if ((i & 255u) == 255u) {
       if (*abort_flag) return false;
       if (globaltimer() - t0 > 4000000000ull) break;
@@ -118,6 +132,51 @@ __device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
                : "memory");
+}
+// The SM-pair forms (cta_group::2): the two CTAs of a 2-CTA cluster share one M = 256 product.
+// The even CTA issues the MMA; each CTA holds its own 128 rows of A and 128 of the 256 B rows
+// in shared memory at the same offsets, and its own 128 accumulator rows in tensor memory.
+__device__ __forceinline__ void umma_f16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum));
+}
+// Arrive on the mbarrier at this offset in both CTAs of the pair once the pair's MMAs are done.
+__device__ __forceinline__ void umma_commit_pair(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(
+          bar),
+      "h"((uint16_t)3)
+      : "memory");
+}
+// TMA load into this CTA's shared memory whose completion is counted on an mbarrier of either
+// CTA of the pair (bar: a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3}], [%4];\n" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+  return r;
+}
+// The shared::cluster address of this CTA's shared variable at `addr` in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(d) : "r"(addr), "r"(rank));
+  return d;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  __syncwarp();
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;\n" ::: "memory");
 }
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
@@ -239,16 +298,21 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
   }
 }
 
-// BN_ x STAGES_: 256 x 4 for the prefill; 128 x 6 for few-row products with the operands swapped
-// (weights as the 128-row operand, the few activation rows as the N side; EPI_STORE_F32_T).
-template <int EPI, int BN_, int STAGES_>
+// BN_ x STAGES_: 256 x 4 for the prefill on one SM; 128 x 6 for few-row products with the
+// operands swapped (weights as the 128-row operand, the few activation rows as the N side;
+// EPI_STORE_F32_T).  PAIR: 2-CTA clusters on an SM pair, 256 x 256 tiles (cta_group::2): each SM
+// stages 128 rows of A and 128 of the 256 B rows per k-block, half the B traffic of one SM per
+// tile row, and the even CTA issues the M = 256 MMAs into both SMs' tensor memory.
+template <int EPI, int BN_, int STAGES_, bool PAIR = false>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
                    int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride) {
   constexpr int BN = BN_, STAGES = STAGES_;  // this instance's tile width and ring depth
-  constexpr int B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr int TM = PAIR ? 2 * BM : BM;     // rows of a tile (both CTAs of the pair)
+  constexpr int B_ROWS = PAIR ? BN / 2 : BN; // B rows staged by this CTA
+  constexpr int B_BYTES = B_ROWS * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
   constexpr int ACC_COLS = BN, TMEM_COLS = 2 * ACC_COLS;
-  constexpr uint32_t IDESC_T = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+  constexpr uint32_t IDESC_T = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -270,24 +334,35 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), 128);
+      mbar_init(tempty_bar(b), PAIR ? 256 : 128);  // the epilogue threads of every CTA that drains it
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
   }
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  if constexpr (PAIR) cluster_sync();  // both CTAs' barriers initialised before any remote arrival
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+    if constexpr (PAIR) {
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;\n" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+    }
   }
   fence_before();
   __syncthreads();
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int mt = (M + BM - 1) / BM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
+  const int mt = (M + TM - 1) / TM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
   const int n_tiles = mt * nt;
   // unit u: tile u / splits, K-blocks [k0, k1) of slice u % splits (the host makes every slice
   // non-empty)
@@ -297,12 +372,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     k1 = min(kt, k0 + k_per);
   };
 
+  // the pair walks the units together, one unit per cluster
+  const int u_first = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int u_step = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer
+      // ---------------- TMA producer (PAIR: both CTAs load their halves; the even CTA's full
+      // barrier counts the bytes of both)
       int it = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      for (int u = u_first; u < n_units && ok; u += u_step) {
         int m_blk, n_blk, k0, k1;
         tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
         unit_k(u, k0, k1);
@@ -310,31 +390,41 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
           if (!mbar_wait(empty_bar(s), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
-          mbar_expect_tx(full_bar(s), STAGE_BYTES);
-          tma_load_2d(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * BM, full_bar(s));
-          tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+          if constexpr (PAIR) {
+            const uint32_t fb = mapa_shared(full_bar(s), 0);
+            if (rank == 0) mbar_expect_tx(full_bar(s), 2 * STAGE_BYTES);
+            tma_load_2d_pair(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * TM + (int)rank * BM, fb);
+            tma_load_2d_pair(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN + (int)rank * B_ROWS, fb);
+          } else {
+            mbar_expect_tx(full_bar(s), STAGE_BYTES);
+            tma_load_2d(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * BM, full_bar(s));
+            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+          }
         }
       }
-      // Before leaving, make sure no copy this thread issued is still in flight (bounded).
+      // Before leaving, make sure no copy this thread issued is still in flight (bounded).  PAIR:
+      // the copies are counted on the even CTA's barrier, so wait instead for the MMAs' releases
+      // of the last stages, which also keeps this CTA alive until they have all arrived.
       for (int j = 1; j <= STAGES && it - j >= 0; ++j) {
         const int i2 = it - j;
         const int s = i2 % STAGES;
         const uint32_t round = i2 / STAGES;
-        for (uint32_t w = 0; w < (1u << 22) && !mbar_try_wait(full_bar(s), round & 1u); ++w) {
+        const uint32_t bar = PAIR ? empty_bar(s) : full_bar(s);
+        for (uint32_t w = 0; w < (1u << 22) && !mbar_try_wait(bar, round & 1u); ++w) {
         }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (PAIR: the even CTA only)
       int it = 0, tl = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++tl) {
+      for (int u = u_first; u < n_units && ok; u += u_step, ++tl) {
         int k0, k1;
         unit_k(u, k0, k1);
         const int b = tl & 1;
         const uint32_t use = tl >> 1;
-        if (!mbar_wait(tempty_bar(b), (use & 1u) ^ 1u, abort_flag)) break;
+        if (!mbar_wait<PAIR>(tempty_bar(b), (use & 1u) ^ 1u, abort_flag)) break;
         fence_after();
         const uint32_t tmem_d = tmem_base + (uint32_t)(b * ACC_COLS);
         for (int k = k0; k < k1; ++k, ++it) {
@@ -345,18 +435,34 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t ad = smem_desc(smem_u32(sA + s * A_BYTES));
           const uint64_t bd = smem_desc(smem_u32(sB + s * B_BYTES));
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along K per step (encoded >> 4)
-            umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, IDESC_T, (k != k0 || kk != 0) ? 1u : 0u);
-          umma_commit(empty_bar(s));
+          for (int kk = 0; kk < BK / 16; ++kk) {  // +32 bytes along K per step (encoded >> 4)
+            if constexpr (PAIR)
+              umma_f16_pair(tmem_d, ad + 2 * kk, bd + 2 * kk, IDESC_T, (k != k0 || kk != 0) ? 1u : 0u);
+            else
+              umma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, IDESC_T, (k != k0 || kk != 0) ? 1u : 0u);
+          }
+          if constexpr (PAIR) umma_commit_pair(empty_bar(s));
+          else umma_commit(empty_bar(s));
         }
-        if (ok) umma_commit(tfull_bar(b));
+        if (ok) {
+          if constexpr (PAIR) umma_commit_pair(tfull_bar(b));
+          else umma_commit(tfull_bar(b));
+        }
+      }
+      if constexpr (PAIR) {
+        // the last two accumulators' releases (the odd CTA's arrivals among them) have landed
+        for (int t = tl - 1; t >= 0 && t >= tl - 2; --t)
+          for (uint32_t w = 0; w < (1u << 22) && !mbar_try_wait_cluster(tempty_bar(t & 1), (t >> 1) & 1u); ++w) {
+          }
       }
     }
   } else {
     // ---------------- epilogue (warps 2..5 -> TMEM lane quarters 2, 3, 0, 1)
     const int quarter = warp & 3;
+    const uint32_t tempty_even0 = PAIR ? mapa_shared(tempty_bar(0), 0) : tempty_bar(0);
+    const uint32_t tempty_even1 = PAIR ? mapa_shared(tempty_bar(1), 0) : tempty_bar(1);
     int tl = 0;
-    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++tl) {
+    for (int u = u_first; u < n_units; u += u_step, ++tl) {
       int m_blk, n_blk;
       tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
       // split-K partials (EPI_STORE_F32 only): slice u % splits at C + slice * split_stride
@@ -365,7 +471,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t use = tl >> 1;
       if (!mbar_wait(tfull_bar(b), use & 1u, abort_flag)) break;
       fence_after();
-      const int row = m_blk * BM + quarter * 32 + lane;
+      const int row = m_blk * TM + (int)rank * BM + quarter * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * ACC_COLS);
       if constexpr (EPI == EPI_QKV_ROPE) {
         const int half = ep.head_dim >> 1;
@@ -407,15 +513,21 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
       fence_before();
-      mbar_arrive(tempty_bar(b));
+      if constexpr (PAIR) mbar_arrive_cluster(b ? tempty_even1 : tempty_even0);
+      else mbar_arrive(tempty_bar(b));
     }
   }
   fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();  // neither CTA frees its tensor memory or exits before the other is done
   if (warp == 1) {
     fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TMEM_COLS)
-                 : "memory");
+    if constexpr (PAIR)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TMEM_COLS)
+                   : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TMEM_COLS)
+                   : "memory");
   }
 }
 
@@ -476,6 +588,47 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
   gemm_tc_kernel<EPI, BN_, STAGES_><<<grid, THREADS, smem, st>>>(a, b, M, N, K, C, ep, group_m, splits, (size_t)M * N);
   return 0;
+}
+
+// The paired kernel (2-CTA clusters, 256 x 256 tiles), persistent over as many clusters as can be
+// resident at once.  b: the B map with 128-row boxes.  Returns -1 if no cluster can be resident
+// (the caller then uses one SM per tile).
+constexpr int PAIR_STAGES = 6;
+template <int EPI>
+static int launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
+                       cudaStream_t st) {
+  constexpr size_t smem = (size_t)PAIR_STAGES * (A_BYTES + (BN / 2) * BK * 2) + 1024 + 256;
+  auto kern = gemm_tc_kernel<EPI, BN, PAIR_STAGES, true>;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  static int max_clusters = -1;
+  if (max_clusters < 0) {
+    int n = 0;
+    cfg.gridDim = dim3(2, 1, 1);
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    max_clusters = n;
+  }
+  if (max_clusters <= 0) return -1;
+  const int units = ((M + 2 * BM - 1) / (2 * BM)) * ((N + BN - 1) / BN);
+  const int clusters = units < max_clusters ? units : max_clusters;
+  // bands of 256-row tiles whose A rows fit in ~48 MB of L2
+  int group_m = (int)((48u << 20) / ((size_t)2 * BM * K * 2));
+  group_m = group_m < 4 ? 4 : (group_m > 32 ? 32 : group_m);
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  cfg.stream = st;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, M, N, K, C, ep, group_m, 1, (size_t)M * N) == cudaSuccess ? 0 : 1;
 }
 
 // Sum of the split-K slices (in slice order) and the epilogue EPI, four consecutive outputs per
@@ -692,6 +845,21 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   if (splits > 1 || fuse_norm) {
     if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits)) return 1;
     return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st);
+  }
+  // Many rows: 256 x 256 tiles on SM pairs.
+  if (M >= 1024) {
+    CUtensorMap mb2;
+    if (!make_map(&mb2, B, (uint64_t)K, (uint64_t)N, BN / 2)) return 1;
+    int r = -1;
+    switch (epi) {
+      case EPI_STORE_BF16: r = launch_pair<EPI_STORE_BF16>(ma, mb2, M, N, K, C, ep, st); break;
+      case EPI_RESID_F32: r = launch_pair<EPI_RESID_F32>(ma, mb2, M, N, K, C, ep, st); break;
+      case EPI_SWIGLU: r = launch_pair<EPI_SWIGLU>(ma, mb2, M, N, K, C, ep, st); break;
+      case EPI_QKV_ROPE: r = launch_pair<EPI_QKV_ROPE>(ma, mb2, M, N, K, C, ep, st); break;
+      case EPI_STORE_F32: r = launch_pair<EPI_STORE_F32>(ma, mb2, M, N, K, C, ep, st); break;
+      default: return 1;
+    }
+    if (r >= 0) return r;
   }
   switch (epi) {
     case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, ep, st);

@@ -23,8 +23,11 @@ def _rel(g, o):
     return float((g.double() - o).abs().max() / o.abs().max())
 
 
+# M >= 1024 runs on SM pairs (256 x 256 tiles): ragged last tiles whose second 128 rows or second
+# 128 B rows lie wholly or partly outside the operands.
 SHAPES = [(1, 256, 64), (128, 256, 64), (129, 264, 72), (200, 768, 256), (384, 256, 688), (333, 1024, 4096),
-          (1000, 4096, 4096), (300, 12288, 4096)]
+          (1000, 4096, 4096), (300, 12288, 4096), (1100, 264, 72), (2000, 640, 200), (4097, 768, 128),
+          (1024, 4096, 4096)]
 
 
 @pytest.mark.parametrize("M,N,K", SHAPES)
@@ -37,7 +40,8 @@ def test_store_bf16(M, N, K, cuda, riftlib):
     assert _rel(out.cpu(), ref) < F16_TOL
 
 
-@pytest.mark.parametrize("M,N,K", [(129, 264, 72), (384, 256, 688), (777, 4096, 4096), (257, 4096, 11008)])
+@pytest.mark.parametrize("M,N,K", [(129, 264, 72), (384, 256, 688), (777, 4096, 4096), (257, 4096, 11008),
+                                   (1500, 4096, 688), (1030, 264, 11008)])
 def test_residual_f32(M, N, K, cuda, riftlib):
     A, W = _rand((M, K), 3), _rand((N, K), 4, 0.05)
     R0 = rng.normal_f32(5, 77, M * N).view(M, N)
@@ -48,7 +52,7 @@ def test_residual_f32(M, N, K, cuda, riftlib):
     assert _rel(R.cpu(), ref) < F32_TOL
 
 
-@pytest.mark.parametrize("M,F,K", [(96, 688, 256), (300, 1376, 688), (513, 11008, 4096)])
+@pytest.mark.parametrize("M,F,K", [(96, 688, 256), (300, 1376, 688), (513, 11008, 4096), (1300, 1376, 688)])
 def test_swiglu(M, F, K, cuda, riftlib):
     from paper_2609_29029_gb300 import interleave_gate_up
     A = _rand((M, K), 5)
