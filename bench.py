@@ -39,7 +39,7 @@ def parse():
     ap.add_argument("--workload", default="rift400_7b", choices=sorted(W.WORKLOADS))
     ap.add_argument("--impl", default="rift", choices=["rift", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-step measurement")
     ap.add_argument("--no-shared-prefix", action="store_true", help="skip the shared-prefix measurement")
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
@@ -579,10 +579,11 @@ def main():
     barrier(ws)
     torch.cuda.synchronize()
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    f0.record(stream)
-    Te = e2e_steps(args.e2e_steps)
-    f1.record(stream)
-    torch.cuda.synchronize()
+    with ClockSampler(local) as clk_e2e:
+        f0.record(stream)
+        Te = e2e_steps(args.e2e_steps)
+        f1.record(stream)
+        torch.cuda.synchronize()
     e2e_val, _ = job_throughput(float(Te * args.e2e_steps), f0.elapsed_time(f1), ws)
     h2d_bytes = X_host.numel() * X_host.element_size() + embed_host.numel() * 2 + sum(h.numel() * 4 for h in ids_host)
     d2h = Te * s.d * 2 + 8
@@ -627,7 +628,8 @@ def main():
                      "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (of measured)",
                      "launches": gemm_n},
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h},
+        "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h,
+                "steps": args.e2e_steps, "clocks": clk_e2e.summary()},
         "decode_step": decode,
         "shared_prefix": shared,
         "gpu_launches": launches,
