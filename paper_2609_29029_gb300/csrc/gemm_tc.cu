@@ -306,7 +306,8 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
 template <int EPI, int BN_, int STAGES_, bool PAIR = false>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride) {
+                   int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride,
+                   int a_const) {
   constexpr int BN = BN_, STAGES = STAGES_;  // this instance's tile width and ring depth
   constexpr int TM = PAIR ? 2 * BM : BM;     // rows of a tile (both CTAs of the pair)
   constexpr int B_ROWS = PAIR ? BN / 2 : BN; // B rows staged by this CTA
@@ -361,6 +362,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  if (warp != 0) pdl_wait();  // the producer waits after prefetching constant A tiles
 
   const int mt = (M + TM - 1) / TM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
   const int n_tiles = mt * nt;
@@ -380,6 +383,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (lane == 0) {
       // ---------------- TMA producer (PAIR: both CTAs load their halves; the even CTA's full
       // barrier counts the bytes of both)
+      // a_const: A does not depend on earlier kernels (weights), so the first ring round of this
+      // CTA's first unit takes its A tiles before waiting for the kernel before this one.
+      int n_pre = 0;
+      if (!PAIR && a_const && u_first < n_units) {
+        int m_blk, n_blk, k0, k1;
+        tile_coords(u_first / splits, mt, nt, group_m, m_blk, n_blk);
+        unit_k(u_first, k0, k1);
+        n_pre = min(STAGES, k1 - k0);
+        for (int j = 0; j < n_pre; ++j) {
+          mbar_expect_tx(full_bar(j), STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + j * A_BYTES), &tmA, (k0 + j) * BK, m_blk * BM, full_bar(j));
+        }
+      }
+      pdl_wait();
       int it = 0;
       bool ok = true;
       for (int u = u_first; u < n_units && ok; u += u_step) {
@@ -389,6 +406,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int k = k0; k < k1; ++k, ++it) {
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
+          if (it < n_pre) {  // A already requested (first round: the stage is free)
+            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+            continue;
+          }
           if (!mbar_wait(empty_bar(s), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
           if constexpr (PAIR) {
             const uint32_t fb = mapa_shared(full_bar(s), 0);
@@ -571,9 +592,10 @@ static int sm_count() {
   return n;
 }
 
+// pdl: launched as a programmatic dependent of the kernel before it; a_const: A is constant weights.
 template <int EPI, int BN_ = BN, int STAGES_ = STAGES>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
-                  cudaStream_t st, int splits = 1) {
+                  cudaStream_t st, int splits = 1, bool pdl = false, int a_const = 0) {
   constexpr size_t smem = (size_t)STAGES_ * (A_BYTES + BN_ * BK * 2) + 1024 + 256;
   static bool attr = false;
   if (!attr) {
@@ -586,8 +608,8 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   // weight tile is streamed from DRAM once per band.
   int group_m = (int)((48u << 20) / ((size_t)BM * K * 2));
   group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
-  gemm_tc_kernel<EPI, BN_, STAGES_><<<grid, THREADS, smem, st>>>(a, b, M, N, K, C, ep, group_m, splits, (size_t)M * N);
-  return 0;
+  return launch_ex(gemm_tc_kernel<EPI, BN_, STAGES_>, dim3(grid), dim3(THREADS), smem, st, pdl, a, b, M, N, K, C, ep,
+                   group_m, splits, (size_t)M * N, a_const) != cudaSuccess;
 }
 
 // The paired kernel (2-CTA clusters, 256 x 256 tiles), persistent over as many clusters as can be
@@ -628,7 +650,7 @@ static int launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
   group_m = group_m < 4 ? 4 : (group_m > 32 ? 32 : group_m);
   cfg.gridDim = dim3(2 * clusters, 1, 1);
   cfg.stream = st;
-  return cudaLaunchKernelEx(&cfg, kern, a, b, M, N, K, C, ep, group_m, 1, (size_t)M * N) == cudaSuccess ? 0 : 1;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, M, N, K, C, ep, group_m, 1, (size_t)M * N, 0) == cudaSuccess ? 0 : 1;
 }
 
 // Sum of the split-K slices (in slice order) and the epilogue EPI, four consecutive outputs per
@@ -638,6 +660,8 @@ static int launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
 template <int EPI>
 __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, int M, int N, void* C,
                                      const EpiParams ep) {
+  pdl_trigger();
+  pdl_wait();
   const size_t stride = (size_t)M * N;
   const int n_out = EPI == EPI_SWIGLU ? N / 2 : N;
   const int q_out = n_out / 4;
@@ -709,6 +733,8 @@ __global__ void __launch_bounds__(256) splitk_resid_norm_kernel(const float* __r
                                                                 const uint16_t* __restrict__ gain, float eps,
                                                                 uint16_t* __restrict__ out) {
   __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
   const size_t row = blockIdx.x, stride = (size_t)M * N;
   const int nv = N / 4;
   float4 v[8];
@@ -787,23 +813,23 @@ __global__ void wait_timeout_check_kernel() {
 // The slices' partial products [splits][M][N] summed in slice order with the epilogue epi (a
 // residual product with ep.norm_out also applies the following RMSNorm).
 static int reduce_slices(const float* part, int splits, int M, int N, int epi, void* C, const EpiParams& ep,
-                         cudaStream_t st) {
-  if (epi == EPI_RESID_F32 && ep.norm_out) {
-    splitk_resid_norm_kernel<<<M, 256, 0, st>>>(part, splits, M, N, static_cast<float*>(C),
-                                                 static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out);
-    return 0;
-  }
+                         cudaStream_t st, bool pdl) {
+  if (epi == EPI_RESID_F32 && ep.norm_out)
+    return launch_ex(splitk_resid_norm_kernel, dim3(M), dim3(256), 0, st, pdl, part, splits, M, N,
+                     static_cast<float*>(C), static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out) !=
+           cudaSuccess;
   const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N) / 4;
-  const int grid = (int)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048);
+  const dim3 grid((unsigned)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048));
+  cudaError_t e;
   switch (epi) {
-    case EPI_STORE_BF16: splitk_reduce_kernel<EPI_STORE_BF16><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-    case EPI_RESID_F32: splitk_reduce_kernel<EPI_RESID_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-    case EPI_SWIGLU: splitk_reduce_kernel<EPI_SWIGLU><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-    case EPI_QKV_ROPE: splitk_reduce_kernel<EPI_QKV_ROPE><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
-    case EPI_STORE_F32: splitk_reduce_kernel<EPI_STORE_F32><<<grid, 256, 0, st>>>(part, splits, M, N, C, ep); break;
+    case EPI_STORE_BF16: e = launch_ex(splitk_reduce_kernel<EPI_STORE_BF16>, grid, dim3(256), 0, st, pdl, part, splits, M, N, C, ep); break;
+    case EPI_RESID_F32: e = launch_ex(splitk_reduce_kernel<EPI_RESID_F32>, grid, dim3(256), 0, st, pdl, part, splits, M, N, C, ep); break;
+    case EPI_SWIGLU: e = launch_ex(splitk_reduce_kernel<EPI_SWIGLU>, grid, dim3(256), 0, st, pdl, part, splits, M, N, C, ep); break;
+    case EPI_QKV_ROPE: e = launch_ex(splitk_reduce_kernel<EPI_QKV_ROPE>, grid, dim3(256), 0, st, pdl, part, splits, M, N, C, ep); break;
+    case EPI_STORE_F32: e = launch_ex(splitk_reduce_kernel<EPI_STORE_F32>, grid, dim3(256), 0, st, pdl, part, splits, M, N, C, ep); break;
     default: return 1;
   }
-  return 0;
+  return e != cudaSuccess;
 }
 
 }  // namespace tc
@@ -816,7 +842,7 @@ int launch_wait_timeout_check(cudaStream_t st) {
 // Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
 // the RoPE epilogue), A, B and C 16-byte aligned.
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st, void* split_ws, size_t split_ws_bytes) {
+                   cudaStream_t st, void* split_ws, size_t split_ws_bytes, bool pdl) {
   using namespace tc;
   if (M <= 0 || N <= 0 || K <= 0) return 0;
   if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
@@ -832,8 +858,9 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     // a unit's partials (M x 128 fp32, written and read back) cost M / 16 K-blocks of weight
     // traffic; its fill and drain about 1.5 more
     const int splits = choose_splits(N, M, K, split_ws_bytes, SW_BN, M / 16.0 + 1.5);
-    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits)) return 1;
-    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st);
+    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits, pdl, 1))
+      return 1;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st, pdl);
   }
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
@@ -843,8 +870,8 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   if (fuse_norm && (!split_ws || N > 8192 || (size_t)M * N * sizeof(float) > split_ws_bytes)) return 1;
   const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
   if (splits > 1 || fuse_norm) {
-    if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits)) return 1;
-    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st);
+    if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits, pdl)) return 1;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st, pdl);
   }
   // Many rows: 256 x 256 tiles on SM pairs.
   if (M >= 1024) {

@@ -149,9 +149,9 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
 }
 
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C, cudaStream_t st,
-                const EpiParams& ep, void* split_ws, size_t split_ws_bytes) {
+                const EpiParams& ep, void* split_ws, size_t split_ws_bytes, bool pdl) {
   prof_begin(RIFT_PROF_GEMM, st);
-  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, ep, st, split_ws, split_ws_bytes);
+  const int r = launch_gemm_tc(A, B, M, N, K, epi, C, ep, st, split_ws, split_ws_bytes, pdl);
   prof_end(RIFT_PROF_GEMM, st, 1);
   return r;
 }
@@ -356,6 +356,8 @@ __global__ void __launch_bounds__(DEC_HG * 32, 3) decode_attn_kernel(const uint1
                                                                      const int* __restrict__ cu, int H, int hg,
                                                                      int max_chunks, float scale_log2,
                                                                      float* __restrict__ part) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int LPK = HD / 8, KPL = 32 / LPK;  // lanes per key, keys per warp-wide load
   constexpr int NL = 4;                        // warp-wide loads of K (and of V) in flight
   const int groups = H / hg;  // hg = blockDim.x / 32 heads per CTA
@@ -450,6 +452,8 @@ __global__ void __launch_bounds__(DEC_HG * 32, 3) decode_attn_kernel(const uint1
 // A sequence with more than max_keys keys sets RIFT_EBIT_CAPACITY and gets zeros.
 __global__ void decode_combine_kernel(const float* __restrict__ part, const int* __restrict__ cu, int H, int HD,
                                       int max_chunks, int max_keys, uint16_t* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x / H, h = blockIdx.x % H;
   const int nk = cu[i + 1] - cu[i] + 1;
   uint16_t* o = out + ((size_t)i * H + h) * HD;
@@ -517,8 +521,12 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
     return e;
   };
   norm_launch(0, n, x0, h32, m.g_attn[0], xn, d, m.eps, st);
+  // The layer's kernels are launched as programmatic dependents of the kernel before them: each
+  // starts while its predecessor drains (the GEMMs already streaming their first weight tiles)
+  // and waits for it before touching activations.
+  const bool pdl = true;
   for (int l = 0; l < m.n_layers; ++l) {
-    if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep, split, sb)) return 1;
+    if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep, split, sb, pdl)) return 1;
     if (kv_new) {
       uint16_t* kl = static_cast<uint16_t*>(kv_new) + (size_t)l * 2 * n * d;
       kv_store(qkv, n, d, kl, kl + (size_t)n * d, st);
@@ -527,24 +535,28 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
     const uint16_t* Vc = Kc + (size_t)T * d;
     prof_begin(RIFT_PROF_ATTN, st);
     const int units = n * max_chunks * (m.n_heads / hg);
+    cudaError_t e;
     if (m.head_dim == 128)
-      decode_attn_kernel<128><<<units, hg * 32, 0, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, hg, max_chunks, scale_log2,
-                                                         dpart);
+      e = launch_ex(decode_attn_kernel<128>, dim3(units), dim3(hg * 32), 0, st, pdl, (const uint16_t*)qkv, Kc, Vc,
+                    cu_seqlens, (int)m.n_heads, hg, max_chunks, scale_log2, dpart);
     else
-      decode_attn_kernel<64><<<units, hg * 32, 0, st>>>(qkv, Kc, Vc, cu_seqlens, m.n_heads, hg, max_chunks, scale_log2,
-                                                        dpart);
-    decode_combine_kernel<<<n * m.n_heads, m.head_dim, 0, st>>>(dpart, cu_seqlens, m.n_heads, m.head_dim, max_chunks,
-                                                                max_len, att);
+      e = launch_ex(decode_attn_kernel<64>, dim3(units), dim3(hg * 32), 0, st, pdl, (const uint16_t*)qkv, Kc, Vc,
+                    cu_seqlens, (int)m.n_heads, hg, max_chunks, scale_log2, dpart);
+    if (e != cudaSuccess) return 1;
+    if (launch_ex(decode_combine_kernel, dim3(n * m.n_heads), dim3(m.head_dim), 0, st, pdl, (const float*)dpart,
+                  cu_seqlens, (int)m.n_heads, (int)m.head_dim, max_chunks, max_len, att) != cudaSuccess)
+      return 1;
     prof_end(RIFT_PROF_ATTN, st, 2);
-    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st, resid_norm(m.g_ffn[l]), split, sb)) return 1;
-    if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st, EpiParams(), split, sb)) return 1;
+    if (launch_gemm(att, m.w_o[l], n, d, d, EPI_RESID_F32, h32, st, resid_norm(m.g_ffn[l]), split, sb, pdl)) return 1;
+    if (launch_gemm(xn, m.w_gate_up[l], n, 2 * m.ffn, d, EPI_SWIGLU, act, st, EpiParams(), split, sb, pdl)) return 1;
     const void* next_gain = l + 1 < m.n_layers ? m.g_attn[l + 1] : m.g_final;
-    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st, resid_norm(next_gain), split, sb)) return 1;
+    if (launch_gemm(act, m.w_down[l], n, d, m.ffn, EPI_RESID_F32, h32, st, resid_norm(next_gain), split, sb, pdl))
+      return 1;
   }
   // xn now holds RMSNorm(h) g_final in fp16 (the logits operand)
   if (hidden_out) norm_launch(2, n, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden_out), d, m.eps, st);
   if (logits) {
-    if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st, EpiParams(), split, sb)) return 1;
+    if (launch_gemm(xn, m.lm_head, n, m.vocab, d, EPI_STORE_F32, logits, st, EpiParams(), split, sb, pdl)) return 1;
   }
   return 0;
 }

@@ -116,11 +116,12 @@ struct EpiParams {
 };
 // split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
 // most SMs idle run as (tile, K-slice) units plus a reduction kernel.
+// pdl: launch as a programmatic dependent of the previous kernel in the stream (decode step).
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
                 cudaStream_t st, const EpiParams& ep = EpiParams(), void* split_ws = nullptr,
-                size_t split_ws_bytes = 0);
+                size_t split_ws_bytes = 0, bool pdl = false);
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0);
+                   cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0, bool pdl = false);
 int launch_wait_timeout_check(cudaStream_t st);
 
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
