@@ -42,6 +42,7 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-step measurement")
     ap.add_argument("--no-shared-prefix", action="store_true", help="skip the shared-prefix measurement")
+    ap.add_argument("--no-batch", action="store_true", help="skip the multi-query batch measurement")
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
@@ -412,6 +413,47 @@ def decode_measure(pipe, dm, sc, dec, n_kept, T, stream, steps):
             "bound": "hbm", "inputs": "seeded token ids; KV cache from the prefill of the same query"}
 
 
+def batch_measure(dm, dec, base, stream, steps, B=8, N=64):
+    """Several scene queries per prefill (rift_pack_ragged_at): B queries over B different
+    N-tile scenes (the small end of the paper's 64..400-tile scenes), timed batched against one
+    query at a time.  Reported beside the metric."""
+    from dataclasses import replace
+    from paper_2609_29029_gb300 import ScenePipeline
+    dev = torch.device("cuda", torch.cuda.current_device())
+    i32 = dict(dtype=torch.int32, device=dev)
+    spec = replace(base.scene, N=N)
+    queries = []
+    for b in range(B):
+        sc = W.make_scene(replace(spec, seed=100 + b), dec.vocab, dev)
+        q = torch.tensor(sc.query_ids, **i32)
+        queries.append((sc.X, sc.embed, q, torch.tensor(sc.bg_ids, **i32), torch.tensor(sc.sys_ids, **i32), q))
+    pipe = ScenePipeline(N, spec.n_v, spec.d, spec.x_dtype, spec.M, spec.S, spec.Q, base.knn_m, base.policy,
+                         model=dm, device=dev)
+    res = pipe.run_batch(queries, stream=stream)
+    for qq in queries:
+        pipe.run(*qq, stream=stream)
+    torch.cuda.synchronize()
+    rows = sum(r[1] for r in res)
+
+    def timed(fn):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps
+
+    ms_b = timed(lambda: pipe.run_batch(queries, stream=stream))
+    ms_1 = timed(lambda: [pipe.run(*qq, stream=stream) for qq in queries])
+    del queries, pipe
+    torch.cuda.empty_cache()
+    return {"queries": B, "tiles_per_scene": N, "retained_rows": rows,
+            "batched_ms": ms_b, "one_at_a_time_ms": ms_1,
+            "batched_scene_queries_per_s": B / (ms_b / 1e3), "one_at_a_time_scene_queries_per_s": B / (ms_1 / 1e3),
+            "batched_tokens_per_s": rows / (ms_b / 1e3)}
+
+
 def kernel_case(name: str):
     """Small cases for ncu captures: inputs larger than L2, about 1 GB on the device."""
     import __graft_entry__
@@ -589,6 +631,7 @@ def main():
     d2h = Te * s.d * 2 + 8
     decode = None if args.no_decode else decode_measure(pipe, dm, sc, dec, n_kept, T, stream, args.steps)
     shared = None if args.no_shared_prefix else shared_prefix_measure(pipe, sc, q, bg, sy, T, stream, args.steps)
+    batch = None if args.no_batch else batch_measure(dm, dec, wl, stream, max(2, args.steps // 2))
 
     if rank != 0:
         return
@@ -632,6 +675,7 @@ def main():
                 "steps": args.e2e_steps, "clocks": clk_e2e.summary()},
         "decode_step": decode,
         "shared_prefix": shared,
+        "batch": batch,
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }

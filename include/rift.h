@@ -12,6 +12,7 @@
  *                                (Section 2.3 Stage 2), and each kept tile's top-b tokens
  *   rift_pack_ragged             one sequence per kept tile, [system | tokens | query],
  *                                packed back to back with varlen offsets
+ *                                (rift_pack_ragged_at: a later query of a batch)
  *   rift_prefill_layers          the decoder prefill over the packed batch (Section 2.1)
  *
  * Conventions shared by every call
@@ -267,6 +268,25 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
                              const void* embed, int vocab, const void* ctx, const int* ctx_off,
                              void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
                              rift_stream_t stream);
+
+/* ---- a8 for a batch of scene queries (several queries in one prefill) ----
+ * The paper answers one scene query at a time; a server batches several.  Packing them into
+ * one batch is rift_pack_ragged once per query, each time with packed, positions and
+ * cu_seqlens pointing at the query's part of the batch buffers (after the rows and sequences
+ * of the queries before it) and row_base = the rows before it, so that the batch's
+ * cu_seqlens holds absolute row offsets:
+ *   cu_seqlens[j] = row_base + (the rift_pack_ragged value); T out = this query's rows alone;
+ *   max_T = the rows left in the batch buffer.  row_base = 0 is rift_pack_ragged.
+ * The sequences stay independent (no attention across them), so each query's final hidden
+ * states are those of its own prefill, row for row.
+ * row_base < 0 returns RIFT_ERR_INVALID. */
+rift_status rift_pack_ragged_at(const void* X, rift_dtype xdt, int N, int n_v, int d,
+                                const int* kept, const int* n_kept,
+                                const int* sel, const int* sel_off,
+                                const int* sys_ids, int S, const int* query_ids, int Q,
+                                const void* embed, int vocab, const void* ctx, const int* ctx_off,
+                                void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
+                                int row_base, rift_stream_t stream);
 
 /* ---- a9. Decoder prefill (Section 2.1) ----
  *   hidden     bf16 [T, d]: in, the packed batch; out, the final hidden states (after the

@@ -56,6 +56,8 @@ SIGNATURES = {
                                          _vp, _vp, _sz, _vp]),
     "rift_pack_ragged": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp,
                               _vp, _i, _vp, _vp, _vp, _vp]),
+    "rift_pack_ragged_at": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp,
+                                 _vp, _i, _vp, _vp, _vp, _i, _vp]),
     "rift_features_workspace_bytes": (_sz, [_i, _i]),
     "rift_tile_features": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "rift_merge_workspace_bytes": (_sz, [_i, _i]),
@@ -183,7 +185,15 @@ def select_budgeted_tokens(token_scores, tile_s, N, n_v, p, policy: Policy, u, k
 
 
 def pack_ragged(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, packed,
-                max_T, cu_seqlens, positions, T, stream=None, ctx=None, ctx_off=None):
+                max_T, cu_seqlens, positions, T, stream=None, ctx=None, ctx_off=None, row_base=0):
+    """rift_pack_ragged, or rift_pack_ragged_at with row_base > 0 (a later query of a batch:
+    packed, cu_seqlens and positions are then that query's part of the batch buffers)."""
+    if row_base:
+        _check(lib.rift_pack_ragged_at(ptr(X), xdt, N, n_v, d, ptr(kept), ptr(n_kept), ptr(sel), ptr(sel_off),
+                                       ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(ctx),
+                                       ptr(ctx_off), ptr(packed), max_T, ptr(cu_seqlens), ptr(positions), ptr(T),
+                                       row_base, stream_handle(stream)), "rift_pack_ragged_at")
+        return
     _check(lib.rift_pack_ragged(ptr(X), xdt, N, n_v, d, ptr(kept), ptr(n_kept), ptr(sel), ptr(sel_off),
                                 ptr(sys_ids), S, ptr(query_ids), Q, ptr(embed), vocab, ptr(ctx), ptr(ctx_off),
                                 ptr(packed), max_T, ptr(cu_seqlens), ptr(positions), ptr(T), stream_handle(stream)),

@@ -23,15 +23,16 @@ unsigned int read_clear_err_pack() {
 constexpr int PK_ROWS = 32;
 constexpr int PK_THREADS = 256;
 
-// cu_seqlens[j] = min(j, n) (S + Q) + sel_off[min(j, n)] + ctx_off[min(j, n)], T = cu_seqlens[n].
+// cu_seqlens[j] = row_base + min(j, n) (S + Q) + sel_off[min(j, n)] + ctx_off[min(j, n)],
+// T = cu_seqlens[n] - row_base (row_base: rows of the queries packed before this one).
 __global__ void seqlens_kernel(const int* __restrict__ n_kept, const int* __restrict__ sel_off,
-                               const int* __restrict__ ctx_off, int N, int S, int Q, int max_T,
+                               const int* __restrict__ ctx_off, int N, int S, int Q, int max_T, int row_base,
                                int* __restrict__ cu, int* __restrict__ T) {
   const int n = *n_kept;
   for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= N; j += gridDim.x * blockDim.x) {
     const int jj = min(j, n);
     const int v = jj * (S + Q) + sel_off[jj] + (ctx_off ? ctx_off[jj] : 0);
-    cu[j] = v;
+    cu[j] = row_base + v;
     if (j == N) {
       *T = v;
       if (v > max_T) atomicOr(&g_err_pack, RIFT_EBIT_CAPACITY);
@@ -218,8 +219,10 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
 void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
                  const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
                  const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
-                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, cudaStream_t st) {
-  seqlens_kernel<<<(N + 1 + 255) / 256, 256, 0, st>>>(n_kept, sel_off, ctx_off, N, S, Q, max_T, cu_seqlens, T);
+                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, int row_base,
+                 cudaStream_t st) {
+  seqlens_kernel<<<(N + 1 + 255) / 256, 256, 0, st>>>(n_kept, sel_off, ctx_off, N, S, Q, max_T, row_base,
+                                                      cu_seqlens, T);
   const uint16_t* cx = static_cast<const uint16_t*>(ctx);
   const int max_L = S + n_v + Q;
   dim3 grid(N, (max_L + PK_ROWS - 1) / PK_ROWS);

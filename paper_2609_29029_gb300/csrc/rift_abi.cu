@@ -98,7 +98,7 @@ rift_status rift_profile_read(double* ms, long long* launches, int n_classes) {
 
 long long rift_launch_count(void) { return g_launches.load(); }
 
-int rift_abi_version(void) { return 3; }
+int rift_abi_version(void) { return 4; }
 
 const char* rift_status_string(rift_status s) {
   switch (s) {
@@ -204,8 +204,17 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
                              const int* query_ids, int Q, const void* embed, int vocab, const void* ctx,
                              const int* ctx_off, void* packed, int max_T, int* cu_seqlens, int* positions, int* T,
                              rift_stream_t stream) {
+  return rift_pack_ragged_at(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab,
+                             ctx, ctx_off, packed, max_T, cu_seqlens, positions, T, 0, stream);
+}
+
+rift_status rift_pack_ragged_at(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
+                                const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
+                                const int* query_ids, int Q, const void* embed, int vocab, const void* ctx,
+                                const int* ctx_off, void* packed, int max_T, int* cu_seqlens, int* positions,
+                                int* T, int row_base, rift_stream_t stream) {
   if (!dims_ok(N, n_v, d) || !X || !kept || !n_kept || !sel || !sel_off || !embed || !packed || !cu_seqlens ||
-      !positions || !T)
+      !positions || !T || row_base < 0)
     return RIFT_ERR_INVALID;
   if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
   if (S < 0 || Q < 0 || (S > 0 && !sys_ids) || (Q > 0 && !query_ids) || vocab < 1 || max_T < 0)
@@ -214,7 +223,7 @@ rift_status rift_pack_ragged(const void* X, rift_dtype xdt, int N, int n_v, int 
   if ((ctx == nullptr) != (ctx_off == nullptr) || (ctx && !aligned16(ctx))) return RIFT_ERR_INVALID;
   prof_begin(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream));
   launch_pack(X, xdt, N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q, embed, vocab, ctx, ctx_off,
-              packed, max_T, cu_seqlens, positions, T, static_cast<cudaStream_t>(stream));
+              packed, max_T, cu_seqlens, positions, T, row_base, static_cast<cudaStream_t>(stream));
   prof_end(RIFT_PROF_PACK, static_cast<cudaStream_t>(stream), 2);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;

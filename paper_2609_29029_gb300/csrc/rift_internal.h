@@ -62,7 +62,8 @@ int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
 void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept,
                  const int* n_kept, const int* sel, const int* sel_off, const int* sys_ids, int S,
                  const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
-                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, cudaStream_t st);
+                 void* packed, int max_T, int* cu_seqlens, int* positions, int* T, int row_base,
+                 cudaStream_t st);
 
 // ---- prefill (prefill.cu, gemm.cu, attention.cu) ----
 struct PrefillLayout {

@@ -215,6 +215,40 @@ class ScenePipeline:
         abi.decode_step(self.model.struct, kv_cache, T, self.cu, n_seq, max_len, token_ids, embed, embed.shape[0],
                         hidden_out, kv_new, logits, ws, need, stream)
 
+    def run_batch(self, queries, prefill=True, stream=None):
+        """Several scene queries through one prefill: each query (a tuple X, embed, phrase_ids,
+        bg_ids, sys_ids, query_ids) is scored, selected and packed after the rows of the ones
+        before it (rift_pack_ragged_at), then the whole batch is prefilled at once.  Returns
+        [(n_kept, T, first row, first sequence)] per query; self.batch_packed[:rows] holds the
+        batch (final hidden states after the prefill), self.batch_cu and
+        self.batch_positions its offsets and positions."""
+        B = len(queries)
+        cap_rows, cap_seq = B * self.max_T, B * self.N
+        if getattr(self, "batch_cap", (0, 0)) < (cap_rows, cap_seq):
+            dev, i32 = self.device, dict(dtype=torch.int32, device=self.device)
+            self.batch_packed = torch.empty(cap_rows, self.d, dtype=torch.bfloat16, device=dev)
+            self.batch_positions = torch.empty(cap_rows, **i32)
+            self.batch_cu = torch.empty(cap_seq + 1, **i32)
+            self.batch_cap = (cap_rows, cap_seq)
+        out, row0, seq0 = [], 0, 0
+        for (X, embed, phrase_ids, bg_ids, sys_ids, query_ids) in queries:
+            self.select(X, embed, phrase_ids, bg_ids, stream=stream)
+            if self.max_m:
+                self.merge(X, stream)
+            abi.pack_ragged(X, self.xdt, self.N, self.n_v, self.d, self.kept, self.n_kept, self.sel, self.sel_off,
+                            sys_ids if self.S else None, self.S, query_ids, self.Q, embed, embed.shape[0],
+                            self.batch_packed[row0:], cap_rows - row0, self.batch_cu[seq0:],
+                            self.batch_positions[row0:], self.T, stream, ctx=self.ctx, ctx_off=self.ctx_off,
+                            row_base=row0)
+            n_kept, T = self.read_counts(stream)
+            out.append((n_kept, T, row0, seq0))
+            row0, seq0 = row0 + T, seq0 + n_kept
+        if prefill and self.model is not None and row0 > 0:
+            ws, need = self._prefill_ws(row0, seq0)
+            abi.prefill_layers(self.model.struct, self.batch_packed, row0, self.batch_cu, seq0, self.max_len,
+                               self.batch_positions, ws, need, stream)
+        return out
+
     def run(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, prefill=True, stream=None):
         self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)
         self.pack(X, embed, sys_ids, query_ids, stream)

@@ -31,7 +31,7 @@ def test_library_exports_every_declared_symbol(riftlib):
 def test_status_strings(riftlib):
     assert riftlib.status_string(0) == "ok"
     assert riftlib.status_string(riftlib.RIFT_ERR_CAPACITY) == "output capacity exceeded"
-    assert riftlib.abi_version() == 3
+    assert riftlib.abi_version() == 4
 
 
 FAKE = 0x10000  # a 16-byte aligned non-null address; validation rejects before using it
@@ -103,6 +103,8 @@ def test_pack_and_prefill_reject_bad_arguments(riftlib):
                                 None, FAKE, 100, FAKE, FAKE, FAKE, 0) == INV  # contextual rows without offsets
     assert lib.rift_pack_ragged(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000, FAKE + 8,
                                 FAKE, FAKE, 100, FAKE, FAKE, FAKE, 0) == INV  # misaligned contextual rows
+    assert lib.rift_pack_ragged_at(FAKE, 1, 4, 576, 256, FAKE, FAKE, FAKE, FAKE, FAKE, 8, FAKE, 16, FAKE, 1000, None,
+                                   None, FAKE, 100, FAKE, FAKE, FAKE, -1, 0) == INV  # negative row base
     m = riftlib.Model()
     m.n_layers, m.d, m.n_heads, m.head_dim, m.ffn, m.eps, m.rope_theta = 2, 256, 4, 64, 688, 1e-6, 1e4
     assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0  # null weight arrays
