@@ -552,6 +552,161 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- merge screening (Stage 2)
+// Similarity of every token of a kept tile to the tile's merge targets on the tensor cores: per
+// (kept slot j, 128-token block) a 128 x 128 x d bf16 product against 128 target rows at a time,
+// one token row per epilogue thread, which keeps the two best targets by x.t / ||t|| (fp32, ties
+// to the lower target) for each unselected token that is not itself a target.  The choice
+// between the two is then made at ~fp64 accuracy outside (merge.cu).  Rows of the block past the
+// tile's tokens and target columns past the slot's m are computed and ignored.
+namespace ms {
+constexpr int STAGES = 3, THREADS = 192, COLS = 128;
+constexpr int A_BYTES = 128 * BK * 2, B_BYTES = COLS * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+// kind::f16 with bf16 A and B (bits 7-9 and 10-12 = 1), fp32 D, K-major, M = N = 128
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(COLS >> 3) << 17) | ((128u >> 4) << 24);
+}  // namespace ms
+
+__global__ void __launch_bounds__(ms::THREADS, 2)
+    merge_screen_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmT, int n_v,
+                        int d, const int* __restrict__ kept, const int* __restrict__ n_kept,
+                        const int* __restrict__ sel_off, const int* __restrict__ ctx_off, int max_ctx,
+                        const float* __restrict__ tinv, const int* __restrict__ pos, int2* __restrict__ cand) {
+  constexpr int STAGES = ms::STAGES, COLS = ms::COLS, A_BYTES = ms::A_BYTES, B_BYTES = ms::B_BYTES,
+                STAGE_BYTES = ms::STAGE_BYTES;
+  constexpr uint32_t IDESC = ms::IDESC;
+  const int j = blockIdx.y, mb = blockIdx.x;
+  if (j >= *n_kept) return;
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  if (m == 0 || co + m > max_ctx) return;  // uniform over the CTA, before any setup
+  const int R = n_v - (sel_off[j + 1] - sel_off[j]);
+  const int step = R / m;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  const uint32_t tfull = bar0 + 8u * (2 * STAGES), tempty = bar0 + 8u * (2 * STAGES + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s2 = 0; s2 < STAGES; ++s2) {
+      mbar_init(full_bar(s2), 1);
+      mbar_init(empty_bar(s2), 1);
+    }
+    mbar_init(tfull, 1);
+    mbar_init(tempty, 128);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)),
+                 "r"(COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int kt = d / BK, nblk = (m + COLS - 1) / COLS;
+  const int xrow = kept[j] * n_v + mb * 128;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int nb = 0; nb < nblk && ok; ++nb)
+        for (int k = 0; k < kt; ++k, ++it) {
+          const int s2 = it % STAGES;
+          const uint32_t round = it / STAGES;
+          if (!mbar_wait(empty_bar(s2), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+          mbar_expect_tx(full_bar(s2), STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + s2 * A_BYTES), &tmX, k * BK, xrow, full_bar(s2));
+          tma_load_2d(smem_u32(sB + s2 * B_BYTES), &tmT, k * BK, co + nb * COLS, full_bar(s2));
+        }
+      for (int q = 1; q <= STAGES && it - q >= 0; ++q) {  // no copy left in flight (bounded)
+        const int i2 = it - q;
+        for (uint32_t w = 0; w < (1u << 22) && !mbar_try_wait(full_bar(i2 % STAGES), (i2 / STAGES) & 1u); ++w) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int nb = 0; nb < nblk && ok; ++nb) {
+        if (!mbar_wait(tempty, (nb & 1) ^ 1, abort_flag)) break;
+        fence_after();
+        for (int k = 0; k < kt; ++k, ++it) {
+          const int s2 = it % STAGES;
+          if (!mbar_wait(full_bar(s2), (it / STAGES) & 1u, abort_flag)) { ok = false; break; }
+          fence_after();
+          const uint64_t ad = smem_desc(smem_u32(sA + s2 * A_BYTES));
+          const uint64_t bd = smem_desc(smem_u32(sB + s2 * B_BYTES));
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            umma_f16(tmem_base, ad + 2 * kk, bd + 2 * kk, IDESC, (k != 0 || kk != 0) ? 1u : 0u);
+          umma_commit(empty_bar(s2));
+        }
+        if (ok) umma_commit(tfull);
+      }
+    }
+  } else {
+    // epilogue: warps 2..5 -> TMEM lane quarters 2, 3, 0, 1; thread = token row
+    const int quarter = warp & 3, r = quarter * 32 + lane;
+    const int tok = mb * 128 + r;
+    const int a = tok < n_v ? pos[(size_t)j * n_v + tok] : -1;
+    const bool want = a >= 0 && !(a % step == 0 && a / step < m);
+    float v1 = -INFINITY, v2 = -INFINITY;
+    int b1 = -1, b2 = -1;
+    bool ok = true;
+    for (int nb = 0; nb < nblk; ++nb) {
+      const int c0 = nb * COLS, nc = min(COLS, m - c0);
+      const float* inv_n = tinv + co + c0;  // 1 / ||t|| (0 for a zero target: similarity 0)
+      if (!mbar_wait(tfull, nb & 1, abort_flag)) { ok = false; break; }
+      fence_after();
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16);
+      for (int c = 0; c < nc; c += 32) {
+        uint32_t acc[32];
+        tmem_ld32(taddr + c, acc);
+        if (want) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            if (c + e < nc) {
+              const float v = __uint_as_float(acc[e]) * inv_n[c + e];
+              const int b = c0 + c + e;
+              if (v > v1) {
+                v2 = v1;
+                b2 = b1;
+                v1 = v;
+                b1 = b;
+              } else if (v > v2) {
+                v2 = v;
+                b2 = b;
+              }
+            }
+          }
+        }
+      }
+      fence_before();
+      mbar_arrive(tempty);
+    }
+    if (ok && want) cand[(size_t)j * n_v + a] = make_int2(b1, b2);
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(COLS) : "memory");
+  }
+}
+
 // ------------------------------------------------------------------------------------------ host
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -569,14 +724,15 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 2-D fp16 tensor [rows, inner] (row-major, inner contiguous), box [box_rows, 64], 128B swizzle,
 // out-of-bounds elements read as zero.
-static bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+static bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                     CUtensorMapDataType dt = CU_TENSOR_MAP_DATA_TYPE_FLOAT16) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {inner, rows};
   cuuint64_t strides[1] = {inner * 2};
   cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  return fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -833,6 +989,26 @@ static int reduce_slices(const float* part, int splits, int M, int N, int epi, v
 }
 
 }  // namespace tc
+
+int launch_merge_screen(const uint16_t* X, int N, int n_v, int d, const int* kept, const int* n_kept,
+                        const int* sel_off, const int* ctx_off, int max_ctx, const uint16_t* targets,
+                        const float* tinv, const int* pos, int2* cand, cudaStream_t st) {
+  using namespace tc;
+  CUtensorMap mx, mt;
+  if (!make_map(&mx, X, (uint64_t)d, (uint64_t)N * n_v, 128, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) ||
+      !make_map(&mt, targets, (uint64_t)d, (uint64_t)max_ctx, ms::COLS, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16))
+    return 1;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(merge_screen_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ms::SMEM) !=
+        cudaSuccess)
+      return 1;
+    attr = true;
+  }
+  merge_screen_kernel<<<dim3((n_v + 127) / 128, N), ms::THREADS, ms::SMEM, st>>>(
+      mx, mt, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, tinv, pos, cand);
+  return 0;
+}
 
 int launch_wait_timeout_check(cudaStream_t st) {
   tc::wait_timeout_check_kernel<<<1, 32, 0, st>>>();

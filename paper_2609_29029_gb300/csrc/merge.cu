@@ -5,11 +5,14 @@
 //   merge_plan_kernel     m_j (capped at the R_j unselected tokens) and their offsets ctx_off
 //   merge_targets_kernel  the unselected tokens in ascending index, the targets (every
 //                         floor(R_j / m_j)-th of them from the first) and the targets' norms
-//   merge_assign_kernel   per 64 unselected tokens x 64 targets: fp32 dot products in 32-term
-//                         chunks, a running top 2 per token; the two are recomputed as float-float
-//                         sums (good to ~2^-44) and compared as x.t1 ||t2|| vs x.t2 ||t1|| in fp64,
-//                         so the decision is the cosine argmax of the exact arithmetic (ties to
-//                         the lower target)
+//   merge_assign_kernel   (fp32 tokens) per 64 unselected tokens x 64 targets: fp32 dot products in
+//                         32-term chunks, a running top 2 per token; the two are recomputed as
+//                         float-float sums (good to ~2^-44) and compared as x.t1 / ||t1|| vs
+//                         x.t2 / ||t2|| in fp64, so the decision is the cosine argmax of the exact
+//                         arithmetic (ties to the lower target)
+//   (bf16 tokens) merge_screen_kernel (gemm_tc.cu) takes the top 2 from a tcgen05 product of
+//                         each 128-token block with the slot's target rows, and
+//                         merge_decide_kernel makes the same float-float decision between them
 //   merge_groups_kernel   the groups as member lists in ascending token index (counting sort)
 //   merge_mean_kernel     per contextual token: the fp32 sum of its members' rows in that order,
 //                         divided by the group size, stored as bf16
@@ -76,6 +79,39 @@ __device__ double ff_dot(const XT* a, const XT* b, int d, int lane) {
   return acc;
 }
 
+// a.b and a.c in one pass over a, each summed as ff_dot does.
+template <typename XT>
+__device__ double2 ff_dot2(const XT* a, const XT* b, const XT* c, int d, int lane) {
+  float hb = 0.f, lb = 0.f, hc = 0.f, lc = 0.f;
+  auto step = [](float x, float y, float& hi, float& lo) {
+    const float p = __fmul_rn(x, y);
+    const float pe = fmaf(x, y, -p);
+    const float s = __fadd_rn(hi, p);
+    const float bb = __fsub_rn(s, hi);
+    const float er = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(p, bb));
+    hi = s;
+    lo = __fadd_rn(lo, __fadd_rn(er, pe));
+  };
+  for (int k = lane * 8; k < d; k += 256) {
+    float x[8], y[8], z[8];
+    load8(a + k, x);
+    load8(b + k, y);
+    load8(c + k, z);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      step(x[e], y[e], hb, lb);
+      step(x[e], z[e], hc, lc);
+    }
+  }
+  double sb = (double)hb + (double)lb, sc = (double)hc + (double)lc;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sb += __shfl_xor_sync(0xffffffffu, sb, o);
+    sc += __shfl_xor_sync(0xffffffffu, sc, o);
+  }
+  return make_double2(sb, sc);
+}
+
 // m_j = min(budgets[j] - s_j, n_v - s_j) and its exclusive prefix sum over the kept slots.  If
 // the total exceeds max_ctx, RIFT_EBIT_CAPACITY is set and every m_j is taken as 0 (no contextual
 // row is then written or read).
@@ -120,7 +156,8 @@ __global__ void __launch_bounds__(256) merge_targets_kernel(const XT* __restrict
                                                             const int* __restrict__ sel_off,
                                                             const int* __restrict__ ctx_off, int max_ctx,
                                                             int* __restrict__ rest, int* __restrict__ ctx_target,
-                                                            double* __restrict__ tnorm) {
+                                                            double* __restrict__ tnorm, int* __restrict__ pos,
+                                                            float* __restrict__ tinv, uint16_t* __restrict__ trow) {
   __shared__ unsigned char chosen[RIFT_MAX_NV];
   __shared__ int sh[33];
   const int j = blockIdx.x;
@@ -140,8 +177,9 @@ __global__ void __launch_bounds__(256) merge_targets_kernel(const XT* __restrict
     const int k = c0 + threadIdx.x;
     const int f = (k < n_v && !chosen[k]) ? 1 : 0;
     int total;
-    const int pos = block_excl_scan(f, sh, &total);
-    if (f) rj[base + pos] = k;
+    const int at = block_excl_scan(f, sh, &total);
+    if (f) rj[base + at] = k;
+    if (pos && k < n_v) pos[(size_t)j * n_v + k] = f ? base + at : -1;
     base += total;
   }
   __syncthreads();
@@ -153,11 +191,59 @@ __global__ void __launch_bounds__(256) merge_targets_kernel(const XT* __restrict
   for (int q = warp; q < m; q += blockDim.x / 32) {
     const int t = rj[q * step];
     const double nn = ff_dot(Xt + (size_t)t * d, Xt + (size_t)t * d, d, lane);
-    if (lane == 0 && co + q < max_ctx) {
+    if (co + q >= max_ctx) continue;
+    if (lane == 0) {
       ctx_target[co + q] = t;
       tnorm[co + q] = sqrt(nn);
+      if (tinv) tinv[co + q] = nn > 0.0 ? (float)(1.0 / sqrt(nn)) : 0.f;  // a zero target has similarity 0
+    }
+    if (trow) {  // the target's row, for the tensor-core screening (bf16 tokens only)
+      const uint4* src = reinterpret_cast<const uint4*>(Xt + (size_t)t * d);
+      uint4* dst = reinterpret_cast<uint4*>(trow + (size_t)(co + q) * d);
+      for (int c = lane; c < d / 8; c += 32) dst[c] = src[c];
     }
   }
+}
+
+// Grid (blocks of 8 unselected positions, kept slot), 8 warps: for the position a of each warp
+// (not a target), the better of its two screened candidates cand[j][a] at ~fp64 accuracy:
+// x.t1 / ||t1|| vs x.t2 / ||t2|| from float-float dot products (ties to the lower target).
+template <typename XT>
+__global__ void __launch_bounds__(256) merge_decide_kernel(const XT* __restrict__ X, int n_v, int d,
+                                                           const int* __restrict__ kept,
+                                                           const int* __restrict__ n_kept,
+                                                           const int* __restrict__ sel_off,
+                                                           const int* __restrict__ ctx_off, int max_ctx,
+                                                           const int* __restrict__ rest,
+                                                           const int* __restrict__ ctx_target,
+                                                           const double* __restrict__ tnorm,
+                                                           const int2* __restrict__ cand, int* __restrict__ assign) {
+  const int j = blockIdx.y;
+  if (j >= *n_kept) return;
+  const int R = n_v - (sel_off[j + 1] - sel_off[j]);
+  const int co = ctx_off[j], m = ctx_off[j + 1] - co;
+  if (m == 0 || co + m > max_ctx) return;
+  const int step = R / m;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int a = blockIdx.x * 8 + warp;
+  if (a >= R || (a % step == 0 && a / step < m)) return;  // targets keep their own group
+  int2 c = cand[(size_t)j * n_v + a];
+  if (c.x < 0 || c.x >= m) {  // no finite similarity (a NaN token): the first target
+    if (lane == 0) atomicOr(&g_err_merge, RIFT_EBIT_NONFINITE);
+    c = make_int2(0, -1);
+  }
+  int choice = c.x;
+  if (c.y >= 0 && c.y < m) {
+    const XT* Xt = X + (size_t)kept[j] * n_v * d;
+    const int k = rest[(size_t)j * n_v + a];
+    const int t1 = ctx_target[co + c.x], t2 = ctx_target[co + c.y];
+    const double2 dd = ff_dot2(Xt + (size_t)k * d, Xt + (size_t)t1 * d, Xt + (size_t)t2 * d, d, lane);
+    const double d1 = dd.x, d2 = dd.y;
+    const double n1 = tnorm[co + c.x], n2 = tnorm[co + c.y];
+    const double s1 = n1 > 0.0 ? d1 / n1 : 0.0, s2 = n2 > 0.0 ? d2 / n2 : 0.0;
+    if (s2 > s1 || (s2 == s1 && c.y < c.x)) choice = c.y;
+  }
+  if (lane == 0) assign[(size_t)j * n_v + a] = choice;
 }
 
 // Grid (kept slot, block of TB unselected tokens).  assign[j][a] = target index of rest[a].
@@ -293,7 +379,7 @@ __global__ void __launch_bounds__(256) merge_assign_kernel(const XT* __restrict_
 
 // One CTA per kept slot: the slot's groups as member lists, ascending token index within each
 // group (targets at their own index): gstart[j][q] .. gstart[j][q+1] in memb[j].  A counting sort
-// whose placement pass runs in token order on one thread.
+// whose placement pass runs in token order on one warp.
 __global__ void __launch_bounds__(256) merge_groups_kernel(int n_v, const int* __restrict__ n_kept,
                                                            const int* __restrict__ sel_off,
                                                            const int* __restrict__ ctx_off, int max_ctx,
@@ -309,7 +395,11 @@ __global__ void __launch_bounds__(256) merge_groups_kernel(int n_v, const int* _
   const int step = R / m;
   const int* rj = rest + (size_t)j * n_v;
   const int* aj = assign + (size_t)j * n_v;
-  auto group = [&](int a) { return (a % step == 0 && a / step < m) ? a / step : aj[a]; };
+  auto group = [&](int a) {
+    if (a % step == 0 && a / step < m) return a / step;
+    const int g = aj[a];
+    return (g >= 0 && g < m) ? g : 0;  // an unassigned token (no finite similarity) joins the first group
+  };
   for (int q = threadIdx.x; q <= m; q += blockDim.x) cnt[q] = 0;
   __syncthreads();
   for (int a = threadIdx.x; a < R; a += blockDim.x) atomicAdd(&cnt[group(a)], 1);
@@ -324,8 +414,22 @@ __global__ void __launch_bounds__(256) merge_groups_kernel(int n_v, const int* _
       acc += c;
     }
     gs[m] = acc;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    // placement in token order by one warp, 32 tokens at a time: a token's slot is its group's
+    // next free one plus the number of lower lanes of the same group
+    const int lane = threadIdx.x;
     int* mj = memb + (size_t)j * n_v;
-    for (int a = 0; a < R; ++a) mj[cnt[group(a)]++] = rj[a];
+    for (int a0 = 0; a0 < R; a0 += 32) {
+      const int a = a0 + lane;
+      const int g = a < R ? group(a) : -1 - lane;  // idle lanes match no one
+      const unsigned same = __match_any_sync(0xffffffffu, g);
+      if (a < R) mj[cnt[g] + __popc(same & ((1u << lane) - 1u))] = rj[a];
+      __syncwarp();
+      if (a < R && (same >> lane) == 1u) cnt[g] += __popc(same);  // the group's highest lane
+      __syncwarp();
+    }
   }
 }
 
@@ -391,6 +495,9 @@ MergeLayout merge_layout(int N, int n_v) {
   L.tnorm_off = take((size_t)N * n_v * sizeof(double));
   L.memb_off = take((size_t)N * n_v * sizeof(int));
   L.gstart_off = take((size_t)N * (n_v + 1) * sizeof(int));
+  L.pos_off = take((size_t)N * n_v * sizeof(int));
+  L.tinv_off = take((size_t)N * n_v * sizeof(float));  // at most n_v - 1 targets per slot
+  L.cand_off = take((size_t)N * n_v * sizeof(int2));
   L.total = off;
   return L;
 }
@@ -405,26 +512,31 @@ int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
   double* tnorm = reinterpret_cast<double*>(ws + L.tnorm_off);
   int* memb = reinterpret_cast<int*>(ws + L.memb_off);
   int* gstart = reinterpret_cast<int*>(ws + L.gstart_off);
+  int* pos = reinterpret_cast<int*>(ws + L.pos_off);
+  float* tinv = reinterpret_cast<float*>(ws + L.tinv_off);
+  int2* cand = reinterpret_cast<int2*>(ws + L.cand_off);
   merge_plan_kernel<<<1, 1024, 0, st>>>(n_kept, budgets, sel_off, N, n_v, max_ctx, ctx_off);
   const dim3 ga((n_v + TB - 1) / TB, N), gm(N, 32);
   const size_t ab_bytes = 2 * (size_t)KC * (TB + 4) * sizeof(float);
   if (xdt == RIFT_BF16) {
+    // bf16 tokens: the target rows go to ctx (overwritten by the means at the end), the top two
+    // of every token come from the tensor cores, the choice between them from float-float sums
     const uint16_t* x = static_cast<const uint16_t*>(X);
     merge_targets_kernel<uint16_t><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
-                                                      ctx_target, tnorm);
-    static bool attr16 = false;
-    if (!attr16) {
-      cudaFuncSetAttribute(merge_assign_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ab_bytes);
-      attr16 = true;
-    }
-    merge_assign_kernel<uint16_t><<<ga, 256, ab_bytes, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
-                                                      ctx_target, tnorm, assign);
+                                                      ctx_target, tnorm, pos, tinv, ctx);
+    if (max_ctx > 0 &&
+        launch_merge_screen(x, N, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, ctx, tinv, pos, cand, st))
+      return -1;
+    merge_decide_kernel<uint16_t><<<dim3((n_v + 7) / 8, N), 256, 0, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off,
+                                                                        max_ctx, rest, ctx_target, tnorm, cand,
+                                                                        assign);
     merge_groups_kernel<<<N, 256, 0, st>>>(n_v, n_kept, sel_off, ctx_off, max_ctx, rest, assign, memb, gstart);
     merge_mean_kernel<uint16_t><<<gm, MT, 0, st>>>(x, n_v, d, kept, n_kept, ctx_off, max_ctx, memb, gstart, ctx);
+    return max_ctx > 0 ? 6 : 5;
   } else {
     const float* x = static_cast<const float*>(X);
     merge_targets_kernel<float><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
-                                                   ctx_target, tnorm);
+                                                   ctx_target, tnorm, nullptr, nullptr, nullptr);
     static bool attr32 = false;
     if (!attr32) {
       cudaFuncSetAttribute(merge_assign_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ab_bytes);

@@ -271,6 +271,7 @@ rift_status rift_merge_contextual(const void* X, rift_dtype xdt, int N, int n_v,
   prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
   const int nk = launch_merge(X, xdt, N, n_v, d, kept, n_kept, budgets, sel, sel_off, static_cast<uint16_t*>(ctx),
                               max_ctx, ctx_off, ctx_target, static_cast<char*>(ws), static_cast<cudaStream_t>(stream));
+  if (nk < 0) return RIFT_ERR_CUDA;
   prof_end(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream), nk);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;

@@ -48,12 +48,12 @@ int launch_features(const void* X, rift_dtype xdt, int N, int n_v, int d, int g,
 
 // ---- merge.cu ----
 struct MergeLayout {
-  size_t rest_off, assign_off, tnorm_off, memb_off, gstart_off, total;
+  size_t rest_off, assign_off, tnorm_off, memb_off, gstart_off, pos_off, tinv_off, cand_off, total;
 };
 #define RIFT_MERGE_MAX_D 8192
 MergeLayout merge_layout(int N, int n_v);
 unsigned int read_clear_err_merge();
-// Returns the number of kernels launched.
+// Returns the number of kernels launched, or -1 if a launch could not be set up.
 int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int* kept, const int* n_kept,
                  const int* budgets, const int* sel, const int* sel_off, uint16_t* ctx, int max_ctx, int* ctx_off,
                  int* ctx_target, char* ws, cudaStream_t st);
@@ -124,6 +124,13 @@ int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
                    cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0, bool pdl = false);
 int launch_wait_timeout_check(cudaStream_t st);
+// Merge screening on the tensor cores (bf16 tokens): per kept slot and 128-token block, the two
+// best merge targets (by x.t / ||t||) of every unselected non-target token.  targets: bf16
+// [max_ctx, d] target rows; tinv [max_ctx] = 1 / ||t||; pos [N, n_v] = position of each token
+// among the slot's unselected ones (-1 if selected); cand [N, n_v] out, indexed by that position.
+int launch_merge_screen(const uint16_t* X, int N, int n_v, int d, const int* kept, const int* n_kept,
+                        const int* sel_off, const int* ctx_off, int max_ctx, const uint16_t* targets,
+                        const float* tinv, const int* pos, int2* cand, cudaStream_t st);
 
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].
