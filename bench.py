@@ -212,6 +212,10 @@ def oracle_sample(wl, sc, n_tiles: int, n_layers: int, budget: int, device):
     torch.set_num_threads(len(os.sched_getaffinity(0)))
     cores = torch.get_num_threads()
     dec = wl.decoder
+    # a sample never exceeds the workload: small scenes and decoders are taken whole
+    n_tiles = max(1, min(n_tiles, wl.scene.N))
+    n_layers = max(1, min(n_layers, dec.n_layers))
+    budget = max(0, min(budget, wl.scene.n_v))
     Xs = sc.X[:n_tiles].cpu()
     embed = sc.embed.cpu()
     t0 = time.perf_counter()

@@ -58,3 +58,17 @@ def test_reference_arm_prints_the_contract_line():
     assert line["impl"] == "reference" and line["metric"] == "retained prefill tokens/s"
     assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+
+
+def test_cpu_baseline_sample_is_clamped_to_a_small_workload():
+    """The CPU-baseline sample asks for 8 tiles and 4 layers; the tiny scene has 4 tiles and a
+    2-layer decoder, so the sample takes the whole scene and decoder instead of indexing past them."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    from synth import workloads as W
+    wl = W.TINY
+    sc = W.make_scene(wl.scene, wl.decoder.vocab)
+    t_tile, t_tok, cores, text = bench.oracle_sample(wl, sc, 8, 4, 10_000, torch.device("cpu"))
+    assert t_tile > 0 and t_tok > 0 and cores >= 1
+    assert "on 4 of 4 tiles" in text and "2 of 2 layers" in text
+    assert f"one {wl.scene.S + wl.scene.n_v + wl.scene.Q}-token sequence" in text
