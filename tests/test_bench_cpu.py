@@ -72,3 +72,15 @@ def test_cpu_baseline_sample_is_clamped_to_a_small_workload():
     assert t_tile > 0 and t_tok > 0 and cores >= 1
     assert "on 4 of 4 tiles" in text and "2 of 2 layers" in text
     assert f"one {wl.scene.S + wl.scene.n_v + wl.scene.Q}-token sequence" in text
+
+
+def test_l2_note_and_traffic_belong_to_the_workload():
+    """A workload whose inputs fit in L2 says it is flushed between steps, and the GEMM's DRAM
+    traffic is reported only for the workload its ncu capture was taken on."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    assert bench.l2_note(2 * 10**9, 13 * 10**9, False).startswith("inputs larger than L2")
+    assert "flushed between timed steps" in bench.l2_note(2 * 10**6, 3 * 10**6, True)
+    assert bench.gemm_traffic("tiny") is None
+    t = bench.gemm_traffic(bench.PROFILED_WORKLOAD)
+    assert t is None or t > 0
