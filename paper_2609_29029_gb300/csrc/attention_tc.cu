@@ -224,7 +224,7 @@ template <int HD, int KB>
 __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
                    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int S_pre,
-                   const int* __restrict__ cu, const int2* __restrict__ sched, int n_entries, int H, float scale_log2,
+                   const int4* __restrict__ sched, int n_entries, int H, float scale_log2,
                    uint16_t* __restrict__ out) {
   using CF = Cfg<HD, KB>;
   constexpr int NST = CF::NST, NO = CF::NO, NC = KB / 32;  // NC: 32-key chunks per block
@@ -283,21 +283,22 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
   const int np = (S_pre + KB - 1) / KB;  // prefix blocks ahead of every sequence's own
 
   // An item's sequence start, length, first row, head and number of KB-key blocks (causal:
-  // keys up to the block's last valid row).  Every role reads the next item's entry while it
-  // works on the current one.
+  // keys up to the block's last valid row).  Every role fetches the next item's schedule entry
+  // (one 16-byte load, no branch on it) while it works on the current one, and decodes it only
+  // when that item starts, so the load's latency is hidden behind a whole item.
   struct Item {
     int seq0, L, q0, h, nkv;
   };
-  auto load_item = [&](int item) -> Item {
-    Item it{0, 0, 0, 0, 0};
-    if (item >= n_items) return it;
-    const int2 e = sched[item / H];
+  auto fetch_item = [&](int item) -> int4 {
+    return item < n_items ? sched[item / H] : make_int4(0, 0, 0, 0);
+  };
+  auto decode_item = [&](const int4& e, int item) -> Item {
+    Item it;
     it.h = item % H;
-    if (e.x < 0) return it;
-    it.seq0 = cu[e.x];
-    it.L = cu[e.x + 1] - it.seq0;
-    it.q0 = e.y;
-    it.nkv = np + (min(it.L, it.q0 + BQ) - 1) / KB + 1;
+    it.seq0 = e.x;
+    it.L = e.y;
+    it.q0 = e.z;
+    it.nkv = (item < n_items && e.y > 0) ? np + (min(e.y, e.z + BQ) - 1) / KB + 1 : 0;
     return it;
   };
   // Counters shared by every role: g counts KB-key blocks, t counts items of this CTA.  Block g
@@ -309,10 +310,10 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
       // ---------------- TMA producers: lane 0 K tiles; lane 1 Q and V tiles
       uint32_t g = 0, t = 0;
       bool ok = true;
-      Item nxt = load_item(blockIdx.x);
+      int4 nxt = fetch_item(blockIdx.x);
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        const Item cur = nxt;
-        nxt = load_item(item + gridDim.x);
+        const Item cur = decode_item(nxt, item);
+        nxt = fetch_item(item + gridDim.x);
         if (cur.nkv == 0) continue;
         if (lane == 1) {
           if (!mbar_wait(Q_EMPTY, (t & 1u) ^ 1u, abort_flag)) { ok = false; break; }
@@ -362,10 +363,10 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
         umma_commit(BAR(K_EMPTY, st));
         return true;
       };
-      Item nxt = load_item(blockIdx.x);
+      int4 nxt = fetch_item(blockIdx.x);
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        const int nkv = nxt.nkv;
-        nxt = load_item(item + gridDim.x);
+        const int nkv = decode_item(nxt, item).nkv;
+        nxt = fetch_item(item + gridDim.x);
         if (nkv == 0) continue;
         const int ob = t % NO;
         if (!mbar_wait(Q_FULL, t & 1u, abort_flag)) break;
@@ -404,10 +405,10 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     uint32_t g = 0, t = 0;
     bool ok = true;
-    Item nxt = load_item(blockIdx.x);
+    int4 nxt = fetch_item(blockIdx.x);
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-      const Item cur = nxt;
-      nxt = load_item(item + gridDim.x);
+      const Item cur = decode_item(nxt, item);
+      nxt = fetch_item(item + gridDim.x);
       const int L = cur.L, q0 = cur.q0, nkv = cur.nkv;
       if (nkv == 0) continue;
       const int ob = t % NO;
@@ -536,23 +537,29 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
   }
 }
 
-// One entry per 128-row q-block, (sequence, first row); the rest (-1, 0).  Longer sequences'
-// entries are not reordered: items are interleaved across CTAs by the persistent loop.
+// One entry per 128-row q-block: (first row of its sequence in the packed batch, sequence length,
+// first row of the block within the sequence, 0); the rest (0, 0, 0, 0), which the kernel skips.
+// Longer sequences' entries are not reordered: items are interleaved across CTAs by the
+// persistent loop.
 __global__ void __launch_bounds__(1024) schedule128_kernel(const int* __restrict__ cu, int n_seq,
-                                                           int2* __restrict__ sched, int n_max) {
+                                                           int4* __restrict__ sched, int n_max) {
   __shared__ int sh[33];
   int base = 0;
   for (int c0 = 0; c0 < n_seq; c0 += blockDim.x) {
     const int s = c0 + threadIdx.x;
-    int nb = 0;
-    if (s < n_seq) nb = (cu[s + 1] - cu[s] + BQ - 1) / BQ;
+    int nb = 0, s0 = 0, len = 0;
+    if (s < n_seq) {
+      s0 = cu[s];
+      len = cu[s + 1] - s0;
+      nb = (len + BQ - 1) / BQ;
+    }
     int total;
     int off = block_excl_scan(nb, sh, &total);
     for (int b = 0; b < nb; ++b)
-      if (base + off + b < n_max) sched[base + off + b] = make_int2(s, b * BQ);
+      if (base + off + b < n_max) sched[base + off + b] = make_int4(s0, len, b * BQ, 0);
     base += total;
   }
-  for (int i = base + threadIdx.x; i < n_max; i += blockDim.x) sched[i] = make_int2(-1, 0);
+  for (int i = base + threadIdx.x; i < n_max; i += blockDim.x) sched[i] = make_int4(0, 0, 0, 0);
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -582,7 +589,7 @@ static int sm_count() {
 }  // namespace fa
 
 // q-block schedule of the tcgen05 attention (one entry per 128 rows of a sequence)
-void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st) {
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, int4* sched, int n_sched_max, cudaStream_t st) {
   fa::schedule128_kernel<<<1, 1024, 0, st>>>(cu_seqlens, n_seq, sched, n_sched_max);
 }
 
@@ -595,8 +602,8 @@ constexpr int kAttnKB = 64;
 
 template <int HD, int KB>
 int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& mpk, const CUtensorMap& mpv,
-                 int S_pre, const int* cu_seqlens, const int2* sched, int n_sched_max, int n_heads, float scale_log2,
-                 void* out, cudaStream_t st) {
+                 int S_pre, const int4* sched, int n_sched_max, int n_heads, float scale_log2, void* out,
+                 cudaStream_t st) {
   using namespace fa;
   using CF = Cfg<HD, KB>;
   static bool attr = false;
@@ -609,8 +616,8 @@ int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMa
   const int items = n_sched_max * n_heads;
   const int slots = CF::CTAS * sm_count();
   const int grid = items < slots ? items : slots;
-  attn_tc_kernel<HD, KB><<<grid, THREADS, CF::SMEM, st>>>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max,
-                                                          n_heads, scale_log2, static_cast<uint16_t*>(out));
+  attn_tc_kernel<HD, KB><<<grid, THREADS, CF::SMEM, st>>>(mq, mkv, mpk, mpv, S_pre, sched, n_sched_max, n_heads,
+                                                          scale_log2, static_cast<uint16_t*>(out));
   return 0;
 }
 
@@ -632,10 +639,11 @@ bool make_attn_map(CUtensorMap* map, const void* base, uint64_t cols, uint64_t r
 // qkv fp16 [T, 3 H hd] (q | k | v, heads contiguous), out fp16 [T, H hd]; optional prefix keys and
 // values fp16 [S_pre, H hd] attended to by every sequence before its own rows.
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
-                     const int2* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k,
+                     const int4* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k,
                      const void* prefix_v, int S_pre) {
   using namespace fa;
   (void)n_seq;
+  (void)cu_seqlens;  // the schedule entries carry the sequence bounds
   if (T <= 0) return 0;
   if (head_dim != 64 && head_dim != 128) return 1;
   if (S_pre > 0 && (!prefix_k || !prefix_v)) return 1;
@@ -651,10 +659,8 @@ int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, i
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
   if (head_dim == 128)
-    return launch_shape<128, kAttnKB>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max, n_heads, scale_log2,
-                                      out, st);
-  return launch_shape<64, kAttnKB>(mq, mkv, mpk, mpv, S_pre, cu_seqlens, sched, n_sched_max, n_heads, scale_log2, out,
-                                   st);
+    return launch_shape<128, kAttnKB>(mq, mkv, mpk, mpv, S_pre, sched, n_sched_max, n_heads, scale_log2, out, st);
+  return launch_shape<64, kAttnKB>(mq, mkv, mpk, mpv, S_pre, sched, n_sched_max, n_heads, scale_log2, out, st);
 }
 
 }  // namespace rift

@@ -141,7 +141,7 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   L.act_off = take(T * m.ffn * 2);
   L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
   L.max_qblocks = attention_max_qblocks(max_T, max_seqs);
-  L.sched_off = take((size_t)L.max_qblocks * sizeof(int2));
+  L.sched_off = take((size_t)L.max_qblocks * sizeof(int4));
   L.last32_off = take((size_t)max_seqs * m.d * 4);
   L.last16_off = take((size_t)max_seqs * m.d * 2);
   L.total = off;
@@ -181,7 +181,7 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   uint16_t* att = reinterpret_cast<uint16_t*>(ws + L.attn_off);
   uint16_t* act = reinterpret_cast<uint16_t*>(ws + L.act_off);
   float2* rope = reinterpret_cast<float2*>(ws + L.rope_off);
-  int2* sched = reinterpret_cast<int2*>(ws + L.sched_off);
+  int4* sched = reinterpret_cast<int4*>(ws + L.sched_off);
   const int d = m.d, half = m.head_dim / 2;
 
   prof_begin(RIFT_PROF_ROPE, st);

@@ -392,7 +392,7 @@ rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int e
 
 size_t rift_attention_workspace_bytes(int max_T, int max_seqs) {
   if (max_T < 0 || max_seqs < 0) return 0;
-  return (size_t)attention_max_qblocks(max_T, max_seqs) * sizeof(int2);
+  return (size_t)attention_max_qblocks(max_T, max_seqs) * sizeof(int4);
 }
 
 rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
@@ -405,7 +405,7 @@ rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens,
   if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
   if (T == 0) return RIFT_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int2* sched = static_cast<int2*>(ws);
+  int4* sched = static_cast<int4*>(ws);
   const int n_max = attention_max_qblocks(T, n_seq);
   prof_begin(RIFT_PROF_ATTN, st);
   launch_attention_schedule(cu_seqlens, n_seq, sched, n_max, st);

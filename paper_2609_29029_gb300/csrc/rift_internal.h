@@ -135,11 +135,11 @@ int launch_merge_screen(const uint16_t* X, int N, int n_v, int d, const int* kep
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].
 int attention_max_qblocks(int max_T, int max_seqs);
-void launch_attention_schedule(const int* cu_seqlens, int n_seq, int2* sched, int n_sched_max, cudaStream_t st);
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, int4* sched, int n_sched_max, cudaStream_t st);
 // prefix_k, prefix_v (optional): fp16 [S_pre, d] keys (after RoPE) and values of a prefix that every
 // sequence attends to before its own rows.
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,
-                     const int2* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k = nullptr,
+                     const int4* sched, int n_sched_max, void* out, cudaStream_t st, const void* prefix_k = nullptr,
                      const void* prefix_v = nullptr, int S_pre = 0);
 unsigned int read_clear_err_attn();
 
