@@ -51,7 +51,7 @@ typedef enum {
   RIFT_ERR_NONFINITE = 3,   /* a NaN or Inf score reached a decision */
   RIFT_ERR_CUDA = 4,        /* a CUDA runtime call failed */
   RIFT_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
-  RIFT_ERR_UNSUPPORTED = 6, /* a valid request this build does not implement */
+  RIFT_ERR_UNSUPPORTED = 6, /* a valid request the library does not implement */
   RIFT_ERR_BAD_ID = 7       /* a token or tile id outside its range */
 } rift_status;
 
@@ -310,7 +310,7 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
                                 const int* positions, void* kv_out, float* last_logits,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
 
-/* ---- Prefill over a shared system prompt (SURVEY-style extension of Section 2.1's prefill:
+/* ---- Prefill over a shared system prompt (an extension of Section 2.1's prefill, not in the paper:
  * the S system-prompt rows open every per-tile sequence at positions 0..S-1, so their hidden
  * states and cache are the same in every sequence) ----
  * The prompt is prefilled once and every sequence's remaining rows (its b_i vision tokens and
