@@ -588,6 +588,14 @@ int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids
     normalize_rows_kernel<<<1 + M, 256, 0, st>>>(t, B, d);
     return 2;
   }
+  // two fp32 rows of d in shared memory: 64 KB at the widest d (8192), past the 48 KB default
+  static bool smem_attr = false;
+  if (!smem_attr) {
+    if (cudaFuncSetAttribute(query_prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(2 * 8192 * sizeof(float))) != cudaSuccess)
+      return 0;  // the launch check of the caller reports the failure
+    smem_attr = true;
+  }
   query_prep_kernel<<<1, 256, 2 * d * sizeof(float), st>>>(
       static_cast<const uint16_t*>(embed), vocab, d, phrase_ids, n_tmpl, n_phrase, bg_ids, M, t, B);
   return 1;
