@@ -19,6 +19,8 @@
 // fp16 rather than bf16 operands: after 32 layers the bf16 rounding of the GEMM inputs alone
 // moves the final hidden states by about 3% of their largest magnitude; fp16 (3 more mantissa
 // bits, same tensor-core rate, LLaVA-1.5-7B's checkpoint dtype) keeps the whole path near 0.5%.
+#include <type_traits>
+
 #include "rift_internal.h"
 
 namespace rift {
@@ -33,12 +35,13 @@ unsigned int read_clear_err_prefill() {
 }
 
 constexpr int NORM_THREADS = 256;
-constexpr int NORM_MAXV = 8;  // float4 per thread: d <= 8192
 
 // y = h / sqrt(mean(h^2) + eps) * g, one CTA per row.  IN_BF16: h is the bf16 packed input,
 // which is also widened into the fp32 residual stream h32.  OUT_F16: y in fp16 (the GEMM
-// operand); otherwise bf16 (the final hidden states).
-template <bool IN_BF16, bool OUT_F16>
+// operand); otherwise bf16 (the final hidden states).  VPT: float4 per thread, the fewest that
+// cover d (4 at d = 4096, 8 at the widest d = 8192), so the row held in registers is no larger
+// than the row: fewer registers, more CTAs per SM and more bytes in flight.
+template <bool IN_BF16, bool OUT_F16, int VPT>
 __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __restrict__ in,
                                                                float* __restrict__ h32,
                                                                const uint16_t* __restrict__ gain,
@@ -47,10 +50,10 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __res
   __shared__ float red[32];
   const size_t row = blockIdx.x;
   const int nv = d / 4;
-  float4 v[NORM_MAXV];
+  float4 v[VPT];
   float ss = 0.f;
 #pragma unroll
-  for (int q = 0; q < NORM_MAXV; ++q) {
+  for (int q = 0; q < VPT; ++q) {
     const int c = threadIdx.x + q * NORM_THREADS;
     if (c < nv) {
       if constexpr (IN_BF16) {
@@ -66,7 +69,7 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __res
   }
   const float inv = rsqrtf(block_sum(ss, red) / (float)d + eps);
 #pragma unroll
-  for (int q = 0; q < NORM_MAXV; ++q) {
+  for (int q = 0; q < VPT; ++q) {
     const int c = threadIdx.x + q * NORM_THREADS;
     if (c < nv) {
       uint2 gr = reinterpret_cast<const uint2*>(gain)[c];
@@ -161,12 +164,20 @@ static void norm_launch(int kind, int T, const void* in, float* h32, const void*
                         float eps, cudaStream_t st) {
   prof_begin(RIFT_PROF_NORM, st);
   const uint16_t* g = static_cast<const uint16_t*>(gain);
-  if (kind == 0)
-    rmsnorm_kernel<true, true><<<T, NORM_THREADS, 0, st>>>(in, h32, g, out, d, eps);
-  else if (kind == 1)
-    rmsnorm_kernel<false, true><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
-  else
-    rmsnorm_kernel<false, false><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
+  const int per_thread = (d / 4 + NORM_THREADS - 1) / NORM_THREADS;  // d <= 8192: at most 8
+  auto go = [&](auto vpt) {
+    constexpr int V = decltype(vpt)::value;
+    if (kind == 0)
+      rmsnorm_kernel<true, true, V><<<T, NORM_THREADS, 0, st>>>(in, h32, g, out, d, eps);
+    else if (kind == 1)
+      rmsnorm_kernel<false, true, V><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
+    else
+      rmsnorm_kernel<false, false, V><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
+  };
+  if (per_thread <= 1) go(std::integral_constant<int, 1>{});
+  else if (per_thread <= 2) go(std::integral_constant<int, 2>{});
+  else if (per_thread <= 4) go(std::integral_constant<int, 4>{});
+  else go(std::integral_constant<int, 8>{});
   prof_end(RIFT_PROF_NORM, st, 1);
 }
 
