@@ -606,13 +606,8 @@ int launch_shape(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMa
                  cudaStream_t st) {
   using namespace fa;
   using CF = Cfg<HD, KB>;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(attn_tc_kernel<HD, KB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)CF::SMEM) !=
-        cudaSuccess)
-      return 1;
-    attr = true;
-  }
+  static std::atomic<unsigned long long> smem_raised{0};
+  if (raise_smem_limit(smem_raised, attn_tc_kernel<HD, KB>, (int)CF::SMEM) != cudaSuccess) return 1;
   const int items = n_sched_max * n_heads;
   const int slots = CF::CTAS * sm_count();
   const int grid = items < slots ? items : slots;

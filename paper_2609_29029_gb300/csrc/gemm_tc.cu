@@ -753,11 +753,8 @@ template <int EPI, int BN_ = BN, int STAGES_ = STAGES>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
                   cudaStream_t st, int splits = 1, bool pdl = false, int a_const = 0) {
   constexpr size_t smem = (size_t)STAGES_ * (A_BYTES + BN_ * BK * 2) + 1024 + 256;
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(gemm_tc_kernel<EPI, BN_, STAGES_>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    attr = true;
-  }
+  static std::atomic<unsigned long long> smem_raised{0};
+  if (raise_smem_limit(smem_raised, gemm_tc_kernel<EPI, BN_, STAGES_>, (int)smem) != cudaSuccess) return 1;
   const int units = ((M + BM - 1) / BM) * ((N + BN_ - 1) / BN_) * splits;
   const int grid = units < sm_count() ? units : sm_count();
   // Band height: as many M-tiles as keep the band's A rows within ~48 MB of L2 (8..64), so each
@@ -787,17 +784,27 @@ static int launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
   cfg.dynamicSmemBytes = smem;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  static int max_clusters = -1;
-  if (max_clusters < 0) {
+  // per device: the raised shared-memory limit, and how many 2-CTA clusters fit at once (+1; 0 = not
+  // asked yet)
+  static std::atomic<unsigned long long> smem_raised{0};
+  static std::atomic<int> clusters_plus1[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  int known = (dev >= 0 && dev < 64) ? clusters_plus1[dev].load(std::memory_order_acquire) : 0;
+  if (known == 0) {
     int n = 0;
     cfg.gridDim = dim3(2, 1, 1);
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+    if (raise_smem_limit(smem_raised, kern, (int)smem) != cudaSuccess ||
         cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
       cudaGetLastError();
       n = 0;
     }
-    max_clusters = n;
+    known = n + 1;
+    if (dev >= 0 && dev < 64) clusters_plus1[dev].store(known, std::memory_order_release);
+  } else if (raise_smem_limit(smem_raised, kern, (int)smem) != cudaSuccess) {
+    return 1;
   }
+  const int max_clusters = known - 1;
   if (max_clusters <= 0) return -1;
   const int units = ((M + 2 * BM - 1) / (2 * BM)) * ((N + BN - 1) / BN);
   const int clusters = units < max_clusters ? units : max_clusters;
@@ -998,13 +1005,8 @@ int launch_merge_screen(const uint16_t* X, int N, int n_v, int d, const int* kep
   if (!make_map(&mx, X, (uint64_t)d, (uint64_t)N * n_v, 128, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) ||
       !make_map(&mt, targets, (uint64_t)d, (uint64_t)max_ctx, ms::COLS, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16))
     return 1;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(merge_screen_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ms::SMEM) !=
-        cudaSuccess)
-      return 1;
-    attr = true;
-  }
+  static std::atomic<unsigned long long> smem_raised{0};
+  if (raise_smem_limit(smem_raised, merge_screen_kernel, (int)ms::SMEM) != cudaSuccess) return 1;
   merge_screen_kernel<<<dim3((n_v + 127) / 128, N), ms::THREADS, ms::SMEM, st>>>(
       mx, mt, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, tinv, pos, cand);
   return 0;

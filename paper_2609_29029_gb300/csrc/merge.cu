@@ -537,11 +537,8 @@ int launch_merge(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
     const float* x = static_cast<const float*>(X);
     merge_targets_kernel<float><<<N, 256, 0, st>>>(x, n_v, d, kept, n_kept, sel, sel_off, ctx_off, max_ctx, rest,
                                                    ctx_target, tnorm, nullptr, nullptr, nullptr);
-    static bool attr32 = false;
-    if (!attr32) {
-      cudaFuncSetAttribute(merge_assign_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ab_bytes);
-      attr32 = true;
-    }
+    static std::atomic<unsigned long long> smem_raised{0};
+    if (raise_smem_limit(smem_raised, merge_assign_kernel<float>, (int)ab_bytes) != cudaSuccess) return -1;
     merge_assign_kernel<float><<<ga, 256, ab_bytes, st>>>(x, n_v, d, kept, n_kept, sel_off, ctx_off, max_ctx, rest,
                                                    ctx_target, tnorm, assign);
     merge_groups_kernel<<<N, 256, 0, st>>>(n_v, n_kept, sel_off, ctx_off, max_ctx, rest, assign, memb, gstart);

@@ -228,11 +228,9 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
   dim3 grid(N, (max_L + PK_ROWS - 1) / PK_ROWS);
   if (xdt == RIFT_BF16) {
     const size_t smem = (size_t)PKB_SLOTS * d * 2;
-    static bool attr = false;
-    if (!attr) {
-      cudaFuncSetAttribute(pack_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, PKB_SLOTS * 8192 * 2);
-      attr = true;
-    }
+    static std::atomic<unsigned long long> smem_raised{0};
+    if (raise_smem_limit(smem_raised, pack_bulk_kernel, PKB_SLOTS * 8192 * 2) != cudaSuccess)
+      return;  // the error stays pending for the caller's launch check
     dim3 gb(N, (max_L + PKB_ROWS - 1) / PKB_ROWS);
     pack_bulk_kernel<<<gb, 64, smem, st>>>(
         static_cast<const uint16_t*>(X), N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q,

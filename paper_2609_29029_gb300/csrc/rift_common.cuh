@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "rift.h"
 
 // Device error bits, OR-ed into a per-translation-unit flag and collected by rift_sync_status.
@@ -27,6 +29,22 @@
 #define RIFT_LAUNCH_CHECK() RIFT_CUDA_TRY(cudaGetLastError())
 
 namespace rift {
+
+// Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current device, once per
+// device: a function's attributes belong to each device's context, so a process that drives
+// several GPUs needs the call on every one of them.  `done` is the call site's record of the
+// devices already raised (a device id of 64 or more is raised on every call).
+template <typename K>
+inline cudaError_t raise_smem_limit(std::atomic<unsigned long long>& done, K* kernel, int bytes) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0ull;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
+}
 
 // Programmatic dependent launch.  A kernel launched with `pdl` set (launch_ex) may begin while
 // the kernel before it in the stream is still running: each of its threads calls pdl_wait()

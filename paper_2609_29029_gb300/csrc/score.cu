@@ -589,13 +589,9 @@ int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids
     return 2;
   }
   // two fp32 rows of d in shared memory: 64 KB at the widest d (8192), past the 48 KB default
-  static bool smem_attr = false;
-  if (!smem_attr) {
-    if (cudaFuncSetAttribute(query_prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)(2 * 8192 * sizeof(float))) != cudaSuccess)
-      return 0;  // the launch check of the caller reports the failure
-    smem_attr = true;
-  }
+  static std::atomic<unsigned long long> smem_raised{0};
+  if (raise_smem_limit(smem_raised, query_prep_kernel, (int)(2 * 8192 * sizeof(float))) != cudaSuccess)
+    return 0;  // the launch check of the caller reports the failure
   query_prep_kernel<<<1, 256, 2 * d * sizeof(float), st>>>(
       static_cast<const uint16_t*>(embed), vocab, d, phrase_ids, n_tmpl, n_phrase, bg_ids, M, t, B);
   return 1;
