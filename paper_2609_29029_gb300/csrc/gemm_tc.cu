@@ -891,20 +891,24 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits,
 // The residual add of a split-K product fused with the RMSNorm that follows it: one CTA per row,
 // h[row] += sum of the slices (in slice order), then out[row] = fp16(h / sqrt(mean(h^2) + eps) g)
 // with the bf16 gain g (the arithmetic of the standalone RMSNorm kernel).  N % 4 == 0, N <= 8192.
-__global__ void __launch_bounds__(256) splitk_resid_norm_kernel(const float* __restrict__ part, int splits, int M,
-                                                                int N, float* __restrict__ h32,
-                                                                const uint16_t* __restrict__ gain, float eps,
-                                                                uint16_t* __restrict__ out) {
+// The rows are few (one per sequence in a decode step), so the kernel is latency-bound: a CTA has
+// up to 1024 threads and each holds VPT float4 columns of its row (1 at N = 4096), so that all of
+// a thread's loads (its columns of h and of every slice) are independent and issue together.
+template <int VPT>
+__global__ void __launch_bounds__(1024) splitk_resid_norm_kernel(const float* __restrict__ part, int splits, int M,
+                                                                 int N, float* __restrict__ h32,
+                                                                 const uint16_t* __restrict__ gain, float eps,
+                                                                 uint16_t* __restrict__ out) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
   const size_t row = blockIdx.x, stride = (size_t)M * N;
   const int nv = N / 4;
-  float4 v[8];
+  float4 v[VPT];
   float ss = 0.f;
 #pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    const int c = threadIdx.x + q * 256;
+  for (int q = 0; q < VPT; ++q) {
+    const int c = threadIdx.x + q * blockDim.x;
     if (c < nv) {
       float4 a = reinterpret_cast<const float4*>(h32 + row * N)[c];
       const float4* p = reinterpret_cast<const float4*>(part + row * N) + c;
@@ -923,8 +927,8 @@ __global__ void __launch_bounds__(256) splitk_resid_norm_kernel(const float* __r
   }
   const float inv = rsqrtf(block_sum(ss, red) / (float)N + eps);
 #pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    const int c = threadIdx.x + q * 256;
+  for (int q = 0; q < VPT; ++q) {
+    const int c = threadIdx.x + q * blockDim.x;
     if (c < nv) {
       const uint2 gr = reinterpret_cast<const uint2*>(gain)[c];
       const float g0 = __uint_as_float(gr.x << 16), g1 = __uint_as_float(gr.x & 0xffff0000u);
@@ -977,10 +981,17 @@ __global__ void wait_timeout_check_kernel() {
 // residual product with ep.norm_out also applies the following RMSNorm).
 static int reduce_slices(const float* part, int splits, int M, int N, int epi, void* C, const EpiParams& ep,
                          cudaStream_t st, bool pdl) {
-  if (epi == EPI_RESID_F32 && ep.norm_out)
-    return launch_ex(splitk_resid_norm_kernel, dim3(M), dim3(256), 0, st, pdl, part, splits, M, N,
-                     static_cast<float*>(C), static_cast<const uint16_t*>(ep.norm_gain), ep.norm_eps, ep.norm_out) !=
-           cudaSuccess;
+  if (epi == EPI_RESID_F32 && ep.norm_out) {
+    float* h = static_cast<float*>(C);
+    const uint16_t* g = static_cast<const uint16_t*>(ep.norm_gain);
+    const cudaError_t e =
+        N / 4 <= 1024
+            ? launch_ex(splitk_resid_norm_kernel<1>, dim3(M), dim3((N / 4 + 31) / 32 * 32), 0, st, pdl, part, splits,
+                        M, N, h, g, ep.norm_eps, ep.norm_out)
+            : launch_ex(splitk_resid_norm_kernel<2>, dim3(M), dim3(1024), 0, st, pdl, part, splits, M, N, h, g,
+                        ep.norm_eps, ep.norm_out);
+    return e != cudaSuccess;
+  }
   const size_t n_out = (size_t)M * (epi == EPI_SWIGLU ? N / 2 : N) / 4;
   const dim3 grid((unsigned)((n_out + 255) / 256 < 2048 ? (n_out + 255) / 256 : 2048));
   cudaError_t e;
