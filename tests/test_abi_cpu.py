@@ -205,3 +205,24 @@ def test_tile_features_reject_bad_arguments(riftlib):
     assert call(M=2, B=None) == INV and call(f=FAKE + 4) == INV and call(wsb=ws - 1) == INV
     assert call(n_v=200) == riftlib.RIFT_ERR_UNSUPPORTED  # not a square grid
     assert call(n_v=225) == riftlib.RIFT_ERR_UNSUPPORTED  # odd side: no quadrants
+
+
+def test_noalloc_scoring_rejects_before_touching_the_gpu(riftlib):
+    """The allocation-free scoring call checks its arguments, and that the scene's scratch fits the
+    library's fixed array, before any CUDA call: these rejections need no GPU."""
+    lib = riftlib.lib
+    args = dict(X=FAKE, xdt=riftlib.RIFT_BF16, N=4, n_v=576, d=256, t=FAKE, B=FAKE, M=8, knn_m=6, r=FAKE, s0=FAKE,
+                s1=FAKE, nbr=None, st=0)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return lib.rift_score_tiles_noalloc(a["X"], a["xdt"], a["N"], a["n_v"], a["d"], a["t"], a["B"], a["M"],
+                                            a["knn_m"], a["r"], a["s0"], a["s1"], a["nbr"], a["st"])
+
+    INV = riftlib.RIFT_ERR_INVALID
+    assert call(N=0) == INV and call(n_v=1025) == INV and call(d=100) == INV
+    assert call(X=None) == INV and call(X=FAKE + 4) == INV and call(knn_m=17) == INV
+    assert call(xdt=riftlib.RIFT_F32, d=8192) == riftlib.RIFT_ERR_UNSUPPORTED
+    # 2000 tiles of 576 x 4096 need more scratch than the fixed array holds
+    assert riftlib.score_workspace_bytes(2000, 576, 4096, 8) > riftlib.NOALLOC_SCORE_SCRATCH_BYTES
+    assert call(N=2000, d=4096) == riftlib.RIFT_ERR_CAPACITY
