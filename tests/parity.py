@@ -52,6 +52,28 @@ def oracle_select(wl, sc, p_ext=None):
     return O.select(sc.X, sc.embed, sc.query_ids, sc.bg_ids, wl.knn_m, wl.policy, p_ext=p_ext)
 
 
+class HostTiles:
+    """A device scene X [N, n_v, d] handed to the oracle tile by tile: indexing copies a block of
+    tiles to the host, so a scene larger than host memory (30 GB at 6400 tiles) never has to be
+    copied whole.  The values are the generator's, unchanged."""
+
+    def __init__(self, X, block: int = 64):
+        self.X, self.block = X, block
+        self.shape = tuple(X.shape)
+        self._b0, self._blk = -1, None
+
+    def __len__(self):
+        return self.shape[0]
+
+    def __getitem__(self, i):
+        i = int(i)
+        b0 = (i // self.block) * self.block
+        if b0 != self._b0:
+            self._blk = self.X[b0:b0 + self.block].cpu()
+            self._b0 = b0
+        return self._blk[i - b0]
+
+
 # Bounds on |CUDA fp32 value - oracle fp32 value| of the quantities that decide integers.
 #  * similarity G (compared in fp64 on both sides): the CUDA path recomputes its kNN candidates
 #    with fp64 accumulation of the fp32 tile embeddings, whose elements carry ~1e-7 relative error
