@@ -205,11 +205,16 @@ def smooth(s32: np.ndarray, nbr: np.ndarray) -> np.ndarray:
 # a5  per-scene min-max and the threshold (Section 2.3 Stage 1; Appendix B Step 3)
 # ------------------------------------------------------------------------------------------
 
-def minmax_normalize(s32: np.ndarray) -> np.ndarray:
+def minmax_normalize(s32: np.ndarray, lo=None, hi=None) -> np.ndarray:
+    """u = (s - min) / (max - min) in fp32 over the scene.  lo, hi: the scene's min and max when
+    s32 holds only some of its tiles (a shard); by default those of s32 itself."""
     s32 = np.asarray(s32, dtype=F32)
     if not np.all(np.isfinite(s32)):
         raise OracleError("non-finite tile score")
-    lo, hi = F32(s32.min()), F32(s32.max())
+    lo = F32(s32.min()) if lo is None else F32(lo)
+    hi = F32(s32.max()) if hi is None else F32(hi)
+    if not (np.isfinite(lo) and np.isfinite(hi)):
+        raise OracleError("non-finite score range")
     if hi == lo:
         return np.ones_like(s32)
     rng = F32(hi - lo)

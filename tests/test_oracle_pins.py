@@ -146,6 +146,22 @@ def test_minmax_two_tiles_and_all_equal():
     assert O.minmax_normalize(np.array([7.0], dtype=F32)).tolist() == [1.0]
 
 
+def test_minmax_of_a_shard_with_the_scene_range():
+    # a shard normalised with the scene's min and max gives, tile for tile, the scene's u: the
+    # per-scene min-max (Section 2.3 Stage 1) needs only those two numbers from other shards
+    rng = np.random.default_rng(9)
+    s = rng.standard_normal(37).astype(F32)
+    u = O.minmax_normalize(s)
+    for a, b in [(0, 12), (12, 25), (25, 37), (3, 4)]:
+        part = O.minmax_normalize(s[a:b], lo=s.min(), hi=s.max())
+        assert part.view(np.uint32).tolist() == u[a:b].view(np.uint32).tolist()
+    # the shard's own range is the default; a range with max = min gives u = 1
+    assert O.minmax_normalize(s, lo=s.min(), hi=s.max()).tolist() == u.tolist()
+    assert O.minmax_normalize(s[:3], lo=0.5, hi=0.5).tolist() == [1.0] * 3
+    with pytest.raises(O.OracleError):
+        O.minmax_normalize(s, lo=np.nan, hi=1.0)
+
+
 def test_threshold_is_greater_or_equal():
     # u = 0.37f exactly must be kept (Appendix B: u_i >= 0.37; Listing 1: >=)
     s = np.array([0.0, F32(0.37), 1.0], dtype=F32)
