@@ -46,9 +46,11 @@ def parse():
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
-    ap.add_argument("--kernel-case", choices=["prefill", "score", "decode", "merge"],
+    ap.add_argument("--kernel-case", choices=["prefill", "prefill_full", "score", "decode", "merge"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
-                         "'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); each runs 3 times")
+                         "'prefill_full' = one 7B-shaped layer over the 400-tile query's retained length mix "
+                         "(73 sequences, T = 23,819), 'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); "
+                         "each runs 3 times")
     return ap.parse_args()
 
 
@@ -295,17 +297,18 @@ def l2_note(x_bytes: int, w_bytes: int, flushed: bool) -> str:
         return "inputs fit in L2 (%s): L2 flushed between timed steps (a buffer of twice its size written outside the events)" % sizes
     return "inputs larger than L2 (%s)" % sizes
 
-PROFILED_WORKLOAD = "rift400_7b"  # the workload of profiles/launches_rift400_7b.md
+PROFILED_WORKLOAD = "rift400_7b"  # the workload of profiles/gemm_tc_traffic_rift400_7b.md
 
 
 def gemm_traffic(workload: str):
-    """DRAM bytes per GEMM launch from the committed ncu summary, if it was taken on this workload
-    and on the current gemm_tc.cu (source hash match); otherwise None."""
+    """DRAM bytes per GEMM launch from the committed ncu summary (one 7B layer at the 400-tile
+    query's 23,819 retained rows: every GEMM shape of the query at its full size), if it was taken
+    for this workload and on the current gemm_tc.cu (source hash match); otherwise None."""
     import hashlib
     import re
     if workload != PROFILED_WORKLOAD:
         return None
-    prof = ROOT / "profiles" / "launches_rift400_7b.md"
+    prof = ROOT / "profiles" / "gemm_tc_traffic_rift400_7b.md"
     src = ROOT / "paper_2609_29029_gb300" / "csrc" / "gemm_tc.cu"
     if not prof.exists() or not src.exists():
         return None
@@ -315,6 +318,19 @@ def gemm_traffic(workload: str):
     if not h or not b or hashlib.sha256(src.read_bytes()).hexdigest()[:16] != h.group(1):
         return None
     return int(b.group(1))
+
+
+def select_latency(pipe, sc, q, bg, sy, steps: int, stream=None) -> float:
+    """ms per query of scoring + selection + packing (the pre-prefill path), queries enqueued back
+    to back and timed by events around them only."""
+    st = stream if stream is not None else torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(steps):
+        pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False, counts=False, stream=st)
+    e1.record(st)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
 
 
 def sweep(steps: int, warmup: int):
@@ -336,16 +352,15 @@ def sweep(steps: int, warmup: int):
         for _ in range(warmup):
             pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False)
         torch.cuda.synchronize()
+        ms = select_latency(pipe, sc, q, bg, sy, steps)
+        n_kept, T = pipe.read_counts()
+        # per-class breakdown in a separate pass (its events sit between the classes' launches)
         abi.profile_enable(True)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
         for _ in range(steps):
-            n_kept, T = pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False)
-        e1.record()
+            pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False, counts=False)
         torch.cuda.synchronize()
         abi.profile_enable(False)
         prof = abi.profile_read()
-        ms = e0.elapsed_time(e1) / steps
         x_bytes = sc.X.numel() * sc.X.element_size()
         line = {"sweep": f"select+gather N={N}", "ms_per_query": ms,
                 "kernels_ms": {k: round(v[0] / steps, 4) for k, v in prof.items() if v[1]},
@@ -390,7 +405,7 @@ def decode_measure(pipe, dm, sc, dec, n_kept, T, stream, steps):
              prefill=False, stream=stream)
     kv = torch.empty(dec.n_layers, 2, T, d, dtype=torch.float16, device=dev)
     last = torch.empty(n_kept, dec.vocab, dtype=torch.float32, device=dev)
-    pipe.prefill(T, n_kept, stream, kv_out=kv, last_logits=last)
+    pipe.prefill(stream, kv_out=kv, last_logits=last, counts=(n_kept, T))
     key = rng.stream_key(0, rng.stream_id("bench-decode"))
     ids = torch.tensor([rng.hash_u32_int(key, i) % dec.vocab for i in range(n_kept)], dtype=torch.int32, device=dev)
     hid = torch.empty(n_kept, d, dtype=torch.bfloat16, device=dev)
@@ -464,7 +479,7 @@ def batch_measure(dm, dec, base, stream, steps, B=8, N=64):
         return e0.elapsed_time(e1) / steps
 
     ms_b = timed(lambda: pipe.run_batch(queries, stream=stream))
-    ms_1 = timed(lambda: [pipe.run(*qq, stream=stream) for qq in queries])
+    ms_1 = timed(lambda: [pipe.run(*qq, stream=stream, counts=False) for qq in queries])
     del queries, pipe
     torch.cuda.empty_cache()
     return {"queries": B, "tiles_per_scene": N, "retained_rows": rows,
@@ -479,10 +494,12 @@ def kernel_case(name: str):
     __graft_entry__.build()
     from paper_2609_29029_gb300 import DeviceModel, ScenePipeline, abi
     dev = torch.device("cuda", 0)
-    if name == "prefill":
+    if name in ("prefill", "prefill_full"):
         dec = W.DecoderShape(n_layers=1, d=4096, n_heads=32, head_dim=128, ffn=11008, vocab=32000)
         dm = DeviceModel(dec, [W.make_layer(dec, 0, dev)], W.make_final_norm(dec, dev), dev)
-        lens = [341] * 12
+        # prefill_full: the retained length mix of the 400-tile query (63 tiles at b = 288, 9 at
+        # 144, 1 at 72, each with the 35 system and 24 query rows): every GEMM at its full M
+        lens = [341] * 12 if name == "prefill" else [347] * 63 + [203] * 9 + [131]
         T = sum(lens)
         from synth import rng
         H0 = rng.normal_f32(0, rng.stream_id("case"), T * dec.d, dev).view(T, dec.d).to(torch.bfloat16)
@@ -571,8 +588,8 @@ def main():
     sy = torch.tensor(sc.sys_ids, **i32)
     stream = torch.cuda.current_stream()
 
-    def step(X):
-        return pipe.run(X, sc.embed, q, bg, sy, q, stream=stream)
+    def step(X, counts=True):
+        return pipe.run(X, sc.embed, q, bg, sy, q, stream=stream, counts=counts)
 
     for _ in range(max(args.warmup, 1)):
         n_kept, T = step(sc.X)
@@ -593,22 +610,24 @@ def main():
         if flush is None:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            for _ in range(args.steps):
-                n_kept, T = step(sc.X)
+            for _ in range(args.steps):  # whole queries enqueued back to back: no host read-back
+                step(sc.X, counts=False)
             e1.record(stream)
             torch.cuda.synchronize()
             ms = e0.elapsed_time(e1)
+            n_kept, T = pipe.read_counts(stream)
         else:
             evs = []
             for _ in range(args.steps):
                 flush.fill_(1.0)
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-                n_kept, T = step(sc.X)
+                step(sc.X, counts=False)
                 e1.record(stream)
                 evs.append((e0, e1))
             torch.cuda.synchronize()
             ms = sum(a.elapsed_time(b) for a, b in evs)
+            n_kept, T = pipe.read_counts(stream)
     launches = abi.launch_count() - l0
     abi.profile_enable(False)
     prof = abi.profile_read()
@@ -654,8 +673,10 @@ def main():
                 nxt.record(stream)
                 copy_stream.wait_event(nxt)
                 ready = h2d(bufs[(k + 1) % 2])
-            nk, Te = p.run(buf["X"], sc.embed, buf["ids"][0], buf["ids"][1], buf["ids"][2], buf["ids"][0],
-                           stream=stream)
+            p.run(buf["X"], sc.embed, buf["ids"][0], buf["ids"][1], buf["ids"][2], buf["ids"][0], stream=stream,
+                  counts=False)
+            # the result's size: wait for this query's packing only (its prefill stays queued)
+            nk, Te = p.counts()
             done = torch.cuda.Event()
             done.record(stream)
             d2h_stream.wait_event(done)
@@ -698,7 +719,9 @@ def main():
     achieved = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
     traffic = gemm_traffic(wl.name)
     per_step = {k: round(v[0] / args.steps, 3) for k, v in prof.items()}
-    sel_ms = (prof["score"][0] + prof["select"][0] + prof["pack"][0]) / args.steps
+    # the pre-prefill path alone, without the profiler's events between its classes
+    sel_ms = select_latency(pipe, sc, q, bg, sy, args.steps, stream)
+    x_bytes = sc.X.numel() * sc.X.element_size()
 
     cpu = None
     if not args.no_cpu_baseline and ws == 1:
@@ -720,6 +743,7 @@ def main():
                                  flush is not None)},
         "scene_queries_per_s": 1e3 * args.steps / ms_max,
         "select_latency_ms": sel_ms,
+        "select_latency_floor_ms": x_bytes / (peaks.get("hbm_gbs", 6796.5) * 1e6),
         "kernels_ms_per_step": per_step,
         "roofline": {"bound": "tensor", "kernel": "prefill GEMM", "achieved": achieved, "peak": peak,
                      "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None, "traffic": traffic,

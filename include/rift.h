@@ -19,7 +19,9 @@
  *   - Every array argument is a DEVICE pointer owned by the caller, unless marked
  *     "host".  The library never allocates device memory: scratch comes from the
  *     caller's workspace `ws` (size from the matching *_workspace_bytes query; pass
- *     at least that many bytes, 256-byte aligned).
+ *     at least that many bytes, 256-byte aligned).  One exception: the library image
+ *     holds a static device array of RIFT_NOALLOC_SCORE_SCRATCH_BYTES (64 MiB), the
+ *     scratch of rift_score_tiles_noalloc, on every device that loads it.
  *   - Sizes are host ints.  Counts that only the device knows (n_kept, T) are written
  *     to device ints and can be read after rift_sync_status.
  *   - Calls are asynchronous on `stream` (a cudaStream_t; 0 = the legacy default stream)
@@ -171,8 +173,11 @@ rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int 
  * those of rift_score_tiles without ws/ws_bytes; results are the same.
  *   - A scene whose scratch (rift_score_workspace_bytes(N, n_v, d, M)) exceeds the array
  *     returns RIFT_ERR_CAPACITY and launches nothing (64 MiB holds N = 400 tiles at d = 4096).
- *   - The first call on each device looks up the array's device address while that device is
- *     current; make that first call before any stream capture.
+ *   - Each call looks the array's device address up in the CUDA context current on the calling
+ *     thread (each context has its own copy of the array).  A call made while its stream is being
+ *     captured does not look it up but reuses the address an earlier call recorded for that
+ *     context (RIFT_ERR_UNSUPPORTED if there was none): make the first call in each context
+ *     before any stream capture.
  *   - All calls share the array and it keeps the last call's contents (nothing needs to start
  *     at zero).  Calls whose work overlaps on the GPU race on it: order them. */
 #define RIFT_NOALLOC_SCORE_SCRATCH_BYTES (64u << 20)
@@ -203,6 +208,55 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
                                         float* u, int* kept, int* n_kept, int* budgets,
                                         int* sel, int* sel_off,
                                         void* ws, size_t ws_bytes, rift_stream_t stream);
+
+/* ---- One scene sharded over several ranks (GPUs or hosts) ----
+ * Every step of the method is per tile except two that need the whole scene: the kNN smoothing of
+ * Appendix B Step 2 (each tile's m most similar tiles, anywhere in the scene) and the per-scene
+ * min-max of Section 2.3 Stage 1 (Listing 1's u = (s - min) / (max - min)).  A scene split into
+ * contiguous shards of tiles runs, on each rank:
+ *   rift_score_shard                   Eq. 1 on the shard's tokens and tiles, and its tile
+ *                                      embeddings V
+ *   (exchange: every rank's V and tile_s_raw, gathered in tile order)
+ *   rift_smooth_rows                   the smoothing of the shard's tiles against the whole scene
+ *   rift_score_range                   (min, max) of the shard's smoothed scores
+ *   (exchange: the scene's min of the mins and max of the maxes)
+ *   rift_select_budgeted_tokens_ranged prune, budgets and top-b of the shard's tiles with the
+ *                                      scene's range
+ *   rift_pack_ragged                   the shard's kept tiles, as for one rank
+ * The exchanges are the caller's (two collectives; the library makes no collective call).  With
+ * the same inputs every score, neighbour, kept tile, budget and selected token equals what
+ * rift_score_tiles and rift_select_budgeted_tokens compute on the whole scene on one rank (the
+ * fp32 sums of a tile's scores and of a pair's similarity do not depend on the split).
+ *
+ *   rift_score_shard: X [N_local, n_v, d] the shard's tokens; t, B, M as for rift_score_tiles;
+ *     token_scores out fp32 [N_local, n_v], tile_s_raw out fp32 [N_local] (Eq. 1, as
+ *     rift_score_tiles), V out fp32 [N_local, d]: V_i = P_i / ||P_i||, P_i = sum_k x_ik.
+ *     ws: rift_score_shard_workspace_bytes(N_local, n_v, d) bytes.
+ *   rift_smooth_rows: V fp32 [N, d] and tile_s_raw fp32 [N] of the whole scene (16-byte aligned
+ *     V); the rows row0 .. row0 + n_rows - 1 are smoothed: tile_s out fp32 [n_rows] and nbr out
+ *     int32 [n_rows, m] (nullable) for those rows, m = min(knn_m, N - 1), exactly as
+ *     rift_score_tiles' tile_s and nbr.  ws: rift_smooth_workspace_bytes(N, n_rows, d) bytes.
+ *   rift_score_range: range out fp32 [2] = (min, max) of tile_s [n]; a NaN or Inf sets
+ *     RIFT_ERR_NONFINITE.
+ *   rift_select_budgeted_tokens_ranged: rift_select_budgeted_tokens for N tiles of a larger scene,
+ *     with u_i = (s~_i - s_range[0]) / (s_range[1] - s_range[0]) (device fp32 [2], the scene's
+ *     min and max; u = 1 for every tile if they are equal).  kept holds shard-local tile
+ *     indices.  A non-finite range or score sets RIFT_ERR_NONFINITE. */
+size_t rift_score_shard_workspace_bytes(int N_local, int n_v, int d);
+rift_status rift_score_shard(const void* X, rift_dtype xdt, int N_local, int n_v, int d,
+                             const float* t, const float* B, int M, float* token_scores,
+                             float* tile_s_raw, float* V, void* ws, size_t ws_bytes,
+                             rift_stream_t stream);
+size_t rift_smooth_workspace_bytes(int N, int n_rows, int d);
+rift_status rift_smooth_rows(const float* V, const float* tile_s_raw, int N, int d, int row0,
+                             int n_rows, int knn_m, float* tile_s, int* nbr, void* ws,
+                             size_t ws_bytes, rift_stream_t stream);
+rift_status rift_score_range(const float* tile_s, int n, float* range, rift_stream_t stream);
+rift_status rift_select_budgeted_tokens_ranged(const float* token_scores, const float* tile_s,
+                                               int N, int n_v, const float* s_range,
+                                               const float* p, const rift_policy* policy,
+                                               float* u, int* kept, int* n_kept, int* budgets,
+                                               int* sel, int* sel_off, rift_stream_t stream);
 
 /* ---- Predictor features (Section 2.3, Stage 2: the features of the paper's p_i predictor,
  * computed for the listed tiles, e.g. the kept ones, whose p_i the budget rule uses) ----
@@ -289,24 +343,35 @@ rift_status rift_pack_ragged_at(const void* X, rift_dtype xdt, int N, int n_v, i
                                 int row_base, rift_stream_t stream);
 
 /* ---- a9. Decoder prefill (Section 2.1) ----
- *   hidden     bf16 [T, d]: in, the packed batch; out, the final hidden states (after the
- *              final RMSNorm).  The residual stream is kept in fp32 in the workspace.
- *   T          packed rows (host int, e.g. read back after rift_sync_status)
- *   cu_seqlens int32 [n_seq + 1], positions int32 [T] from rift_pack_ragged
+ *   hidden     bf16 [max_T, d]: in, the packed batch; out, the final hidden states (after the
+ *              final RMSNorm) of its first T rows.  The residual stream is kept in fp32 in the
+ *              workspace.
+ *   T          int32 [1] DEVICE: the packed rows, as rift_pack_ragged writes it; read by the
+ *              kernels, so the call can be enqueued right after the packing with no host read-back.
+ *              NULL: max_T is the row count.
+ *   max_T      host: the rows that hidden, positions and kv_out hold (a count above it is clamped
+ *              to it; rift_pack_ragged has then already raised RIFT_ERR_CAPACITY)
+ *   cu_seqlens int32 [max_seqs + 1], positions int32 [max_T] from rift_pack_ragged
+ *   n_seq      int32 [1] DEVICE: the packed sequences (rift_select_budgeted_tokens' n_kept);
+ *              NULL: max_seqs is the count.  Above max_seqs sets RIFT_ERR_CAPACITY (the first
+ *              max_seqs are prefilled); so does a sequence that ends past max_T (it and the ones
+ *              after it are left out).
+ *   max_seqs   host: an upper bound on the sequence count (sizes the workspace and the logits)
  *   max_len    an upper bound on every sequence length (host int)
  * Each layer: h += W_o Attn(RoPE(q), RoPE(k), v) with x = RMSNorm(h) g_attn, causal within
  * each sequence only; h += W_down(SiLU(W_gate x) * (W_up x)) with x = RMSNorm(h) g_ffn.
  * GEMM and attention operands are fp16 (normalised activations, q/k/v, softmax weights,
- * attention output, SwiGLU output), accumulation fp32, residual stream fp32.
+ * attention output, SwiGLU output), accumulation fp32, residual stream fp32.  The launches are
+ * sized for the capacities and stop at the device counts.
  * Optional outputs (NULL = not written):
- *   kv_out      fp16 [n_layers][2][T][d]: per layer the keys after RoPE ([l][0]) and the values
+ *   kv_out      fp16 [n_layers][2][max_T][d]: per layer the keys after RoPE ([l][0]) and the values
  *               ([l][1]) of every packed row, heads contiguous: the KV cache the prefill builds
  *               (Section 2.1), as rift_decode_step reads it.  16-byte aligned.
- *   last_logits fp32 [n_seq, vocab]: logits of each sequence's last row,
+ *   last_logits fp32 [max_seqs, vocab]: logits of each sequence's last row,
  *               (RMSNorm(h_last) g_final) lm_head^T; needs m->lm_head.  16-byte aligned. */
 size_t rift_prefill_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len);
-rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
-                                const int* cu_seqlens, int n_seq, int max_len,
+rift_status rift_prefill_layers(const rift_model* m, void* hidden, const int* T, int max_T,
+                                const int* cu_seqlens, const int* n_seq, int max_seqs, int max_len,
                                 const int* positions, void* kv_out, float* last_logits,
                                 void* ws, size_t ws_bytes, rift_stream_t stream);
 
@@ -319,18 +384,20 @@ rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T,
  *   sys_ids     int32 [S] (device), embed bf16 [vocab, d]
  *   prefix_hidden out bf16 [S, d]: the prompt's final hidden states
  *   prefix_kv   out fp16 [n_layers][2][S][d]: the prompt's cache (the layout of kv_out)
- *   hidden      bf16 [T, d] in/out: the suffix rows (packed with S = 0), then their final hidden
- *               states; cu_seqlens [n_seq + 1] and positions [T] (0-based) over them
+ *   hidden      bf16 [max_T, d] in/out: the suffix rows (packed with S = 0), then their final
+ *               hidden states; T (device, nullable), max_T, cu_seqlens [max_seqs + 1], n_seq (device,
+ *               nullable), max_seqs and positions [max_T] (0-based) over them, as for
+ *               rift_prefill_layers
  *   max_len     an upper bound on S + every suffix length
- *   last_logits out fp32 [n_seq, vocab] (nullable; needs m->lm_head): each sequence's last row
- *   ws          rift_prefill_shared_prefix_workspace_bytes(m, T, n_seq, max_len, S) bytes */
+ *   last_logits out fp32 [max_seqs, vocab] (nullable; needs m->lm_head): each sequence's last row
+ *   ws          rift_prefill_shared_prefix_workspace_bytes(m, max_T, max_seqs, max_len, S) bytes */
 size_t rift_prefill_shared_prefix_workspace_bytes(const rift_model* m, int max_T, int max_seqs, int max_len,
                                                   int S);
 rift_status rift_prefill_shared_prefix(const rift_model* m, const int* sys_ids, int S, const void* embed,
                                        int vocab, void* prefix_hidden, void* prefix_kv, void* hidden,
-                                       int T, const int* cu_seqlens, int n_seq, int max_len,
-                                       const int* positions, float* last_logits, void* ws,
-                                       size_t ws_bytes, rift_stream_t stream);
+                                       const int* T, int max_T, const int* cu_seqlens, const int* n_seq,
+                                       int max_seqs, int max_len, const int* positions, float* last_logits,
+                                       void* ws, size_t ws_bytes, rift_stream_t stream);
 
 /* ---- Decode step after the prefill (Section 2.1: decoding extends the prefilled KV cache one
  * token at a time) ----
@@ -338,7 +405,7 @@ rift_status rift_prefill_shared_prefix(const rift_model* m, const int* sys_ids, 
  * bf16) at position L_i = cu_seqlens[i+1] - cu_seqlens[i], attending to that sequence's cached
  * rows and to itself, through every layer and the final RMSNorm.
  *   kv_cache   fp16 [n_layers][2][T][d] as written by rift_prefill_layers (kv_out) for the
- *              same cu_seqlens
+ *              same cu_seqlens; T is the row capacity it was written with (that call's max_T)
  *   max_len    an upper bound on every L_i + 1 (host int, at most 32768)
  *   hidden_out bf16 [n_seq, d] final hidden states of the new tokens, or NULL
  *   kv_new     fp16 [n_layers][2][n_seq][d] the new tokens' keys (after RoPE) and values, or NULL

@@ -64,14 +64,21 @@ SIGNATURES = {
     "rift_merge_contextual": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz,
                                    _vp]),
     "rift_prefill_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i]),
-    "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "rift_prefill_layers": (_i, [C.POINTER(Model), _vp, _vp, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "rift_prefill_shared_prefix_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i, _i, _i]),
-    "rift_prefill_shared_prefix": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _vp, _vp, _vp, _i, _vp, _i, _i, _vp, _vp,
-                                        _vp, _sz, _vp]),
+    "rift_prefill_shared_prefix": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _vp, _vp, _vp, _vp, _i, _vp, _vp, _i, _i,
+                                        _vp, _vp, _vp, _sz, _vp]),
     "rift_decode_workspace_bytes": (_sz, [C.POINTER(Model), _i, _i]),
     "rift_decode_step": (_i, [C.POINTER(Model), _vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _sz,
                               _vp]),
     "rift_score_tiles_noalloc": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp]),
+    "rift_score_shard_workspace_bytes": (_sz, [_i, _i, _i]),
+    "rift_score_shard": (_i, [_vp, _i, _i, _i, _i, _vp, _vp, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "rift_smooth_workspace_bytes": (_sz, [_i, _i, _i]),
+    "rift_smooth_rows": (_i, [_vp, _vp, _i, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp]),
+    "rift_score_range": (_i, [_vp, _i, _vp, _vp]),
+    "rift_select_budgeted_tokens_ranged": (_i, [_vp, _vp, _i, _i, _vp, _vp, C.POINTER(Policy), _vp, _vp, _vp, _vp,
+                                                _vp, _vp, _vp]),
     "rift_linear": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
     "rift_attention_workspace_bytes": (_sz, [_i, _i]),
     "rift_attention_varlen": (_i, [_vp, _i, _vp, _i, _i, _i, _vp, _vp, _sz, _vp]),
@@ -172,6 +179,36 @@ def score_tiles_noalloc(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_
 NOALLOC_SCORE_SCRATCH_BYTES = 64 << 20
 
 
+def score_shard_workspace_bytes(N_local, n_v, d) -> int:
+    return lib.rift_score_shard_workspace_bytes(N_local, n_v, d)
+
+
+def score_shard(X, xdt, N_local, n_v, d, t, B, M, token_scores, tile_s_raw, V, ws, ws_bytes, stream=None):
+    _check(lib.rift_score_shard(ptr(X), xdt, N_local, n_v, d, ptr(t), ptr(B), M, ptr(token_scores), ptr(tile_s_raw),
+                                ptr(V), ptr(ws), ws_bytes, stream_handle(stream)), "rift_score_shard")
+
+
+def smooth_workspace_bytes(N, n_rows, d) -> int:
+    return lib.rift_smooth_workspace_bytes(N, n_rows, d)
+
+
+def smooth_rows(V, tile_s_raw, N, d, row0, n_rows, knn_m, tile_s, nbr, ws, ws_bytes, stream=None):
+    _check(lib.rift_smooth_rows(ptr(V), ptr(tile_s_raw), N, d, row0, n_rows, knn_m, ptr(tile_s), ptr(nbr), ptr(ws),
+                                ws_bytes, stream_handle(stream)), "rift_smooth_rows")
+
+
+def score_range(tile_s, n, out, stream=None):
+    _check(lib.rift_score_range(ptr(tile_s), n, ptr(out), stream_handle(stream)), "rift_score_range")
+
+
+def select_budgeted_tokens_ranged(token_scores, tile_s, N, n_v, s_range, p, policy: Policy, u, kept, n_kept, budgets,
+                                  sel, sel_off, stream=None):
+    _check(lib.rift_select_budgeted_tokens_ranged(ptr(token_scores), ptr(tile_s), N, n_v, ptr(s_range), ptr(p),
+                                                  C.byref(policy), ptr(u), ptr(kept), ptr(n_kept), ptr(budgets),
+                                                  ptr(sel), ptr(sel_off), stream_handle(stream)),
+           "rift_select_budgeted_tokens_ranged")
+
+
 def select_workspace_bytes(N, n_v) -> int:
     return lib.rift_select_workspace_bytes(N, n_v)
 
@@ -243,9 +280,25 @@ def prefill_workspace_bytes(model: Model, max_T, max_seqs, max_len) -> int:
     return lib.rift_prefill_workspace_bytes(C.byref(model), max_T, max_seqs, max_len)
 
 
+def _count(c, cap, what):
+    """A count argument of the prefill calls: a device int32 tensor (with its host capacity `cap`),
+    or a host int, which is then both the count and the capacity (a NULL device pointer)."""
+    if isinstance(c, int):
+        if cap is not None and cap != c:
+            raise ValueError(f"{what}: a host count is its own capacity; pass a device count to use {cap}")
+        return None, c
+    if cap is None:
+        raise ValueError(f"{what}: a device count needs its host capacity")
+    return ptr(c), cap
+
+
 def prefill_layers(model: Model, hidden, T, cu_seqlens, n_seq, max_len, positions, ws, ws_bytes, stream=None,
-                   kv_out=None, last_logits=None):
-    _check(lib.rift_prefill_layers(C.byref(model), ptr(hidden), T, ptr(cu_seqlens), n_seq, max_len,
+                   kv_out=None, last_logits=None, max_T=None, max_seqs=None):
+    """rift_prefill_layers.  T and n_seq: device int32 counts (with max_T and max_seqs, the host
+    capacities), or host ints (then also the capacities)."""
+    T_p, max_T = _count(T, max_T, "T")
+    n_p, max_seqs = _count(n_seq, max_seqs, "n_seq")
+    _check(lib.rift_prefill_layers(C.byref(model), ptr(hidden), T_p, max_T, ptr(cu_seqlens), n_p, max_seqs, max_len,
                                    ptr(positions), ptr(kv_out), ptr(last_logits), ptr(ws), ws_bytes,
                                    stream_handle(stream)),
            "rift_prefill_layers")
@@ -256,10 +309,15 @@ def prefill_shared_prefix_workspace_bytes(model: Model, max_T, max_seqs, max_len
 
 
 def prefill_shared_prefix(model: Model, sys_ids, S, embed, vocab, prefix_hidden, prefix_kv, hidden, T, cu_seqlens,
-                          n_seq, max_len, positions, last_logits, ws, ws_bytes, stream=None):
+                          n_seq, max_len, positions, last_logits, ws, ws_bytes, stream=None, max_T=None,
+                          max_seqs=None):
+    """rift_prefill_shared_prefix; T and n_seq as for prefill_layers."""
+    T_p, max_T = _count(T, max_T, "T")
+    n_p, max_seqs = _count(n_seq, max_seqs, "n_seq")
     _check(lib.rift_prefill_shared_prefix(C.byref(model), ptr(sys_ids), S, ptr(embed), vocab, ptr(prefix_hidden),
-                                          ptr(prefix_kv), ptr(hidden), T, ptr(cu_seqlens), n_seq, max_len,
-                                          ptr(positions), ptr(last_logits), ptr(ws), ws_bytes, stream_handle(stream)),
+                                          ptr(prefix_kv), ptr(hidden), T_p, max_T, ptr(cu_seqlens), n_p, max_seqs,
+                                          max_len, ptr(positions), ptr(last_logits), ptr(ws), ws_bytes,
+                                          stream_handle(stream)),
            "rift_prefill_shared_prefix")
 
 

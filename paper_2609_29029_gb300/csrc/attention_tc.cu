@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
   __syncthreads();
   fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int n_items = n_entries * H;
+  const int n_items = min(n_entries, sched[n_entries].x) * H;  // entries in use (the schedule's count)
   const int d = H * HD;
   const int np = (S_pre + KB - 1) / KB;  // prefix blocks ahead of every sequence's own
 
@@ -539,16 +539,37 @@ __global__ void __launch_bounds__(THREADS, Cfg<HD, KB>::CTAS)
 
 // One entry per 128-row q-block: (first row of its sequence in the packed batch, sequence length,
 // first row of the block within the sequence, 0); the rest (0, 0, 0, 0), which the kernel skips.
-// Longer sequences' entries are not reordered: items are interleaved across CTAs by the
-// persistent loop.
+// Entry n_max holds the number of entries in use (.x), so the attention visits only those.  The
+// sequence count is n_seq_dev's value when given (a count written by an earlier kernel), clamped
+// to n_seq; a sequence that ends past row_cap (the rows the buffers hold) and the sequences after
+// it are left out and RIFT_EBIT_CAPACITY is set.  Longer sequences' entries are not reordered:
+// items are interleaved across CTAs by the persistent loop.
 __global__ void __launch_bounds__(1024) schedule128_kernel(const int* __restrict__ cu, int n_seq,
+                                                           const int* __restrict__ n_seq_dev, int row_cap,
                                                            int4* __restrict__ sched, int n_max) {
   __shared__ int sh[33];
+  __shared__ int s_cut;
+  int n = n_seq;
+  if (n_seq_dev) {
+    const int nd = *n_seq_dev;
+    if (nd > n_seq && threadIdx.x == 0) atomicOr(&g_err_attn, RIFT_EBIT_CAPACITY);
+    n = max(0, min(n_seq, nd));
+  }
+  if (threadIdx.x == 0) s_cut = n;
+  __syncthreads();
+  // the first sequence that does not fit in row_cap rows ends the schedule
+  for (int s = threadIdx.x; s < n; s += blockDim.x)
+    if (cu[s + 1] > row_cap || cu[s + 1] < cu[s]) atomicMin(&s_cut, s);
+  __syncthreads();
+  if (s_cut < n) {
+    if (threadIdx.x == 0) atomicOr(&g_err_attn, RIFT_EBIT_CAPACITY);
+    n = s_cut;
+  }
   int base = 0;
-  for (int c0 = 0; c0 < n_seq; c0 += blockDim.x) {
+  for (int c0 = 0; c0 < n; c0 += blockDim.x) {
     const int s = c0 + threadIdx.x;
     int nb = 0, s0 = 0, len = 0;
-    if (s < n_seq) {
+    if (s < n) {
       s0 = cu[s];
       len = cu[s + 1] - s0;
       nb = (len + BQ - 1) / BQ;
@@ -560,6 +581,7 @@ __global__ void __launch_bounds__(1024) schedule128_kernel(const int* __restrict
     base += total;
   }
   for (int i = base + threadIdx.x; i < n_max; i += blockDim.x) sched[i] = make_int4(0, 0, 0, 0);
+  if (threadIdx.x == 0) sched[n_max] = make_int4(min(base, n_max), 0, 0, 0);
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -589,8 +611,9 @@ static int sm_count() {
 }  // namespace fa
 
 // q-block schedule of the tcgen05 attention (one entry per 128 rows of a sequence)
-void launch_attention_schedule(const int* cu_seqlens, int n_seq, int4* sched, int n_sched_max, cudaStream_t st) {
-  fa::schedule128_kernel<<<1, 1024, 0, st>>>(cu_seqlens, n_seq, sched, n_sched_max);
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, const int* n_seq_dev, int row_cap, int4* sched,
+                               int n_sched_max, cudaStream_t st) {
+  fa::schedule128_kernel<<<1, 1024, 0, st>>>(cu_seqlens, n_seq, n_seq_dev, row_cap, sched, n_sched_max);
 }
 
 int attention_max_qblocks(int max_T, int max_seqs) { return (max_T + fa::BQ - 1) / fa::BQ + max_seqs; }

@@ -194,14 +194,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int group_m, int& m_blk, int& n_blk) {
-  const int per_group = group_m * nt;
+// Tile order.  group > 0: bands of `group` M-tiles, M fastest within a band, so the band's A rows
+// stay in L2 while every B tile streams past them once per band.  group < 0: bands of -group
+// N-tiles, N fastest, so the band's B rows stay in L2 and A streams once per band (the better
+// order when B is the smaller operand: traffic A + B x bands vs B + A x bands).
+__device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int group, int& m_blk, int& n_blk) {
+  const bool n_major = group < 0;
+  const int g = n_major ? -group : group;
+  const int inner = n_major ? nt : mt, outer = n_major ? mt : nt;
+  const int per_group = g * outer;
   const int grp = tile / per_group;
-  const int first_m = grp * group_m;
-  const int gsz = min(mt - first_m, group_m);
+  const int first = grp * g;
+  const int gsz = min(inner - first, g);
   const int r = tile - grp * per_group;
-  m_blk = first_m + r % gsz;
-  n_blk = r / gsz;
+  const int a = first + r % gsz, b = r / gsz;
+  m_blk = n_major ? b : a;
+  n_blk = n_major ? a : b;
 }
 
 __device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
@@ -305,8 +313,8 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
 // tile row, and the even CTA issues the M = 256 MMAs into both SMs' tensor memory.
 template <int EPI, int BN_, int STAGES_, bool PAIR = false>
 __global__ void __launch_bounds__(THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride,
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M_cap,
+                   int N, int K, void* C, const EpiParams ep, int group_m, int splits, size_t split_stride,
                    int a_const) {
   constexpr int BN = BN_, STAGES = STAGES_;  // this instance's tile width and ring depth
   constexpr int TM = PAIR ? 2 * BM : BM;     // rows of a tile (both CTAs of the pair)
@@ -363,7 +371,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_trigger();
-  if (warp != 0) pdl_wait();  // the producer waits after prefetching constant A tiles
+  // The producer waits after prefetching constant A tiles; with a device row count every role
+  // waits first, since the count is written by an earlier kernel.
+  if (warp != 0 || ep.m_dev) pdl_wait();
+  // Rows: M_cap (host), or the device count ep.m_dev clamped to it (the rows the TMA map covers).
+  const int M = ep.m_dev ? max(0, min(M_cap, *ep.m_dev)) : M_cap;
 
   const int mt = (M + TM - 1) / TM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
   const int n_tiles = mt * nt;
@@ -386,7 +398,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       // a_const: A does not depend on earlier kernels (weights), so the first ring round of this
       // CTA's first unit takes its A tiles before waiting for the kernel before this one.
       int n_pre = 0;
-      if (!PAIR && a_const && u_first < n_units) {
+      if (!PAIR && a_const && !ep.m_dev && u_first < n_units) {
         int m_blk, n_blk, k0, k1;
         tile_coords(u_first / splits, mt, nt, group_m, m_blk, n_blk);
         unit_k(u_first, k0, k1);
@@ -748,6 +760,18 @@ static int sm_count() {
   return n;
 }
 
+// L2 band of the tile order (tile_coords): as many tiles of the resident operand as keep its rows
+// within kBandBytes of L2 (lo..hi tiles).  The resident operand is the larger one when
+// kOrientBands (the smaller one is then streamed once per band), else always A.
+constexpr size_t kBandBytes = (size_t)48 << 20;
+constexpr bool kOrientBands = true;
+static int band_group(int M, int N, int K, int tm, int tn, int lo, int hi) {
+  const bool n_major = kOrientBands && (size_t)N < (size_t)M;
+  int g = (int)(kBandBytes / ((size_t)(n_major ? tn : tm) * K * 2));
+  g = g < lo ? lo : (g > hi ? hi : g);
+  return n_major ? -g : g;
+}
+
 // pdl: launched as a programmatic dependent of the kernel before it; a_const: A is constant weights.
 template <int EPI, int BN_ = BN, int STAGES_ = STAGES>
 static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, void* C, const EpiParams& ep,
@@ -757,10 +781,7 @@ static int launch(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int 
   if (raise_smem_limit(smem_raised, gemm_tc_kernel<EPI, BN_, STAGES_>, (int)smem) != cudaSuccess) return 1;
   const int units = ((M + BM - 1) / BM) * ((N + BN_ - 1) / BN_) * splits;
   const int grid = units < sm_count() ? units : sm_count();
-  // Band height: as many M-tiles as keep the band's A rows within ~48 MB of L2 (8..64), so each
-  // weight tile is streamed from DRAM once per band.
-  int group_m = (int)((48u << 20) / ((size_t)BM * K * 2));
-  group_m = group_m < 8 ? 8 : (group_m > 64 ? 64 : group_m);
+  const int group_m = band_group(M, N, K, BM, BN_, 8, 64);
   return launch_ex(gemm_tc_kernel<EPI, BN_, STAGES_>, dim3(grid), dim3(THREADS), smem, st, pdl, a, b, M, N, K, C, ep,
                    group_m, splits, (size_t)M * N, a_const) != cudaSuccess;
 }
@@ -808,9 +829,7 @@ static int launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
   if (max_clusters <= 0) return -1;
   const int units = ((M + 2 * BM - 1) / (2 * BM)) * ((N + BN - 1) / BN);
   const int clusters = units < max_clusters ? units : max_clusters;
-  // bands of 256-row tiles whose A rows fit in ~48 MB of L2
-  int group_m = (int)((48u << 20) / ((size_t)2 * BM * K * 2));
-  group_m = group_m < 4 ? 4 : (group_m > 32 ? 32 : group_m);
+  const int group_m = band_group(M, N, K, 2 * BM, BN, 4, 32);
   cfg.gridDim = dim3(2 * clusters, 1, 1);
   cfg.stream = st;
   return cudaLaunchKernelEx(&cfg, kern, a, b, M, N, K, C, ep, group_m, 1, (size_t)M * N, 0) == cudaSuccess ? 0 : 1;
@@ -1031,10 +1050,11 @@ int launch_wait_timeout_check(cudaStream_t st) {
 // Requirements: K % 8 == 0 (16-byte row pitch), N % 8 == 0 (N % 32 == 0 for SwiGLU, N % 64 == 0 for
 // the RoPE epilogue), A, B and C 16-byte aligned.
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st, void* split_ws, size_t split_ws_bytes, bool pdl) {
+                   cudaStream_t st, void* split_ws, size_t split_ws_bytes, bool pdl, bool b_const) {
   using namespace tc;
   if (M <= 0 || N <= 0 || K <= 0) return 0;
   if (K % 8 != 0 || N % 8 != 0 || (epi == EPI_SWIGLU && N % 32 != 0)) return 1;
+  if (ep.m_dev && split_ws) return 1;  // a device row count is for the unsplit products only
   if (epi == EPI_QKV_ROPE && (N % 64 != 0 || (ep.head_dim != 64 && ep.head_dim != 128) || !ep.positions || !ep.rope))
     return 1;
   // Few rows (<= 128, with scratch: the decode step): the operands swapped so that the weights
@@ -1047,7 +1067,9 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     // a unit's partials (M x 128 fp32, written and read back) cost M / 16 K-blocks of weight
     // traffic; its fill and drain about 1.5 more
     const int splits = choose_splits(N, M, K, split_ws_bytes, SW_BN, M / 16.0 + 1.5);
-    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits, pdl, 1))
+    // constant weights (b_const) are requested before the wait on the kernel before this one
+    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits, pdl,
+                                                  b_const ? 1 : 0))
       return 1;
     return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st, pdl);
   }

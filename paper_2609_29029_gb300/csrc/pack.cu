@@ -28,6 +28,8 @@ constexpr int PK_THREADS = 256;
 __global__ void seqlens_kernel(const int* __restrict__ n_kept, const int* __restrict__ sel_off,
                                const int* __restrict__ ctx_off, int N, int S, int Q, int max_T, int row_base,
                                int* __restrict__ cu, int* __restrict__ T) {
+  pdl_trigger();
+  pdl_wait();
   const int n = *n_kept;
   for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= N; j += gridDim.x * blockDim.x) {
     const int jj = min(j, n);
@@ -47,6 +49,8 @@ __global__ void __launch_bounds__(PK_THREADS) pack_kernel(
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
     const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
     const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
+  pdl_trigger();
+  pdl_wait();
   const int j = blockIdx.x;
   if (j >= *n_kept) return;
   const int so = sel_off[j];
@@ -134,6 +138,8 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
     const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
     const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ __align__(128) uint8_t ring[];
   __shared__ __align__(8) uint64_t bars[PKB_SLOTS];
   const int j = blockIdx.x;
@@ -221,8 +227,8 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
                  const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
                  void* packed, int max_T, int* cu_seqlens, int* positions, int* T, int row_base,
                  cudaStream_t st) {
-  seqlens_kernel<<<(N + 1 + 255) / 256, 256, 0, st>>>(n_kept, sel_off, ctx_off, N, S, Q, max_T, row_base,
-                                                      cu_seqlens, T);
+  launch_ex(seqlens_kernel, dim3((N + 1 + 255) / 256), dim3(256), 0, st, true, n_kept, sel_off, ctx_off, N, S, Q,
+            max_T, row_base, cu_seqlens, T);
   const uint16_t* cx = static_cast<const uint16_t*>(ctx);
   const int max_L = S + n_v + Q;
   dim3 grid(N, (max_L + PK_ROWS - 1) / PK_ROWS);
@@ -232,13 +238,13 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
     if (raise_smem_limit(smem_raised, pack_bulk_kernel, PKB_SLOTS * 8192 * 2) != cudaSuccess)
       return;  // the error stays pending for the caller's launch check
     dim3 gb(N, (max_L + PKB_ROWS - 1) / PKB_ROWS);
-    pack_bulk_kernel<<<gb, 64, smem, st>>>(
-        static_cast<const uint16_t*>(X), N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q,
-        static_cast<const uint16_t*>(embed), vocab, cx, ctx_off, static_cast<uint16_t*>(packed), max_T, positions);
+    launch_ex(pack_bulk_kernel, gb, dim3(64), smem, st, true, static_cast<const uint16_t*>(X), N, n_v, d, kept,
+              n_kept, sel, sel_off, sys_ids, S, query_ids, Q, static_cast<const uint16_t*>(embed), vocab, cx, ctx_off,
+              static_cast<uint16_t*>(packed), max_T, positions);
   } else
-    pack_kernel<float><<<grid, PK_THREADS, 0, st>>>(
-        static_cast<const float*>(X), N, n_v, d, kept, n_kept, sel, sel_off, sys_ids, S, query_ids, Q,
-        static_cast<const uint16_t*>(embed), vocab, cx, ctx_off, static_cast<uint16_t*>(packed), max_T, positions);
+    launch_ex(pack_kernel<float>, grid, dim3(PK_THREADS), 0, st, true, static_cast<const float*>(X), N, n_v, d, kept,
+              n_kept, sel, sel_off, sys_ids, S, query_ids, Q, static_cast<const uint16_t*>(embed), vocab, cx, ctx_off,
+              static_cast<uint16_t*>(packed), max_T, positions);
 }
 
 }  // namespace rift

@@ -19,6 +19,7 @@
 // fp16 rather than bf16 operands: after 32 layers the bf16 rounding of the GEMM inputs alone
 // moves the final hidden states by about 3% of their largest magnitude; fp16 (3 more mantissa
 // bits, same tensor-core rate, LLaVA-1.5-7B's checkpoint dtype) keeps the whole path near 0.5%.
+#include <atomic>
 #include <type_traits>
 
 #include "rift_internal.h"
@@ -36,19 +37,11 @@ unsigned int read_clear_err_prefill() {
 
 constexpr int NORM_THREADS = 256;
 
-// y = h / sqrt(mean(h^2) + eps) * g, one CTA per row.  IN_BF16: h is the bf16 packed input,
-// which is also widened into the fp32 residual stream h32.  OUT_F16: y in fp16 (the GEMM
-// operand); otherwise bf16 (the final hidden states).  VPT: float4 per thread, the fewest that
-// cover d (4 at d = 4096, 8 at the widest d = 8192), so the row held in registers is no larger
-// than the row: fewer registers, more CTAs per SM and more bytes in flight.
+// One row of the RMSNorm below.
 template <bool IN_BF16, bool OUT_F16, int VPT>
-__global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __restrict__ in,
-                                                               float* __restrict__ h32,
-                                                               const uint16_t* __restrict__ gain,
-                                                               uint16_t* __restrict__ out, int d,
-                                                               float eps) {
-  __shared__ float red[32];
-  const size_t row = blockIdx.x;
+__device__ __forceinline__ void rmsnorm_row(const void* __restrict__ in, float* __restrict__ h32,
+                                            const uint16_t* __restrict__ gain, uint16_t* __restrict__ out, int d,
+                                            float eps, size_t row, float* red) {
   const int nv = d / 4;
   float4 v[VPT];
   float ss = 0.f;
@@ -88,6 +81,26 @@ __global__ void __launch_bounds__(NORM_THREADS) rmsnorm_kernel(const void* __res
   }
 }
 
+// y = h / sqrt(mean(h^2) + eps) * g, one row per CTA at a time: rows blockIdx.x, + gridDim.x,
+// ... below the row count (rows_dev: a device count clamped to max_rows, or max_rows itself).
+// IN_BF16: h is the bf16 packed input, which is also widened into the fp32 residual stream h32.
+// OUT_F16: y in fp16 (the GEMM operand); otherwise bf16 (the final hidden states).  VPT: float4
+// per thread, the fewest that cover d (4 at d = 4096, 8 at the widest d = 8192), so the row held
+// in registers is no larger than the row: fewer registers, more CTAs per SM and more bytes in
+// flight.
+template <bool IN_BF16, bool OUT_F16, int VPT>
+__global__ void __launch_bounds__(NORM_THREADS, VPT <= 4 ? 8 : 4) rmsnorm_kernel(const void* __restrict__ in,
+                                                               float* __restrict__ h32,
+                                                               const uint16_t* __restrict__ gain,
+                                                               uint16_t* __restrict__ out, int d,
+                                                               float eps, const int* __restrict__ rows_dev,
+                                                               int max_rows) {
+  __shared__ float red[32];
+  const int n_rows = rows_dev ? max(0, min(max_rows, *rows_dev)) : max_rows;
+  for (size_t row = blockIdx.x; row < (size_t)n_rows; row += gridDim.x)
+    rmsnorm_row<IN_BF16, OUT_F16, VPT>(in, h32, gain, out, d, eps, row, red);
+}
+
 // cos/sin of pos * theta^(-2j/hd), evaluated in double and rounded once to fp32.
 __global__ void rope_table_kernel(float2* __restrict__ tab, int max_len, int half, float theta) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -99,10 +112,12 @@ __global__ void rope_table_kernel(float2* __restrict__ tab, int max_len, int hal
   tab[i] = make_float2((float)c, (float)s);
 }
 
-// KV cache rows: k_out[r] = qkv[r, d .. 2d), v_out[r] = qkv[r, 2d .. 3d) (fp16, heads contiguous).
-__global__ void kv_store_kernel(const uint16_t* __restrict__ qkv, int rows, int d, uint16_t* __restrict__ k_out,
-                                uint16_t* __restrict__ v_out) {
+// KV cache rows: k_out[r] = qkv[r, d .. 2d), v_out[r] = qkv[r, 2d .. 3d) (fp16, heads contiguous),
+// for the rows below the device count rows_dev clamped to rows (all rows without one).
+__global__ void kv_store_kernel(const uint16_t* __restrict__ qkv, int rows, const int* __restrict__ rows_dev, int d,
+                                uint16_t* __restrict__ k_out, uint16_t* __restrict__ v_out) {
   const int nv = d / 8;  // uint4 per row half
+  if (rows_dev) rows = max(0, min(rows, *rows_dev));
   const size_t total = (size_t)rows * 2 * nv;
   for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total; e += (size_t)gridDim.x * blockDim.x) {
     const size_t r = e / (2 * nv);
@@ -115,18 +130,36 @@ __global__ void kv_store_kernel(const uint16_t* __restrict__ qkv, int rows, int 
   }
 }
 
-static void kv_store(const uint16_t* qkv, int rows, int d, uint16_t* k_out, uint16_t* v_out, cudaStream_t st) {
+static void kv_store(const uint16_t* qkv, int rows, const int* rows_dev, int d, uint16_t* k_out, uint16_t* v_out,
+                     cudaStream_t st) {
   const size_t total = (size_t)rows * (d / 4);
   const int grid = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
-  kv_store_kernel<<<grid, 256, 0, st>>>(qkv, rows, d, k_out, v_out);
+  kv_store_kernel<<<grid, 256, 0, st>>>(qkv, rows, rows_dev, d, k_out, v_out);
+}
+
+// Rows T .. T + n_tail - 1 (clamped to the cap rows of the buffer) of an fp16 [cap, cols] buffer
+// set to zero, T = *T_dev.  The attention's last query tile and key block may reach up to 127
+// rows past the last packed row, and a masked key still meets its value row in the P V product,
+// where 0 x NaN = NaN: so the rows past T that the tensor maps can reach must hold finite values
+// (with the row count equal to the capacity they are out of bounds and read as zero instead).
+__global__ void zero_tail_kernel(uint16_t* __restrict__ buf, int cols, const int* __restrict__ T_dev, int cap,
+                                 int n_tail) {
+  const int T = max(0, min(cap, *T_dev));
+  const int rows = min(n_tail, cap - T);
+  const int nv = cols / 8;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < (size_t)rows * nv;
+       e += (size_t)gridDim.x * blockDim.x)
+    reinterpret_cast<uint4*>(buf + (size_t)(T + e / nv) * cols)[e % nv] = make_uint4(0, 0, 0, 0);
 }
 
 // out[i] = h32[cu[i + 1] - 1]: the residual stream of each sequence's last row (zeros for an
-// empty sequence).
-__global__ void last_rows_kernel(const float* __restrict__ h32, const int* __restrict__ cu, int d,
-                                 float* __restrict__ out) {
+// empty sequence, or one that ends past the row_cap rows the buffers hold), for the sequences
+// below the device count n_seq_dev (all gridDim.x of them without one).
+__global__ void last_rows_kernel(const float* __restrict__ h32, const int* __restrict__ cu,
+                                 const int* __restrict__ n_seq_dev, int row_cap, int d, float* __restrict__ out) {
   const int i = blockIdx.x;
-  const bool empty = cu[i + 1] <= cu[i];
+  if (n_seq_dev && i >= *n_seq_dev) return;
+  const bool empty = cu[i + 1] <= cu[i] || cu[i + 1] > row_cap;
   const float4* src = reinterpret_cast<const float4*>(h32 + (size_t)(empty ? 0 : cu[i + 1] - 1) * d);
   float4* dst = reinterpret_cast<float4*>(out + (size_t)i * d);
   for (int c = threadIdx.x; c < d / 4; c += blockDim.x) dst[c] = empty ? make_float4(0.f, 0.f, 0.f, 0.f) : src[c];
@@ -144,7 +177,7 @@ PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int m
   L.act_off = take(T * m.ffn * 2);
   L.rope_off = take((size_t)max_len * (m.head_dim / 2) * sizeof(float2));
   L.max_qblocks = attention_max_qblocks(max_T, max_seqs);
-  L.sched_off = take((size_t)L.max_qblocks * sizeof(int4));
+  L.sched_off = take((size_t)(L.max_qblocks + 1) * sizeof(int4));  // + the entry count
   L.last32_off = take((size_t)max_seqs * m.d * 4);
   L.last16_off = take((size_t)max_seqs * m.d * 2);
   L.total = off;
@@ -159,20 +192,56 @@ int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void
   return r;
 }
 
+static int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+// CTAs of rmsnorm_kernel<IN_BF16, OUT_F16, VPT> resident per SM at once (asked once per
+// instantiation; 1 if the query fails).
+template <bool IN_BF16, bool OUT_F16, int VPT>
+static int norm_resident_ctas() {
+  static std::atomic<int> n{0};
+  int v = n.load(std::memory_order_relaxed);
+  if (v == 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, rmsnorm_kernel<IN_BF16, OUT_F16, VPT>, NORM_THREADS, 0) !=
+            cudaSuccess ||
+        v < 1) {
+      cudaGetLastError();
+      v = 1;
+    }
+    n.store(v, std::memory_order_relaxed);
+  }
+  return v;
+}
+
 // kind 0: packed bf16 input -> h32 + fp16 xn; 1: h32 -> fp16 xn; 2: h32 -> bf16 final output.
+// Rows: min(*rows_dev, T) with a device count, else T.  The grid is four times the CTAs that fit
+// on the GPU at once (8 per SM at d <= 4096), each looping over rows: a CTA that finishes early
+// frees its slot for another, so the last rows spread over the SMs as with one CTA per row.
 static void norm_launch(int kind, int T, const void* in, float* h32, const void* gain, uint16_t* out, int d,
-                        float eps, cudaStream_t st) {
+                        float eps, cudaStream_t st, const int* rows_dev = nullptr) {
   prof_begin(RIFT_PROF_NORM, st);
   const uint16_t* g = static_cast<const uint16_t*>(gain);
   const int per_thread = (d / 4 + NORM_THREADS - 1) / NORM_THREADS;  // d <= 8192: at most 8
   auto go = [&](auto vpt) {
     constexpr int V = decltype(vpt)::value;
+    auto grid = [&](int per_sm) { return T < 4 * per_sm * sm_count() ? T : 4 * per_sm * sm_count(); };
     if (kind == 0)
-      rmsnorm_kernel<true, true, V><<<T, NORM_THREADS, 0, st>>>(in, h32, g, out, d, eps);
+      rmsnorm_kernel<true, true, V><<<grid(norm_resident_ctas<true, true, V>()), NORM_THREADS, 0, st>>>(
+          in, h32, g, out, d, eps, rows_dev, T);
     else if (kind == 1)
-      rmsnorm_kernel<false, true, V><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
+      rmsnorm_kernel<false, true, V><<<grid(norm_resident_ctas<false, true, V>()), NORM_THREADS, 0, st>>>(
+          in, nullptr, g, out, d, eps, rows_dev, T);
     else
-      rmsnorm_kernel<false, false, V><<<T, NORM_THREADS, 0, st>>>(in, nullptr, g, out, d, eps);
+      rmsnorm_kernel<false, false, V><<<grid(norm_resident_ctas<false, false, V>()), NORM_THREADS, 0, st>>>(
+          in, nullptr, g, out, d, eps, rows_dev, T);
   };
   if (per_thread <= 1) go(std::integral_constant<int, 1>{});
   else if (per_thread <= 2) go(std::integral_constant<int, 2>{});
@@ -181,10 +250,10 @@ static void norm_launch(int kind, int T, const void* in, float* h32, const void*
   prof_end(RIFT_PROF_NORM, st, 1);
 }
 
-int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                   int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
-                   cudaStream_t st, const void* prefix_kv, int S_pre) {
-  if (T == 0) return 0;
+int launch_prefill(const rift_model& m, void* hidden, int T, const int* T_dev, const int* cu_seqlens, int n_seq,
+                   const int* n_seq_dev, int max_len, const int* positions, void* kv_out, float* last_logits,
+                   char* ws, cudaStream_t st, const void* prefix_kv, int S_pre) {
+  if (T == 0 || n_seq == 0) return 0;
   const PrefillLayout L = prefill_layout(m, T, n_seq, max_len);
   float* h32 = reinterpret_cast<float*>(ws + L.h32_off);
   uint16_t* xn = reinterpret_cast<uint16_t*>(ws + L.xn_off);
@@ -199,9 +268,13 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   rope_table_kernel<<<(max_len * half + 255) / 256, 256, 0, st>>>(rope, max_len, half, m.rope_theta);
   prof_end(RIFT_PROF_ROPE, st, 1);
   prof_begin(RIFT_PROF_ATTN, st);
-  launch_attention_schedule(cu_seqlens, n_seq, sched, L.max_qblocks, st);
-  prof_end(RIFT_PROF_ATTN, st, 1);
-  EpiParams rope_ep;
+  launch_attention_schedule(cu_seqlens, n_seq, n_seq_dev, T, sched, L.max_qblocks, st);
+  if (T_dev) zero_tail_kernel<<<64, 256, 0, st>>>(qkv, 3 * d, T_dev, T, 128);
+  prof_end(RIFT_PROF_ATTN, st, T_dev ? 2 : 1);
+  // every product covers the rows the device count holds (T rows of capacity)
+  EpiParams rows_ep;
+  rows_ep.m_dev = T_dev;
+  EpiParams rope_ep = rows_ep;
   rope_ep.positions = positions;
   rope_ep.rope = rope;
   rope_ep.rope_cols = 2 * d;
@@ -210,13 +283,13 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
   rope_ep.pos_offset = S_pre;
   for (int l = 0; l < m.n_layers; ++l) {
     if (l == 0)
-      norm_launch(0, T, hidden, h32, m.g_attn[0], xn, d, m.eps, st);
+      norm_launch(0, T, hidden, h32, m.g_attn[0], xn, d, m.eps, st, T_dev);
     else
-      norm_launch(1, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st);
+      norm_launch(1, T, h32, nullptr, m.g_attn[l], xn, d, m.eps, st, T_dev);
     if (launch_gemm(xn, m.w_qkv[l], T, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep)) return 1;
     if (kv_out) {
       uint16_t* kl = static_cast<uint16_t*>(kv_out) + (size_t)l * 2 * T * d;
-      kv_store(qkv, T, d, kl, kl + (size_t)T * d, st);
+      kv_store(qkv, T, T_dev, d, kl, kl + (size_t)T * d, st);
     }
     prof_begin(RIFT_PROF_ATTN, st);
     const uint16_t* pk = prefix_kv ? static_cast<const uint16_t*>(prefix_kv) + (size_t)l * 2 * S_pre * d : nullptr;
@@ -224,18 +297,20 @@ int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqle
                          pk ? pk + (size_t)S_pre * d : nullptr, prefix_kv ? S_pre : 0))
       return 1;
     prof_end(RIFT_PROF_ATTN, st, 1);
-    if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st)) return 1;
-    norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st);
-    if (launch_gemm(xn, m.w_gate_up[l], T, 2 * m.ffn, d, EPI_SWIGLU, act, st)) return 1;
-    if (launch_gemm(act, m.w_down[l], T, d, m.ffn, EPI_RESID_F32, h32, st)) return 1;
+    if (launch_gemm(att, m.w_o[l], T, d, d, EPI_RESID_F32, h32, st, rows_ep)) return 1;
+    norm_launch(1, T, h32, nullptr, m.g_ffn[l], xn, d, m.eps, st, T_dev);
+    if (launch_gemm(xn, m.w_gate_up[l], T, 2 * m.ffn, d, EPI_SWIGLU, act, st, rows_ep)) return 1;
+    if (launch_gemm(act, m.w_down[l], T, d, m.ffn, EPI_RESID_F32, h32, st, rows_ep)) return 1;
   }
-  norm_launch(2, T, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden), d, m.eps, st);
+  norm_launch(2, T, h32, nullptr, m.g_final, static_cast<uint16_t*>(hidden), d, m.eps, st, T_dev);
   if (last_logits) {
     float* last32 = reinterpret_cast<float*>(ws + L.last32_off);
     uint16_t* last16 = reinterpret_cast<uint16_t*>(ws + L.last16_off);
-    last_rows_kernel<<<n_seq, 256, 0, st>>>(h32, cu_seqlens, d, last32);
-    norm_launch(1, n_seq, last32, nullptr, m.g_final, last16, d, m.eps, st);
-    if (launch_gemm(last16, m.lm_head, n_seq, m.vocab, d, EPI_STORE_F32, last_logits, st)) return 1;
+    last_rows_kernel<<<n_seq, 256, 0, st>>>(h32, cu_seqlens, n_seq_dev, T, d, last32);
+    norm_launch(1, n_seq, last32, nullptr, m.g_final, last16, d, m.eps, st, n_seq_dev);
+    EpiParams seq_ep;
+    seq_ep.m_dev = n_seq_dev;
+    if (launch_gemm(last16, m.lm_head, n_seq, m.vocab, d, EPI_STORE_F32, last_logits, st, seq_ep)) return 1;
   }
   return 0;
 }
@@ -279,9 +354,9 @@ SharedPrefixLayout shared_prefix_layout(const rift_model& m, int max_T, int max_
 }
 
 int launch_prefill_shared_prefix(const rift_model& m, const int* sys_ids, int S, const void* embed, int vocab,
-                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
-                                 int n_seq, int max_len, const int* positions, float* last_logits, char* ws,
-                                 cudaStream_t st) {
+                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* T_dev,
+                                 const int* cu_seqlens, int n_seq, const int* n_seq_dev, int max_len,
+                                 const int* positions, float* last_logits, char* ws, cudaStream_t st) {
   const SharedPrefixLayout L = shared_prefix_layout(m, T, n_seq, max_len, S);
   int* cu_pre = reinterpret_cast<int*>(ws + L.cu_off);
   int* pos_pre = reinterpret_cast<int*>(ws + L.pos_off);
@@ -289,9 +364,10 @@ int launch_prefill_shared_prefix(const rift_model& m, const int* sys_ids, int S,
                                         static_cast<uint16_t*>(prefix_hidden), cu_pre, pos_pre);
   // the prefix as one sequence, keeping its cache; then the suffixes over it (the two share the
   // prefill workspace: they run in order on the stream)
-  if (launch_prefill(m, prefix_hidden, S, cu_pre, 1, max_len, pos_pre, prefix_kv, nullptr, ws, st)) return 1;
-  if (T > 0 && launch_prefill(m, hidden, T, cu_seqlens, n_seq, max_len, positions, nullptr, last_logits, ws, st,
-                              prefix_kv, S))
+  if (launch_prefill(m, prefix_hidden, S, nullptr, cu_pre, 1, nullptr, max_len, pos_pre, prefix_kv, nullptr, ws, st))
+    return 1;
+  if (T > 0 && launch_prefill(m, hidden, T, T_dev, cu_seqlens, n_seq, n_seq_dev, max_len, positions, nullptr,
+                              last_logits, ws, st, prefix_kv, S))
     return 1;
   return 0;
 }
@@ -540,7 +616,7 @@ int launch_decode(const rift_model& m, const void* kv_cache, int T, const int* c
     if (launch_gemm(xn, m.w_qkv[l], n, 3 * d, d, EPI_QKV_ROPE, qkv, st, rope_ep, split, sb, pdl)) return 1;
     if (kv_new) {
       uint16_t* kl = static_cast<uint16_t*>(kv_new) + (size_t)l * 2 * n * d;
-      kv_store(qkv, n, d, kl, kl + (size_t)n * d, st);
+      kv_store(qkv, n, nullptr, d, kl, kl + (size_t)n * d, st);
     }
     const uint16_t* Kc = kv + (size_t)l * 2 * T * d;
     const uint16_t* Vc = Kc + (size_t)T * d;

@@ -66,6 +66,17 @@ void prof_end(int cls, cudaStream_t st, int n) {
   g_open[cls] = nullptr;
 }
 
+rift_status score_args_check(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                             int M, int knn_m, const float* token_scores, const float* tile_s_raw,
+                             const float* tile_s) {
+  if (!dims_ok(N, n_v, d) || !X || !t || !token_scores || !tile_s_raw || !tile_s) return RIFT_ERR_INVALID;
+  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
+  if (xdt == RIFT_F32 && d > 4096) return RIFT_ERR_UNSUPPORTED;
+  if (M < 0 || M > 64 || (M > 0 && !B) || knn_m < 0 || knn_m > RIFT_MAX_KNN) return RIFT_ERR_INVALID;
+  if (!aligned16(X)) return RIFT_ERR_INVALID;
+  return RIFT_OK;
+}
+
 }  // namespace rift
 
 extern "C" {
@@ -98,7 +109,7 @@ rift_status rift_profile_read(double* ms, long long* launches, int n_classes) {
 
 long long rift_launch_count(void) { return g_launches.load(); }
 
-int rift_abi_version(void) { return 4; }
+int rift_abi_version(void) { return 5; }
 
 const char* rift_status_string(rift_status s) {
   switch (s) {
@@ -148,11 +159,8 @@ size_t rift_score_workspace_bytes(int N, int n_v, int d, int M) {
 rift_status rift_score_tiles(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t,
                              const float* B, int M, int knn_m, float* token_scores, float* tile_s_raw,
                              float* tile_s, int* nbr, void* ws, size_t ws_bytes, rift_stream_t stream) {
-  if (!dims_ok(N, n_v, d) || !X || !t || !token_scores || !tile_s_raw || !tile_s) return RIFT_ERR_INVALID;
-  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
-  if (xdt == RIFT_F32 && d > 4096) return RIFT_ERR_UNSUPPORTED;
-  if (M < 0 || M > 64 || (M > 0 && !B) || knn_m < 0 || knn_m > RIFT_MAX_KNN) return RIFT_ERR_INVALID;
-  if (!aligned16(X)) return RIFT_ERR_INVALID;
+  const rift_status chk = score_args_check(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_raw, tile_s);
+  if (chk != RIFT_OK) return chk;
   const size_t need = rift_score_workspace_bytes(N, n_v, d, M);
   if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
   const int m = std::min(knn_m, N - 1);
@@ -171,12 +179,9 @@ size_t rift_select_workspace_bytes(int N, int n_v) {
   return 0;
 }
 
-rift_status rift_select_budgeted_tokens(const float* token_scores, const float* tile_s, int N, int n_v,
-                                        const float* p, const rift_policy* policy, float* u, int* kept,
-                                        int* n_kept, int* budgets, int* sel, int* sel_off, void* ws,
-                                        size_t ws_bytes, rift_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
+static rift_status select_args_check(const float* token_scores, const float* tile_s, int N, int n_v,
+                                     const rift_policy* policy, const float* u, const int* kept, const int* n_kept,
+                                     const int* budgets, const int* sel, const int* sel_off) {
   if (!token_scores || !tile_s || !policy || !u || !kept || !n_kept || !budgets || !sel || !sel_off)
     return RIFT_ERR_INVALID;
   if (N < 1 || N > RIFT_MAX_TILES || n_v < 1 || n_v > RIFT_MAX_NV) return RIFT_ERR_INVALID;
@@ -191,9 +196,92 @@ rift_status rift_select_budgeted_tokens(const float* token_scores, const float* 
   }
   if (!std::isfinite(pol.lambda)) return RIFT_ERR_INVALID;
   if (pol.ctx_num < 0 || pol.ctx_den < 1 || pol.ctx_num >= pol.ctx_den) return RIFT_ERR_INVALID;
+  return RIFT_OK;
+}
+
+rift_status rift_select_budgeted_tokens(const float* token_scores, const float* tile_s, int N, int n_v,
+                                        const float* p, const rift_policy* policy, float* u, int* kept,
+                                        int* n_kept, int* budgets, int* sel, int* sel_off, void* ws,
+                                        size_t ws_bytes, rift_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  const rift_status chk =
+      select_args_check(token_scores, tile_s, N, n_v, policy, u, kept, n_kept, budgets, sel, sel_off);
+  if (chk != RIFT_OK) return chk;
   prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
-  launch_select(token_scores, tile_s, N, n_v, p, pol, u, kept, n_kept, budgets, sel, sel_off,
+  launch_select(token_scores, tile_s, N, n_v, p, *policy, u, kept, n_kept, budgets, sel, sel_off,
                 static_cast<cudaStream_t>(stream));
+  prof_end(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream), 2);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+// ---- one scene sharded over several ranks (a shard of its tiles per rank) ----
+
+size_t rift_score_shard_workspace_bytes(int N_local, int n_v, int d) {
+  if (!dims_ok(N_local, n_v, d)) return 0;
+  return shard_layout(N_local, n_v, d).total;
+}
+
+rift_status rift_score_shard(const void* X, rift_dtype xdt, int N_local, int n_v, int d, const float* t,
+                             const float* B, int M, float* token_scores, float* tile_s_raw, float* V, void* ws,
+                             size_t ws_bytes, rift_stream_t stream) {
+  if (!V) return RIFT_ERR_INVALID;
+  const rift_status chk = score_args_check(X, xdt, N_local, n_v, d, t, B, M, 0, token_scores, tile_s_raw, V);
+  if (chk != RIFT_OK) return chk;
+  if (!ws_ok(ws, ws_bytes, rift_score_shard_workspace_bytes(N_local, n_v, d))) return RIFT_ERR_INVALID;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  prof_begin(RIFT_PROF_SCORE, st);
+  const int nk = launch_score_tokens(X, xdt, N_local, n_v, d, t, B, M, token_scores, tile_s_raw, V,
+                                     static_cast<char*>(ws), st);
+  prof_end(RIFT_PROF_SCORE, st, nk);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+size_t rift_smooth_workspace_bytes(int N, int n_rows, int d) {
+  if (N < 1 || N > RIFT_MAX_TILES || n_rows < 1 || n_rows > N || d < 64 || d > 8192 || d % 64 != 0) return 0;
+  return smooth_layout(N, n_rows, d).total;
+}
+
+rift_status rift_smooth_rows(const float* V, const float* tile_s_raw, int N, int d, int row0, int n_rows, int knn_m,
+                             float* tile_s, int* nbr, void* ws, size_t ws_bytes, rift_stream_t stream) {
+  if (!V || !tile_s_raw || !tile_s || N < 1 || N > RIFT_MAX_TILES || d < 64 || d > 8192 || d % 64 != 0)
+    return RIFT_ERR_INVALID;
+  if (row0 < 0 || n_rows < 1 || row0 + n_rows > N || knn_m < 0 || knn_m > RIFT_MAX_KNN) return RIFT_ERR_INVALID;
+  if (!aligned16(V)) return RIFT_ERR_INVALID;
+  if (!ws_ok(ws, ws_bytes, rift_smooth_workspace_bytes(N, n_rows, d))) return RIFT_ERR_INVALID;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int m = std::min(knn_m, N - 1);
+  prof_begin(RIFT_PROF_SCORE, st);
+  const int nk = launch_smooth(V, tile_s_raw, N, d, row0, n_rows, m, tile_s, nbr, static_cast<char*>(ws), st);
+  prof_end(RIFT_PROF_SCORE, st, nk < 0 ? 0 : nk);
+  if (nk < 0) return RIFT_ERR_CUDA;
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+rift_status rift_score_range(const float* tile_s, int n, float* range, rift_stream_t stream) {
+  if (!tile_s || !range || n < 1 || n > RIFT_MAX_TILES) return RIFT_ERR_INVALID;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  prof_begin(RIFT_PROF_SELECT, st);
+  launch_score_range(tile_s, n, range, st);
+  prof_end(RIFT_PROF_SELECT, st, 1);
+  RIFT_LAUNCH_CHECK();
+  return RIFT_OK;
+}
+
+rift_status rift_select_budgeted_tokens_ranged(const float* token_scores, const float* tile_s, int N, int n_v,
+                                               const float* s_range, const float* p, const rift_policy* policy,
+                                               float* u, int* kept, int* n_kept, int* budgets, int* sel,
+                                               int* sel_off, rift_stream_t stream) {
+  if (!s_range) return RIFT_ERR_INVALID;
+  const rift_status chk =
+      select_args_check(token_scores, tile_s, N, n_v, policy, u, kept, n_kept, budgets, sel, sel_off);
+  if (chk != RIFT_OK) return chk;
+  prof_begin(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream));
+  launch_select(token_scores, tile_s, N, n_v, p, *policy, u, kept, n_kept, budgets, sel, sel_off,
+                static_cast<cudaStream_t>(stream), s_range);
   prof_end(RIFT_PROF_SELECT, static_cast<cudaStream_t>(stream), 2);
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
@@ -309,18 +397,18 @@ static bool lm_head_ok(const rift_model* m) {
   return m->lm_head && aligned16(m->lm_head) && m->vocab >= 8 && m->vocab % 8 == 0;
 }
 
-rift_status rift_prefill_layers(const rift_model* m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                                int max_len, const int* positions, void* kv_out, float* last_logits, void* ws,
-                                size_t ws_bytes, rift_stream_t stream) {
-  if (!model_ok(m) || !hidden || !cu_seqlens || !positions || T < 0 || n_seq < 0 || max_len < 1)
+rift_status rift_prefill_layers(const rift_model* m, void* hidden, const int* T, int max_T, const int* cu_seqlens,
+                                const int* n_seq, int max_seqs, int max_len, const int* positions, void* kv_out,
+                                float* last_logits, void* ws, size_t ws_bytes, rift_stream_t stream) {
+  if (!model_ok(m) || !hidden || !cu_seqlens || !positions || max_T < 0 || max_seqs < 0 || max_len < 1)
     return RIFT_ERR_INVALID;
-  if (T > 0 && n_seq < 1) return RIFT_ERR_INVALID;
+  if (max_T > 0 && max_seqs < 1) return RIFT_ERR_INVALID;
   if (!aligned16(hidden) || (kv_out && !aligned16(kv_out)) || (last_logits && !aligned16(last_logits)))
     return RIFT_ERR_INVALID;
   if (last_logits && !lm_head_ok(m)) return RIFT_ERR_INVALID;
-  const size_t need = prefill_layout(*m, T, n_seq, max_len).total;
+  const size_t need = prefill_layout(*m, max_T, max_seqs, max_len).total;
   if (!ws_ok(ws, ws_bytes, need)) return RIFT_ERR_INVALID;
-  if (launch_prefill(*m, hidden, T, cu_seqlens, n_seq, max_len, positions, kv_out, last_logits,
+  if (launch_prefill(*m, hidden, max_T, T, cu_seqlens, max_seqs, n_seq, max_len, positions, kv_out, last_logits,
                      static_cast<char*>(ws), static_cast<cudaStream_t>(stream)))
     return RIFT_ERR_INVALID;
   RIFT_LAUNCH_CHECK();
@@ -333,21 +421,22 @@ size_t rift_prefill_shared_prefix_workspace_bytes(const rift_model* m, int max_T
 }
 
 rift_status rift_prefill_shared_prefix(const rift_model* m, const int* sys_ids, int S, const void* embed, int vocab,
-                                       void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
-                                       int n_seq, int max_len, const int* positions, float* last_logits, void* ws,
-                                       size_t ws_bytes, rift_stream_t stream) {
-  if (!model_ok(m) || !sys_ids || !embed || !prefix_hidden || !prefix_kv || S < 1 || vocab < 1 || T < 0 ||
-      n_seq < 0 || max_len < 1 || S > max_len)
+                                       void* prefix_hidden, void* prefix_kv, void* hidden, const int* T, int max_T,
+                                       const int* cu_seqlens, const int* n_seq, int max_seqs, int max_len,
+                                       const int* positions, float* last_logits, void* ws, size_t ws_bytes,
+                                       rift_stream_t stream) {
+  if (!model_ok(m) || !sys_ids || !embed || !prefix_hidden || !prefix_kv || S < 1 || vocab < 1 || max_T < 0 ||
+      max_seqs < 0 || max_len < 1 || S > max_len)
     return RIFT_ERR_INVALID;
-  if (T > 0 && (!hidden || !cu_seqlens || !positions || n_seq < 1)) return RIFT_ERR_INVALID;
+  if (max_T > 0 && (!hidden || !cu_seqlens || !positions || max_seqs < 1)) return RIFT_ERR_INVALID;
   if (!aligned16(embed) || !aligned16(prefix_hidden) || !aligned16(prefix_kv) || (hidden && !aligned16(hidden)) ||
       (last_logits && !aligned16(last_logits)))
     return RIFT_ERR_INVALID;
   if (last_logits && !lm_head_ok(m)) return RIFT_ERR_INVALID;
-  if (!ws_ok(ws, ws_bytes, shared_prefix_layout(*m, T, n_seq, max_len, S).total)) return RIFT_ERR_INVALID;
-  if (launch_prefill_shared_prefix(*m, sys_ids, S, embed, vocab, prefix_hidden, prefix_kv, hidden, T, cu_seqlens,
-                                   n_seq, max_len, positions, last_logits, static_cast<char*>(ws),
-                                   static_cast<cudaStream_t>(stream)))
+  if (!ws_ok(ws, ws_bytes, shared_prefix_layout(*m, max_T, max_seqs, max_len, S).total)) return RIFT_ERR_INVALID;
+  if (launch_prefill_shared_prefix(*m, sys_ids, S, embed, vocab, prefix_hidden, prefix_kv, hidden, max_T, T,
+                                   cu_seqlens, max_seqs, n_seq, max_len, positions, last_logits,
+                                   static_cast<char*>(ws), static_cast<cudaStream_t>(stream)))
     return RIFT_ERR_INVALID;
   RIFT_LAUNCH_CHECK();
   return RIFT_OK;
@@ -391,8 +480,8 @@ rift_status rift_linear(const void* A, const void* W, int M, int N, int K, int e
 }
 
 size_t rift_attention_workspace_bytes(int max_T, int max_seqs) {
-  if (max_T < 0 || max_seqs < 0) return 0;
-  return (size_t)attention_max_qblocks(max_T, max_seqs) * sizeof(int4);
+  if (max_T <= 0 || max_seqs < 0) return 0;  // no rows: nothing to schedule
+  return (size_t)(attention_max_qblocks(max_T, max_seqs) + 1) * sizeof(int4);
 }
 
 rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads,
@@ -408,7 +497,7 @@ rift_status rift_attention_varlen(const void* qkv, int T, const int* cu_seqlens,
   int4* sched = static_cast<int4*>(ws);
   const int n_max = attention_max_qblocks(T, n_seq);
   prof_begin(RIFT_PROF_ATTN, st);
-  launch_attention_schedule(cu_seqlens, n_seq, sched, n_max, st);
+  launch_attention_schedule(cu_seqlens, n_seq, nullptr, T, sched, n_max, st);
   if (launch_attention(qkv, T, cu_seqlens, n_seq, n_heads, head_dim, sched, n_max, out, st)) return RIFT_ERR_CUDA;
   prof_end(RIFT_PROF_ATTN, st, 2);
   RIFT_LAUNCH_CHECK();

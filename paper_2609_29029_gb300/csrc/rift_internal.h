@@ -18,24 +18,50 @@ unsigned int read_clear_err_prefill();
 unsigned int read_clear_err_gemm();
 
 // ---- score.cu ----
+// The token pass over N tiles (Eq. 1 per token, pooled sums): w and the partial pooled sums.
+struct ShardLayout {
+  int chunk_tokens, n_chunks;
+  size_t w_off, ppart_off, total;
+};
+ShardLayout shard_layout(int N, int n_v, int d);
+// The kNN smoothing of n_rows rows against all N tiles (Appendix B Step 2).
+struct SmoothLayout {
+  size_t top_off, split_a_off, split_b_off, gram_off, splitk_off, splitk_bytes, total;
+};
+SmoothLayout smooth_layout(int N, int n_rows, int d);
+// rift_score_tiles: the token pass, then V [N, d], then the smoothing of all N rows.
 struct ScoreLayout {
-  int chunk_tokens, n_chunks, n_jblk, n_split;
-  size_t w_off, ppart_off, V_off, cand_g_off, cand_j_off, top_off, gpart_off, split_a_off, split_b_off, gram_off,
-      total;
-  bool tensor_gram;  // N > 1024: the Gram matrix on the tensor cores (fp16 hi/lo split)
+  ShardLayout T;
+  SmoothLayout S;
+  size_t V_off, smooth_off, total;
 };
 ScoreLayout score_layout(int N, int n_v, int d, int M);
+// The host-side argument checks shared by the scoring entry points (rift_score_tiles and
+// rift_score_tiles_noalloc): RIFT_OK, or the status the call returns without launching.
+rift_status score_args_check(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                             int M, int knn_m, const float* token_scores, const float* tile_s_raw,
+                             const float* tile_s);
 int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st);
 // Returns the number of kernels launched, or -1 if a launch could not be set up.
 int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
                  int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
                  cudaStream_t st);
+// a2, a3 on N tiles: token scores, tile scores and the tile embeddings V [N, d] (ws: shard_layout).
+int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st);
+// a4 for tiles row0 .. row0 + n_rows - 1 of a scene of N tiles (V [N, d], s_raw [N]); s_tilde and
+// nbr are indexed by the local row (ws: smooth_layout).
+int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, int n_rows, int m, float* s_tilde,
+                  int* nbr, char* ws, cudaStream_t st);
+// range = (min, max) of n scores.
+void launch_score_range(const float* s, int n, float* range, cudaStream_t st);
 
 // ---- select.cu ----
+// s_range (nullable): the scene's (min, max) of tile_s, when the N tiles are a shard of it.
 void launch_select(const float* token_scores, const float* tile_s, int N, int n_v, const float* p,
                    const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
-                   int* sel_off, cudaStream_t st);
+                   int* sel_off, cudaStream_t st, const float* s_range = nullptr);
 
 // ---- features.cu ----
 struct FeaturesLayout {
@@ -71,19 +97,22 @@ struct PrefillLayout {
   int max_qblocks;
 };
 PrefillLayout prefill_layout(const rift_model& m, int max_T, int max_seqs, int max_len);
+// T, n_seq: the row and sequence capacities (host); T_dev, n_seq_dev (nullable): the device
+// counts the launches read, clamped to the capacities (without them, T and n_seq are the counts).
+// The kv_out layout [n_layers][2][T][d] uses the capacity T as its row stride.
 // prefix_kv (optional): fp16 [n_layers][2][S_pre][d] cache of a prefix shared by every sequence
 // (each sequence's rows attend to it first; their positions are positions[] + S_pre).
-int launch_prefill(const rift_model& m, void* hidden, int T, const int* cu_seqlens, int n_seq,
-                   int max_len, const int* positions, void* kv_out, float* last_logits, char* ws,
-                   cudaStream_t st, const void* prefix_kv = nullptr, int S_pre = 0);
+int launch_prefill(const rift_model& m, void* hidden, int T, const int* T_dev, const int* cu_seqlens, int n_seq,
+                   const int* n_seq_dev, int max_len, const int* positions, void* kv_out, float* last_logits,
+                   char* ws, cudaStream_t st, const void* prefix_kv = nullptr, int S_pre = 0);
 struct SharedPrefixLayout {
   size_t prefill_bytes, cu_off, pos_off, total;
 };
 SharedPrefixLayout shared_prefix_layout(const rift_model& m, int max_T, int max_seqs, int max_len, int S);
 int launch_prefill_shared_prefix(const rift_model& m, const int* sys_ids, int S, const void* embed, int vocab,
-                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* cu_seqlens,
-                                 int n_seq, int max_len, const int* positions, float* last_logits, char* ws,
-                                 cudaStream_t st);
+                                 void* prefix_hidden, void* prefix_kv, void* hidden, int T, const int* T_dev,
+                                 const int* cu_seqlens, int n_seq, const int* n_seq_dev, int max_len,
+                                 const int* positions, float* last_logits, char* ws, cudaStream_t st);
 struct DecodeLayout {
   size_t h32_off, x0_off, xn_off, qkv_off, attn_off, act_off, rope_off, pos_off, dpart_off, split_off, split_bytes,
       total;
@@ -114,6 +143,9 @@ struct EpiParams {
   const void* norm_gain = nullptr;
   uint16_t* norm_out = nullptr;
   float norm_eps = 0.f;
+  // Device row count (nullable): the product covers rows min(M, *m_dev); M is then the capacity
+  // the operands and the output are sized for.  Not used with split-K.
+  const int* m_dev = nullptr;
 };
 // split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
 // most SMs idle run as (tile, K-slice) units plus a reduction kernel.
@@ -121,8 +153,11 @@ struct EpiParams {
 int launch_gemm(const void* A, const void* B, int M, int N, int K, int epi, void* C,
                 cudaStream_t st, const EpiParams& ep = EpiParams(), void* split_ws = nullptr,
                 size_t split_ws_bytes = 0, bool pdl = false);
+// b_const: B does not depend on earlier kernels (constant weights), so a programmatic dependent
+// launch may request its first tiles before waiting for the kernel before it.
 int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, void* C, const EpiParams& ep,
-                   cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0, bool pdl = false);
+                   cudaStream_t st, void* split_ws = nullptr, size_t split_ws_bytes = 0, bool pdl = false,
+                   bool b_const = true);
 int launch_wait_timeout_check(cudaStream_t st);
 // Merge screening on the tensor cores (bf16 tokens): per kept slot and 128-token block, the two
 // best merge targets (by x.t / ||t||) of every unselected non-target token.  targets: bf16
@@ -135,7 +170,10 @@ int launch_merge_screen(const uint16_t* X, int N, int n_v, int d, const int* kep
 // Varlen causal attention (attention_tc.cu): q-block schedule built once per prefill from
 // cu_seqlens, then one launch per layer.  qkv fp16 [T, 3 d], out fp16 [T, d].
 int attention_max_qblocks(int max_T, int max_seqs);
-void launch_attention_schedule(const int* cu_seqlens, int n_seq, int4* sched, int n_sched_max, cudaStream_t st);
+// The schedule holds n_sched_max + 1 entries (the last: the count in use).  n_seq_dev (nullable):
+// a device sequence count clamped to n_seq; sequences ending past row_cap rows are dropped.
+void launch_attention_schedule(const int* cu_seqlens, int n_seq, const int* n_seq_dev, int row_cap, int4* sched,
+                               int n_sched_max, cudaStream_t st);
 // prefix_k, prefix_v (optional): fp16 [S_pre, d] keys (after RoPE) and values of a prefix that every
 // sequence attends to before its own rows.
 int launch_attention(const void* qkv, int T, const int* cu_seqlens, int n_seq, int n_heads, int head_dim,

@@ -85,6 +85,8 @@ __global__ void query_rows_kernel(const uint16_t* __restrict__ embed, int vocab,
                                   const int* __restrict__ phrase_ids, int n_phrase,
                                   const int* __restrict__ bg_ids, int M, float* __restrict__ t,
                                   float* __restrict__ B) {
+  pdl_trigger();
+  pdl_wait();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= d) return;
   float s = 0.f;
@@ -107,6 +109,8 @@ __global__ void query_rows_kernel(const uint16_t* __restrict__ embed, int vocab,
 
 // Row r of {t, B_0, ..., B_{M-1}} divided by its length (zero rows stay zero).
 __global__ void __launch_bounds__(256) normalize_rows_kernel(float* __restrict__ t, float* __restrict__ B, int d) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   float* row = blockIdx.x == 0 ? t : B + (size_t)(blockIdx.x - 1) * d;
   float ss = 0.f;
@@ -119,6 +123,8 @@ __global__ void __launch_bounds__(256) normalize_rows_kernel(float* __restrict__
 // w = t - (1/M) sum_j B_j  (M = 0: w = t)
 __global__ void fold_w_kernel(const float* __restrict__ t, const float* __restrict__ B, int M,
                               int d, float* __restrict__ w) {
+  pdl_trigger();
+  pdl_wait();
   int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= d) return;
   float s = 0.f;
@@ -174,6 +180,8 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
     token_score_kernel(const XT* __restrict__ X, int n_v, int d, int chunk_tokens, int n_chunks,
                        const float* __restrict__ w, float* __restrict__ token_scores,
                        float* __restrict__ Ppart) {
+  pdl_trigger();
+  pdl_wait();
   using VT = VecTraits<XT>;
   constexpr int VW = VT::W;
   constexpr int GROUP = (NVEC <= 2) ? SC_GROUP : SC_GROUP / 2;  // raw loads: GROUP*NVEC*4 regs
@@ -257,172 +265,76 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
   }
 }
 
-// a3: P_i = sum of the tile's partials (fixed order), V_i = P_i / ||P_i||, s_i = V_i . w.
-__global__ void __launch_bounds__(256) tile_finalize_kernel(const float* __restrict__ Ppart,
-                                                            int n_chunks, int d,
-                                                            const float* __restrict__ w,
-                                                            float* __restrict__ V,
-                                                            float* __restrict__ s_raw) {
-  extern __shared__ float tf_sm[];
+// a3: P_i = sum of the tile's partials (fixed order), V_i = P_i / ||P_i||, s_i = V_i . w.  One CTA
+// per tile, a float4 column per thread (two at d > 4096), so that each thread's partial loads all
+// issue together.
+constexpr int TF_THREADS = 1024;
+__global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart,
+                                                                  int n_chunks, int d,
+                                                                  const float* __restrict__ w,
+                                                                  float* __restrict__ V,
+                                                                  float* __restrict__ s_raw) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
-  const int i = blockIdx.x;
+  const int i = blockIdx.x, nv = d / 4;
+  float4 p[2];
   float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    float p = 0.f;
-    for (int q = 0; q < n_chunks; ++q) p += Ppart[((size_t)i * n_chunks + q) * d + c];
-    tf_sm[c] = p;
-    ss += p * p;
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int c = threadIdx.x + k * TF_THREADS;
+    p[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c < nv) {
+      const float4* src = reinterpret_cast<const float4*>(Ppart + (size_t)i * n_chunks * d) + c;
+      for (int q = 0; q < n_chunks; ++q) {
+        const float4 v = src[(size_t)q * nv];
+        p[k].x += v.x;
+        p[k].y += v.y;
+        p[k].z += v.z;
+        p[k].w += v.w;
+      }
+      ss += p[k].x * p[k].x + p[k].y * p[k].y + p[k].z * p[k].z + p[k].w * p[k].w;
+    }
   }
-  float inv = 1.f / sqrtf(block_sum(ss, red));
+  const float inv = 1.f / sqrtf(block_sum(ss, red));
   float dt = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    float v = tf_sm[c] * inv;
-    V[(size_t)i * d + c] = v;
-    dt += v * w[c];
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int c = threadIdx.x + k * TF_THREADS;
+    if (c < nv) {
+      const float4 v = make_float4(p[k].x * inv, p[k].y * inv, p[k].z * inv, p[k].w * inv);
+      reinterpret_cast<float4*>(V + (size_t)i * d)[c] = v;
+      const float4 wc = reinterpret_cast<const float4*>(w)[c];
+      dt += v.x * wc.x + v.y * wc.y + v.z * wc.z + v.w * wc.w;
+    }
   }
   dt = block_sum(dt, red);
   if (threadIdx.x == 0) s_raw[i] = dt;
 }
 
 // ------------------------------------------------------------------------------------------
-// a4: G = V V^T in 64 x 64 blocks (fp32, k ascending, 32-term chunks).  Small scenes split K
-// across CTAs and knn_row_topc_kernel picks each row's top-C from the summed slices; large ones
-// keep a top-C list per block and knn_merge_kernel merges a row's lists.  Then
-// knn_rescore_smooth_kernel recomputes the C candidates to ~fp64 accuracy, keeps the top m and
-// smooths.
+// a4: each row's C candidate neighbours from an approximate Gram matrix G = V V^T on the tensor
+// cores, then knn_rescore_smooth_kernel recomputes the C candidates to ~fp64 accuracy, keeps the
+// top m and smooths.
 // ------------------------------------------------------------------------------------------
-constexpr int KB = 64;   // rows (i) and columns (j) per block
-constexpr int KNN_SPARE = 10;  // fp32 candidates kept beyond m for the fp64 rescoring
-constexpr int KK = 32;   // d-chunk
+constexpr int KNN_SPARE = 10;  // candidates kept beyond m for the fp64 rescoring
 
 // (g, j) beats (g2, j2): larger similarity first, then the lower index.
 __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
   return g > g2 || (g == g2 && j < j2);
 }
 
-// grid (column blocks, row blocks, K slices).  With one slice the kernel also extracts each
-// row's top-C of the block (m here is C); with several it writes its partial similarities to
-// Gpart[slice][i][j] for knn_row_topc_kernel.
-__global__ void __launch_bounds__(256) knn_block_kernel(const float* __restrict__ V, int N, int d,
-                                                        int m, float* __restrict__ cand_g,
-                                                        int* __restrict__ cand_j,
-                                                        float* __restrict__ Gpart) {
-  __shared__ float As[KK][KB + 4];
-  __shared__ float Bs[KK][KB + 4];
-  __shared__ float Gs[KB][KB + 1];
-  const int i0 = blockIdx.y * KB, j0 = blockIdx.x * KB;
-  const int tid = threadIdx.x, ti = tid >> 4, tj = tid & 15;
-  const int kslice = d / gridDim.z;
-  const int kbeg = blockIdx.z * kslice, kend = kbeg + kslice;
-  float acc[4][4] = {};
-  for (int k0 = kbeg; k0 < kend; k0 += KK) {
-    // 64 rows x 32 floats per operand = 512 float4; two per thread.
-    for (int q = tid; q < KB * KK / 4; q += 256) {
-      int row = q >> 3, c4 = (q & 7) * 4;
-      float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
-      if (i0 + row < N) a = *reinterpret_cast<const float4*>(V + (size_t)(i0 + row) * d + k0 + c4);
-      if (j0 + row < N) b = *reinterpret_cast<const float4*>(V + (size_t)(j0 + row) * d + k0 + c4);
-      As[c4 + 0][row] = a.x; As[c4 + 1][row] = a.y; As[c4 + 2][row] = a.z; As[c4 + 3][row] = a.w;
-      Bs[c4 + 0][row] = b.x; Bs[c4 + 1][row] = b.y; Bs[c4 + 2][row] = b.z; Bs[c4 + 3][row] = b.w;
-    }
-    __syncthreads();
-    // Each 32-term chunk is summed on its own and then added to the total: for nearly parallel
-    // tiles the running sum approaches 1, and chunking cuts its rounding error about sixfold.
-    float part[4][4] = {};
-#pragma unroll 8
-    for (int k = 0; k < KK; ++k) {
-      float4 a = *reinterpret_cast<const float4*>(&As[k][ti * 4]);
-      float4 b = *reinterpret_cast<const float4*>(&Bs[k][tj * 4]);
-      float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-      for (int r = 0; r < 4; ++r)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) part[r][c] = fmaf(av[r], bv[c], part[r][c]);
-    }
-#pragma unroll
-    for (int r = 0; r < 4; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] += part[r][c];
-    __syncthreads();
-  }
-  if (gridDim.z > 1) {
-#pragma unroll
-    for (int r = 0; r < 4; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int i = i0 + ti * 4 + r, j = j0 + tj * 4 + c;
-        if (i < N && j < N) Gpart[((size_t)blockIdx.z * N + i) * N + j] = acc[r][c];
-      }
-    return;
-  }
-#pragma unroll
-  for (int r = 0; r < 4; ++r)
-#pragma unroll
-    for (int c = 0; c < 4; ++c) Gs[ti * 4 + r][tj * 4 + c] = acc[r][c];
-  __syncthreads();
-  if (tid < KB && i0 + tid < N) {
-    const int i = i0 + tid;
-    float bg[RIFT_MAX_KNN];
-    int bj[RIFT_MAX_KNN];
-    for (int r = 0; r < m; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
-    for (int c = 0; c < KB; ++c) {
-      const int j = j0 + c;
-      if (j >= N || j == i) continue;
-      float g = Gs[tid][c];
-      if (!(g == g)) { atomicOr(&g_err_score, RIFT_EBIT_NONFINITE); continue; }
-      if (!knn_better(g, j, bg[m - 1], bj[m - 1])) continue;
-      int p = m - 1;
-      while (p > 0 && knn_better(g, j, bg[p - 1], bj[p - 1])) { bg[p] = bg[p - 1]; bj[p] = bj[p - 1]; --p; }
-      bg[p] = g; bj[p] = j;
-    }
-    const size_t o = ((size_t)i * gridDim.x + blockIdx.x) * m;
-    for (int r = 0; r < m; ++r) { cand_g[o + r] = bg[r]; cand_j[o + r] = bj[r]; }
-  }
-}
-
-// After a split-K Gram pass (N <= 1024): one warp per row sums the slices in slice order for
-// every column and extracts the row's top-C directly (C rounds of a warp-wide argmax, larger
-// similarity first, then the lower index).
-constexpr int RT_WARPS = 4;
-__global__ void __launch_bounds__(32 * RT_WARPS) knn_row_topc_kernel(const float* __restrict__ Gpart, int n_split,
-                                                                      int N, int C, int* __restrict__ top_j) {
-  __shared__ float gs[RT_WARPS][1024];
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int i = blockIdx.x * RT_WARPS + w;
-  if (i >= N) return;
-  float* g = gs[w];
-  for (int j = lane; j < N; j += 32) {
-    float v = 0.f;
-    for (int z = 0; z < n_split; ++z) v += Gpart[((size_t)z * N + i) * N + j];
-    if (!(v == v)) { atomicOr(&g_err_score, RIFT_EBIT_NONFINITE); v = -INFINITY; }
-    g[j] = (j == i) ? -INFINITY : v;
-  }
-  __syncwarp();
-  for (int r = 0; r < C; ++r) {
-    float bv = -INFINITY;
-    int bj = 0x7fffffff;
-    for (int j = lane; j < N; j += 32)
-      if (knn_better(g[j], j, bv, bj)) { bv = g[j]; bj = j; }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-      const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
-      if (knn_better(ov, oj, bv, bj)) { bv = ov; bj = oj; }
-    }
-    if (lane == 0) top_j[(size_t)i * C + r] = (bv == -INFINITY) ? 0x7fffffff : bj;
-    if (bj >= 0 && bj < N && (bj & 31) == lane) g[bj] = -INFINITY;
-    __syncwarp();
-  }
-}
-
-// Large scenes (N > 1024): the Gram matrix on the tensor cores.  Each fp32 row of V (scaled
+// The Gram matrix on the tensor cores.  Each fp32 row of V (scaled
 // by 2^10, so that the low parts stay normal in fp16) is split into hi = fp16(v) and
 // lo = fp16(v - hi); A = [hi | hi | lo] and B = [hi | lo | hi] along K, so one fp16 GEMM with
 // K = 3 d gives hi.hi + hi.lo + lo.hi, i.e. V V^T to ~2^-22 relative (lo.lo is below that).
 constexpr float KNN_SPLIT_SCALE = 1024.f;
-// Rows N .. Np - 1 of B (the padding of the Gram matrix's column count to a multiple of 8) are zero.
-__global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, uint16_t* __restrict__ A,
-                                 uint16_t* __restrict__ B) {
+// B holds every tile; A the rows row0 .. row1 - 1 (A row i - row0).  Rows N .. Np - 1 of B (the
+// padding of the Gram matrix's column count to a multiple of 8) are zero.
+__global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, int row0, int row1,
+                                 uint16_t* __restrict__ A, uint16_t* __restrict__ B) {
+  pdl_trigger();
+  pdl_wait();
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (size_t)Np * d) return;
   const size_t i = idx / d;
@@ -436,22 +348,29 @@ __global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int
   const __half hi = __float2half_rn(v);
   const __half lo = __float2half_rn(v - __half2float(hi));
   const uint16_t h = *reinterpret_cast<const uint16_t*>(&hi), l = *reinterpret_cast<const uint16_t*>(&lo);
-  uint16_t* a = A + i * 3 * d;
   uint16_t* b = B + i * 3 * d;
-  a[k] = h; a[d + k] = h; a[2 * d + k] = l;
   b[k] = h; b[d + k] = l; b[2 * d + k] = h;
+  if (i >= (size_t)row0 && i < (size_t)row1) {
+    uint16_t* a = A + (i - row0) * 3 * d;
+    a[k] = h; a[d + k] = h; a[2 * d + k] = l;
+  }
 }
 
 // One warp per row of the materialised Gram matrix: each lane keeps a sorted top-C of its
 // columns, then C rounds of a warp-wide argmax (larger similarity, then lower index) merge them.
-__global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld, int C, int* __restrict__ top_j) {
+// Row il of G is tile row0 + il.
+__global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld, int row0, int n_rows, int C,
+                                     int* __restrict__ top_j) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
-  const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (i >= N) return;
+  const int il = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (il >= n_rows) return;
+  const int i = row0 + il;
   float bg[RIFT_MAX_KNN];
   int bj[RIFT_MAX_KNN];
   for (int r = 0; r < C; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
-  const float* row = G + (size_t)i * ld;
+  const float* row = G + (size_t)il * ld;
   for (int j = lane; j < N; j += 32) {
     if (j == i) continue;
     const float g = row[j];
@@ -474,31 +393,8 @@ __global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld,
       if (knn_better(og, oj, cg, cj)) { cg = og; cj = oj; cl = ol; }
     }
     if (cl == lane) ++head;
-    if (lane == 0) top_j[(size_t)i * C + r] = (cg == -INFINITY) ? 0x7fffffff : cj;
+    if (lane == 0) top_j[(size_t)il * C + r] = (cg == -INFINITY) ? 0x7fffffff : cj;
   }
-}
-
-// One thread per tile: merge the blocks' candidate lists into the row's top-C by fp32
-// similarity (C = m + a few spares).
-__global__ void knn_merge_kernel(const float* __restrict__ cand_g, const int* __restrict__ cand_j, int n_lists,
-                                 int N, int C, int* __restrict__ top_j) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= N) return;
-  float bg[RIFT_MAX_KNN];
-  int bj[RIFT_MAX_KNN];
-  for (int r = 0; r < C; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
-  for (int l = 0; l < n_lists; ++l) {
-    const size_t o = ((size_t)i * n_lists + l) * C;
-    for (int r = 0; r < C; ++r) {
-      float g = cand_g[o + r];
-      int j = cand_j[o + r];
-      if (!knn_better(g, j, bg[C - 1], bj[C - 1])) break;  // lists are sorted
-      int p = C - 1;
-      while (p > 0 && knn_better(g, j, bg[p - 1], bj[p - 1])) { bg[p] = bg[p - 1]; bj[p] = bj[p - 1]; --p; }
-      bg[p] = g; bj[p] = j;
-    }
-  }
-  for (int r = 0; r < C; ++r) top_j[(size_t)i * C + r] = bj[r];
 }
 
 // One CTA per tile, one warp per candidate: recompute the C candidates' similarities to ~fp64
@@ -506,21 +402,27 @@ __global__ void knn_merge_kernel(const float* __restrict__ cand_g, const int* __
 // separate similarities closer to 1 than 6e-8), keep the m best by those values (ties to the
 // lower index), then s~_i = (sum over the ascending set {i} + NN(i) of s_raw) / (m + 1) with
 // correctly rounded fp32 adds and divide.
+// CTA il smooths tile i = row0 + il and writes s_tilde[il], nbr[il].
 __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
-    const float* __restrict__ V, int d, const int* __restrict__ top_j, int N, int C, int m,
+    const float* __restrict__ V, int d, const int* __restrict__ top_j, int N, int row0, int C, int m,
     const float* __restrict__ s_raw, float* __restrict__ s_tilde, int* __restrict__ nbr) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float4 vi_sm[];  // V_i, read by every candidate's warp
   __shared__ double g64[RIFT_MAX_KNN];
   __shared__ int jj[RIFT_MAX_KNN];
-  const int i = blockIdx.x;
+  const int il = blockIdx.x, i = row0 + il;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int k = threadIdx.x; k < d / 4; k += blockDim.x) vi_sm[k] = reinterpret_cast<const float4*>(V + (size_t)i * d)[k];
+  __syncthreads();
   if (w < C) {
-    const int j = top_j[(size_t)i * C + w];
+    const int j = top_j[(size_t)il * C + w];
     // Each lane keeps its partial sum as an unevaluated pair hi + lo of floats: the product of
     // two floats is split exactly with an FMA (Dekker's TwoProduct as rewritten by Ogita, Rump
     // and Oishi) and added with Knuth's TwoSum, so the lane sum is good to ~2^-44 relative.
     float hi = 0.f, lo = 0.f;
     if (j >= 0 && j < N) {
-      const float4* vi = reinterpret_cast<const float4*>(V + (size_t)i * d);
+      const float4* vi = vi_sm;
       const float4* vj = reinterpret_cast<const float4*>(V + (size_t)j * d);
       for (int k = lane; k < d / 4; k += 32) {
         const float4 a4 = vi[k], b4 = vj[k];
@@ -556,7 +458,7 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
     gl[b] = g; jl[b] = j;
   }
   if (nbr)
-    for (int r = 0; r < m; ++r) nbr[(size_t)i * m + r] = jl[r];
+    for (int r = 0; r < m; ++r) nbr[(size_t)il * m + r] = jl[r];
   int mem[RIFT_MAX_KNN + 1];
   int n = 0;
   for (int r = 0; r < m; ++r) {
@@ -574,7 +476,7 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
   }
   float acc = 0.f;
   for (int a = 0; a < n; ++a) acc = __fadd_rn(acc, s_raw[mem[a]]);
-  s_tilde[i] = __fdiv_rn(acc, (float)(m + 1));
+  s_tilde[il] = __fdiv_rn(acc, (float)(m + 1));
 }
 
 // ------------------------------------------------------------------------------------------
@@ -583,9 +485,9 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
 int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st) {
   if (n_tmpl == 1) {
-    query_rows_kernel<<<(d + 255) / 256, 256, 0, st>>>(static_cast<const uint16_t*>(embed), vocab, d, phrase_ids,
-                                                       n_phrase, bg_ids, M, t, B);
-    normalize_rows_kernel<<<1 + M, 256, 0, st>>>(t, B, d);
+    launch_ex(query_rows_kernel, dim3((d + 255) / 256), dim3(256), 0, st, true, static_cast<const uint16_t*>(embed),
+              vocab, d, phrase_ids, n_phrase, bg_ids, M, t, B);
+    launch_ex(normalize_rows_kernel, dim3(1 + M), dim3(256), 0, st, true, t, B, d);
     return 2;
   }
   // two fp32 rows of d in shared memory: 64 KB at the widest d (8192), past the 48 KB default
@@ -597,52 +499,72 @@ int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids
   return 1;
 }
 
-ScoreLayout score_layout(int N, int n_v, int d, int M) {
-  ScoreLayout L{};
+// Scratch of the kNN smoothing of rows row0 .. row0 + n_rows - 1 against all N tiles: the split
+// operands, the Gram rows, split-K partials when the product has fewer tiles than SMs (at most 16
+// slices within 16 MB), the candidate lists.
+SmoothLayout smooth_layout(int N, int n_rows, int d) {
+  SmoothLayout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
+  const size_t Np = ((size_t)N + 7) & ~size_t(7);
+  L.top_off = take(sizeof(int) * (size_t)n_rows * RIFT_MAX_KNN);
+  L.split_a_off = take(sizeof(uint16_t) * (size_t)n_rows * 3 * d);
+  L.split_b_off = take(sizeof(uint16_t) * Np * 3 * d);
+  L.gram_off = take(sizeof(float) * (size_t)n_rows * Np);
+  const size_t slice = sizeof(float) * (size_t)n_rows * Np;
+  size_t part = ((size_t)16 << 20) / slice;
+  part = part > 16 ? 16 : part;
+  L.splitk_bytes = part >= 2 ? part * slice : 0;
+  L.splitk_off = take(L.splitk_bytes);
+  L.total = off;
+  return L;
+}
+
+// Scratch of the token pass over N tiles: w and the partial pooled sums.
+ShardLayout shard_layout(int N, int n_v, int d) {
+  ShardLayout L{};
   L.chunk_tokens = 96;  // 6 CTAs per 576-token tile
   L.n_chunks = (n_v + L.chunk_tokens - 1) / L.chunk_tokens;
-  L.n_jblk = (N + KB - 1) / KB;
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
   L.w_off = take(sizeof(float) * d);
   L.ppart_off = take(sizeof(float) * (size_t)N * L.n_chunks * d);
-  L.V_off = take(sizeof(float) * (size_t)N * d);
-  L.cand_g_off = take(sizeof(float) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
-  L.cand_j_off = take(sizeof(int) * (size_t)N * L.n_jblk * RIFT_MAX_KNN);
-  L.top_off = take(sizeof(int) * (size_t)N * RIFT_MAX_KNN);
-  // K slices of the Gram pass: enough CTAs for small scenes; each slice a whole number of
-  // 32-column chunks of d.
-  int split = N <= 512 ? 8 : (N <= 1024 ? 4 : 1);
-  while (split > 1 && (d / KK) % split != 0) split >>= 1;
-  L.n_split = split;
-  L.gpart_off = take(L.n_split > 1 ? sizeof(float) * (size_t)L.n_split * N * N : 0);
-  L.tensor_gram = N > 1024;
-  const size_t Np = ((size_t)N + 7) & ~size_t(7);
-  L.split_a_off = take(L.tensor_gram ? sizeof(uint16_t) * (size_t)N * 3 * d : 0);
-  L.split_b_off = take(L.tensor_gram ? sizeof(uint16_t) * Np * 3 * d : 0);
-  L.gram_off = take(L.tensor_gram ? sizeof(float) * (size_t)N * Np : 0);
   L.total = off;
+  return L;
+}
+
+ScoreLayout score_layout(int N, int n_v, int d, int M) {
   (void)M;
+  ScoreLayout L{};
+  L.T = shard_layout(N, n_v, d);
+  L.S = smooth_layout(N, N, d);
+  // V after the token pass's scratch; the smoothing's scratch over the partial pooled sums, which
+  // are dead once V is formed (the smoothing runs after tile_finalize_kernel on the stream)
+  L.V_off = L.T.total;
+  const size_t v_end = L.V_off + ((sizeof(float) * (size_t)N * d + 255) & ~size_t(255));
+  L.smooth_off = L.T.ppart_off;
+  const size_t s_end = L.smooth_off + L.S.total;
+  L.total = s_end > v_end ? s_end : v_end;
+  if (s_end > L.V_off && L.smooth_off < v_end) {  // overlapping V: place the smoothing after V
+    L.smooth_off = v_end;
+    L.total = v_end + L.S.total;
+  }
   return L;
 }
 
 template <typename XT, int NVEC>
-static void launch_tokens(const void* X, int N, int n_v, int d, const ScoreLayout& L, const float* w,
+static void launch_tokens(const void* X, int N, int n_v, int d, const ShardLayout& L, const float* w,
                           float* token_scores, float* Ppart, cudaStream_t st) {
-  token_score_kernel<XT, NVEC><<<N * L.n_chunks, SC_THREADS, 0, st>>>(
-      static_cast<const XT*>(X), n_v, d, L.chunk_tokens, L.n_chunks, w, token_scores, Ppart);
+  launch_ex(token_score_kernel<XT, NVEC>, dim3(N * L.n_chunks), dim3(SC_THREADS), 0, st, true,
+            static_cast<const XT*>(X), n_v, d, L.chunk_tokens, L.n_chunks, (const float*)w, token_scores, Ppart);
 }
 
-int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
-                 int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
-                 cudaStream_t st) {
-  ScoreLayout L = score_layout(N, n_v, d, M);
+int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st) {
+  const ShardLayout L = shard_layout(N, n_v, d);
   float* w = reinterpret_cast<float*>(ws + L.w_off);
   float* Ppart = reinterpret_cast<float*>(ws + L.ppart_off);
-  float* V = reinterpret_cast<float*>(ws + L.V_off);
-  float* cg = reinterpret_cast<float*>(ws + L.cand_g_off);
-  int* cj = reinterpret_cast<int*>(ws + L.cand_j_off);
-  fold_w_kernel<<<(d + 255) / 256, 256, 0, st>>>(t, B, M, d, w);
+  launch_ex(fold_w_kernel, dim3((d + 255) / 256), dim3(256), 0, st, true, t, B, M, d, w);
   const int vw = (xdt == RIFT_BF16) ? 8 : 4;
   const int nvec_per_thread = (d / vw + SC_THREADS - 1) / SC_THREADS;
   if (xdt == RIFT_BF16) {
@@ -654,35 +576,83 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
     else if (nvec_per_thread <= 2) launch_tokens<float, 2>(X, N, n_v, d, L, w, token_scores, Ppart, st);
     else launch_tokens<float, 4>(X, N, n_v, d, L, w, token_scores, Ppart, st);
   }
-  tile_finalize_kernel<<<N, 256, d * sizeof(float), st>>>(Ppart, L.n_chunks, d, w, V, s_raw);
+  launch_ex(tile_finalize_kernel, dim3(N), dim3(std::min(TF_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
+            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw);
+  return 3;
+}
+
+int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, int n_rows, int m, float* s_tilde,
+                  int* nbr, char* ws, cudaStream_t st) {
+  const SmoothLayout L = smooth_layout(N, n_rows, d);
+  const int row1 = row0 + n_rows;
   int* topj = reinterpret_cast<int*>(ws + L.top_off);
   // candidates per row: m plus spares for the fp64 rescoring, at most the N - 1 other tiles
   const int C = m > 0 ? std::min(std::min(m + KNN_SPARE, RIFT_MAX_KNN), N - 1) : 0;
-  int launched = 4;
-  if (m > 0 && L.tensor_gram) {
+  int launched = 1;
+  if (m > 0) {
     uint16_t* A16 = reinterpret_cast<uint16_t*>(ws + L.split_a_off);
     uint16_t* B16 = reinterpret_cast<uint16_t*>(ws + L.split_b_off);
     float* G = reinterpret_cast<float*>(ws + L.gram_off);
     const int Np = (N + 7) & ~7;
     const size_t n = (size_t)Np * d;
-    knn_split_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(V, N, Np, d, A16, B16);
+    launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, row0, row1,
+              A16, B16);
     EpiParams ep;
     ep.out_scale = 1.f / (KNN_SPLIT_SCALE * KNN_SPLIT_SCALE);
-    if (launch_gemm_tc(A16, B16, N, Np, 3 * d, EPI_STORE_F32, G, ep, st)) return -1;
-    knn_gram_topc_kernel<<<(N + 3) / 4, 128, 0, st>>>(G, N, Np, C, topj);
-    launched += 3;
-  } else if (m > 0) {
-    float* gpart = reinterpret_cast<float*>(ws + L.gpart_off);
-    dim3 grid(L.n_jblk, L.n_jblk, L.n_split);
-    knn_block_kernel<<<grid, 256, 0, st>>>(V, N, d, C, cg, cj, gpart);
-    if (L.n_split > 1)
-      knn_row_topc_kernel<<<(N + RT_WARPS - 1) / RT_WARPS, 32 * RT_WARPS, 0, st>>>(gpart, L.n_split, N, C, topj);
-    else
-      knn_merge_kernel<<<(N + 127) / 128, 128, 0, st>>>(cg, cj, L.n_jblk, N, C, topj);
-    launched += 2;
+    // split-K partials for products with fewer tiles than SMs (a scene up to ~2000 tiles)
+    void* part = L.splitk_bytes ? static_cast<void*>(ws + L.splitk_off) : nullptr;
+    // B16 is the split kernel's output, not a constant operand
+    if (launch_gemm_tc(A16, B16, n_rows, Np, 3 * d, EPI_STORE_F32, G, ep, st, part, L.splitk_bytes, true, false))
+      return -1;
+    launch_ex(knn_gram_topc_kernel, dim3((n_rows + 3) / 4), dim3(128), 0, st, true, (const float*)G, N, Np, row0,
+              n_rows, C, topj);
+    launched += 4;
   }
-  knn_rescore_smooth_kernel<<<N, 32 * RIFT_MAX_KNN, 0, st>>>(V, d, topj, N, C, m, s_raw, s_tilde, nbr);
-  return launched;  // kernels launched
+  launch_ex(knn_rescore_smooth_kernel, dim3(n_rows), dim3(32 * RIFT_MAX_KNN), d * sizeof(float), st, true, V, d,
+            (const int*)topj, N, row0, C, m, s_raw, s_tilde, nbr);
+  return launched;
+}
+
+int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
+                 int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
+                 cudaStream_t st) {
+  const ScoreLayout L = score_layout(N, n_v, d, M);
+  float* V = reinterpret_cast<float*>(ws + L.V_off);
+  const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws, st);
+  const int b = launch_smooth(V, s_raw, N, d, 0, N, m, s_tilde, nbr, ws + L.smooth_off, st);
+  return b < 0 ? -1 : a + b;
+}
+
+// (min, max) of n fp32 scores into range[0], range[1]; a NaN among them sets RIFT_EBIT_NONFINITE
+// (min and max then skip it, as fminf / fmaxf do).  One CTA.
+__global__ void __launch_bounds__(1024) score_range_kernel(const float* __restrict__ s, int n,
+                                                           float* __restrict__ range) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float rmin[32], rmax[32];
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  float lo = INFINITY, hi = -INFINITY;
+  bool bad = false;
+  for (int i = tid; i < n; i += blockDim.x) {
+    const float v = s[i];
+    if (!isfinite(v)) bad = true;
+    lo = fminf(lo, v);
+    hi = fmaxf(hi, v);
+  }
+  if (bad) atomicOr(&g_err_score, RIFT_EBIT_NONFINITE);
+  lo = warp_min(lo);
+  hi = warp_max(hi);
+  if (lane == 0) { rmin[wid] = lo; rmax[wid] = hi; }
+  __syncthreads();
+  if (tid < 32) {
+    lo = warp_min(tid < (int)(blockDim.x >> 5) ? rmin[tid] : INFINITY);
+    hi = warp_max(tid < (int)(blockDim.x >> 5) ? rmax[tid] : -INFINITY);
+    if (tid == 0) { range[0] = lo; range[1] = hi; }
+  }
+}
+
+void launch_score_range(const float* s, int n, float* range, cudaStream_t st) {
+  launch_ex(score_range_kernel, dim3(1), dim3(1024), 0, st, true, s, n, range);
 }
 
 }  // namespace rift

@@ -9,14 +9,22 @@
 //
 // The array is a file-scope __device__ variable: every GPU that loads the library holds
 // RIFT_NOALLOC_SCORE_SCRATCH_BYTES of it until the process exits.  Host code cannot use the
-// array's name as a device address (on the host it names a stand-in object), so the first call
-// on each device looks the address up with cudaGetSymbolAddress while that device is current and
-// caches it.  That first call should therefore come before any stream capture.
+// array's name as a device address (on the host it names a stand-in object), so each call looks
+// the address up with cudaGetSymbolAddress in the CUDA context current on the calling thread.  The
+// address belongs to that context: a context rebuilt after cudaDeviceReset, or another context on
+// the same device (a driver-API host), has its own copy of the array at another address, so an
+// address is never reused across contexts.  The one exception is a call made while its stream is
+// being captured, where the lookup (which may load the module) is not made: it takes the address
+// recorded for the current context by an earlier call, so the first call in each context should
+// come before any stream capture.
 //
 // All calls share the one array, and it keeps whatever the last call left in it.  Nothing needs
 // clearing: every scratch element a call reads is written earlier by the same call.  Two calls
 // whose work overlaps on the GPU (different streams, or different host threads) race on the
 // array; callers must order them.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "rift_internal.h"
@@ -25,22 +33,62 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_score_scratch[RIFT_NOALLOC_SCORE_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of g_score_scratch on the current device, looked up once per device.
-rift_status scratch_address(void** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess) return RIFT_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return RIFT_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lk(g_mu);
-  if (!g_scratch_ptr[dev]) {
+// The unique id of the calling thread's current CUDA context (cuCtxGetId: ids are never reused
+// within a process, unlike context handles), or 0 if it cannot be read.
+unsigned long long current_context_id() {
+  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_score_scratch) != cudaSuccess || !p) return RIFT_ERR_CUDA;
-    g_scratch_ptr[dev] = p;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// The addresses recorded by uncaptured calls, one per context id (a small table: a process rarely
+// has more than one context per device).
+constexpr int kMaxContexts = 64;
+std::mutex g_mu;
+unsigned long long g_ctx_id[kMaxContexts] = {};
+void* g_ctx_ptr[kMaxContexts] = {};
+int g_n_ctx = 0;
+
+// Device address of g_score_scratch in the current context.
+rift_status scratch_address(cudaStream_t stream, void** out) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) return RIFT_ERR_CUDA;
+  const unsigned long long id = current_context_id();
+  std::lock_guard<std::mutex> lk(g_mu);
+  int slot = -1;
+  for (int i = 0; i < g_n_ctx; ++i)
+    if (id != 0 && g_ctx_id[i] == id) slot = i;
+  if (cs != cudaStreamCaptureStatusNone) {  // no lookup under capture: the recorded address or nothing
+    if (slot < 0) return RIFT_ERR_UNSUPPORTED;
+    *out = g_ctx_ptr[slot];
+    return RIFT_OK;
   }
-  *out = g_scratch_ptr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_score_scratch) != cudaSuccess || !p) return RIFT_ERR_CUDA;
+  if (id != 0) {
+    if (slot < 0 && g_n_ctx < kMaxContexts) slot = g_n_ctx++;
+    if (slot >= 0) {
+      g_ctx_id[slot] = id;
+      g_ctx_ptr[slot] = p;
+    }
+  }
+  *out = p;
   return RIFT_OK;
 }
 
@@ -50,17 +98,13 @@ extern "C" rift_status rift_score_tiles_noalloc(const void* X, rift_dtype xdt, i
                                                 const float* t, const float* B, int M, int knn_m,
                                                 float* token_scores, float* tile_s_raw, float* tile_s,
                                                 int* nbr, rift_stream_t stream) {
-  if (N < 1 || N > RIFT_MAX_TILES || n_v < 1 || n_v > RIFT_MAX_NV || d < 64 || d > 8192 || d % 64 != 0)
-    return RIFT_ERR_INVALID;
-  if (!X || !t || !token_scores || !tile_s_raw || !tile_s) return RIFT_ERR_INVALID;
-  if (xdt != RIFT_F32 && xdt != RIFT_BF16) return RIFT_ERR_INVALID;
-  if (xdt == RIFT_F32 && d > 4096) return RIFT_ERR_UNSUPPORTED;
-  if (M < 0 || M > 64 || (M > 0 && !B) || knn_m < 0 || knn_m > RIFT_MAX_KNN) return RIFT_ERR_INVALID;
-  if (!rift::aligned16(X)) return RIFT_ERR_INVALID;
+  const rift_status chk =
+      rift::score_args_check(X, xdt, N, n_v, d, t, B, M, knn_m, token_scores, tile_s_raw, tile_s);
+  if (chk != RIFT_OK) return chk;
   const size_t need = rift::score_layout(N, n_v, d, M).total;
   if (need > RIFT_NOALLOC_SCORE_SCRATCH_BYTES) return RIFT_ERR_CAPACITY;  // scene too large for the array
   void* ws = nullptr;
-  const rift_status st = scratch_address(&ws);
+  const rift_status st = scratch_address(static_cast<cudaStream_t>(stream), &ws);
   if (st != RIFT_OK) return st;
   const int m = knn_m < N - 1 ? knn_m : N - 1;
   rift::prof_begin(RIFT_PROF_SCORE, static_cast<cudaStream_t>(stream));

@@ -24,10 +24,14 @@ unsigned int read_clear_err_select() {
 
 constexpr int PB_THREADS = 1024;
 
+// s_range (nullable): the min and max of the whole scene's smoothed scores, when these N tiles are
+// one shard of it (the local scores are still checked for non-finite values).
 __global__ void __launch_bounds__(PB_THREADS) prune_budget_kernel(
     const float* __restrict__ s, int N, int n_v, const float* __restrict__ p_ext, rift_policy pol,
-    float* __restrict__ u, int* __restrict__ kept, int* __restrict__ n_kept,
+    const float* __restrict__ s_range, float* __restrict__ u, int* __restrict__ kept, int* __restrict__ n_kept,
     int* __restrict__ budgets, int* __restrict__ sel_off) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float rmin[32], rmax[32];
   __shared__ int sh[33];
   __shared__ int s_bad;
@@ -54,6 +58,12 @@ __global__ void __launch_bounds__(PB_THREADS) prune_budget_kernel(
   __syncthreads();
   lo = rmin[0];
   hi = rmax[0];
+  if (s_range) {
+    lo = s_range[0];
+    hi = s_range[1];
+    if (!isfinite(lo) || !isfinite(hi)) s_bad = 1;  // every thread read s_bad after the barrier above
+  }
+  __syncthreads();
   if (s_bad) {
     if (tid == 0) { atomicOr(&g_err_select, RIFT_EBIT_NONFINITE); *n_kept = 0; }
     for (int j = tid; j <= N; j += PB_THREADS) sel_off[j] = 0;
@@ -125,6 +135,8 @@ __global__ void __launch_bounds__(TB_THREADS) topb_kernel(const float* __restric
                                                           const int* __restrict__ budgets,
                                                           const int* __restrict__ sel_off,
                                                           int* __restrict__ sel) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int hist[256];
   __shared__ int sh[33];
   __shared__ uint32_t s_digit;
@@ -211,9 +223,11 @@ __global__ void __launch_bounds__(TB_THREADS) topb_kernel(const float* __restric
 
 void launch_select(const float* token_scores, const float* tile_s, int N, int n_v, const float* p,
                    const rift_policy& pol, float* u, int* kept, int* n_kept, int* budgets, int* sel,
-                   int* sel_off, cudaStream_t st) {
-  prune_budget_kernel<<<1, PB_THREADS, 0, st>>>(tile_s, N, n_v, p, pol, u, kept, n_kept, budgets, sel_off);
-  topb_kernel<<<N, TB_THREADS, 0, st>>>(token_scores, n_v, kept, n_kept, budgets, sel_off, sel);
+                   int* sel_off, cudaStream_t st, const float* s_range) {
+  launch_ex(prune_budget_kernel, dim3(1), dim3(PB_THREADS), 0, st, true, tile_s, N, n_v, p, pol, s_range, u, kept,
+            n_kept, budgets, sel_off);
+  launch_ex(topb_kernel, dim3(N), dim3(TB_THREADS), 0, st, true, token_scores, n_v, (const int*)kept,
+            (const int*)n_kept, (const int*)budgets, (const int*)sel_off, sel);
 }
 
 }  // namespace rift

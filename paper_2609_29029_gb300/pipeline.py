@@ -1,8 +1,9 @@
 """Device buffers and the call sequence of one scene query through the C ABI.
 
 This module owns memory (torch tensors) and issues the five ABI calls in order; every
-computation is a kernel of libriftgb.so.  One host read-back per query (n_kept and T, after
-packing) sizes the prefill launch.
+computation is a kernel of libriftgb.so.  The prefill reads the counts the selection and the
+packing leave on the device (n_kept, T), so a whole query is enqueued without waiting for the
+GPU; the counts are read back only for reporting (read_counts).
 """
 from __future__ import annotations
 
@@ -126,6 +127,7 @@ class ScenePipeline:
         self.device = dev
 
     def _prefill_ws(self, T, n_seq):
+        """The prefill workspace for T rows and n_seq sequences of capacity (kept across queries)."""
         need = abi.prefill_workspace_bytes(self.model.struct, T, n_seq, self.max_len)
         if need > self.ws_prefill_bytes:
             self.ws_prefill = torch.empty(need, dtype=torch.uint8, device=self.device)
@@ -177,34 +179,59 @@ class ScenePipeline:
         final hidden states, self.prefix_hidden the prompt's."""
         self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)
         self.pack(X, embed, sys_ids, query_ids, stream, with_system=False)
-        n_kept, T = self.read_counts(stream)
         m, S = self.model, self.S
         if not hasattr(self, "prefix_hidden"):
             self.prefix_hidden = torch.empty(S, self.d, dtype=torch.bfloat16, device=self.device)
             self.prefix_kv = torch.empty(m.dec.n_layers, 2, S, self.d, dtype=torch.float16, device=self.device)
-        need = abi.prefill_shared_prefix_workspace_bytes(m.struct, T, n_kept, self.max_len, S)
+        need = abi.prefill_shared_prefix_workspace_bytes(m.struct, self.max_T, self.N, self.max_len, S)
         if need > self.ws_prefill_bytes:
             self.ws_prefill = torch.empty(need, dtype=torch.uint8, device=self.device)
             self.ws_prefill_bytes = need
         abi.prefill_shared_prefix(m.struct, sys_ids, S, embed, embed.shape[0], self.prefix_hidden, self.prefix_kv,
-                                  self.packed, T, self.cu, n_kept, self.max_len, self.positions, None,
-                                  self.ws_prefill, self.ws_prefill_bytes, stream)
-        return n_kept, T
+                                  self.packed, self.T, self.cu, self.n_kept, self.max_len, self.positions, None,
+                                  self.ws_prefill, self.ws_prefill_bytes, stream, max_T=self.max_T, max_seqs=self.N)
+        return self.read_counts(stream)
+
+    def _enqueue_counts(self, stream=None):
+        """Copy (n_kept, T) into pinned host memory on `stream` once they are written, and record
+        an event for counts() to wait on."""
+        s = stream if stream is not None else torch.cuda.current_stream()
+        with torch.cuda.stream(s):
+            self.counts_host[0:1].copy_(self.n_kept, non_blocking=True)
+            self.counts_host[1:2].copy_(self.T, non_blocking=True)
+            self._counts_ev = torch.cuda.Event()
+            self._counts_ev.record(s)
+
+    def counts(self):
+        """(n_kept, T) of the last query run with counts=False: waits only until its packing has
+        finished (the prefill may still be running).  The next query of this pipeline overwrites
+        them."""
+        self._counts_ev.synchronize()
+        return int(self.counts_host[0]), int(self.counts_host[1])
 
     def read_counts(self, stream=None):
         """Sync, check device error flags and read (n_kept, T) back to the host."""
         s = stream if stream is not None else torch.cuda.current_stream()
-        self.counts_host[0:1].copy_(self.n_kept, non_blocking=True)
-        self.counts_host[1:2].copy_(self.T, non_blocking=True)
+        self._enqueue_counts(s)
         abi.sync_status(s)
         return int(self.counts_host[0]), int(self.counts_host[1])
 
-    def prefill(self, T, n_seq, stream=None, kv_out=None, last_logits=None):
-        """a9: decoder prefill over the packed batch, in place; optionally the KV cache
-        (fp16 [n_layers, 2, T, d]) and the last-token logits (fp32 [n_seq, vocab])."""
-        ws, need = self._prefill_ws(T, n_seq)
-        abi.prefill_layers(self.model.struct, self.packed, T, self.cu, n_seq, self.max_len, self.positions, ws,
-                           need, stream, kv_out=kv_out, last_logits=last_logits)
+    def prefill(self, stream=None, kv_out=None, last_logits=None, counts=None):
+        """a9: decoder prefill over the packed batch, in place, with the row and sequence counts
+        the packing left on the device (capacities max_T and N), or with host counts
+        counts = (n_seq, T) read back earlier, which are then also the capacities (so that the
+        optional KV cache, fp16 [n_layers, 2, T, d], is sized for the rows it holds).  Optional
+        last-token logits: fp32 [capacity, vocab]."""
+        if counts is not None:
+            n_seq, T = counts
+            ws, need = self._prefill_ws(T, n_seq)
+            abi.prefill_layers(self.model.struct, self.packed, T, self.cu, n_seq, self.max_len, self.positions, ws,
+                               need, stream, kv_out=kv_out, last_logits=last_logits)
+            return
+        ws, need = self._prefill_ws(self.max_T, self.N)
+        abi.prefill_layers(self.model.struct, self.packed, self.T, self.cu, self.n_kept, self.max_len,
+                           self.positions, ws, need, stream, kv_out=kv_out, last_logits=last_logits,
+                           max_T=self.max_T, max_seqs=self.N)
 
     def decode(self, kv_cache, T, n_seq, token_ids, embed, hidden_out=None, kv_new=None, logits=None,
                stream=None):
@@ -249,13 +276,20 @@ class ScenePipeline:
                                self.batch_positions, ws, need, stream)
         return out
 
-    def run(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, prefill=True, stream=None):
+    def run(self, X, embed, phrase_ids, bg_ids, sys_ids, query_ids, p=None, prefill=True, stream=None,
+            counts=True):
+        """One scene query, a1-a9, enqueued on `stream` with no host wait in between.  counts=True
+        then waits for it, checks the device error flags and returns (n_kept, T); counts=False
+        returns at once (None): counts() gives them once the packing has run."""
         self.select(X, embed, phrase_ids, bg_ids, p, stream=stream)
         self.pack(X, embed, sys_ids, query_ids, stream)
-        n_kept, T = self.read_counts(stream)
-        if prefill and self.model is not None and T > 0:
-            self.prefill(T, n_kept, stream)
-        return n_kept, T
+        self._enqueue_counts(stream)
+        if prefill and self.model is not None:
+            self.prefill(stream)
+        if counts:
+            abi.sync_status(stream)
+            return self.counts()
+        return None
 
     def result(self, n_kept, T) -> QueryResult:
         return QueryResult(n_kept, T, self.t, self.token_scores, self.tile_s_raw, self.tile_s,

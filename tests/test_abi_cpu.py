@@ -31,7 +31,7 @@ def test_library_exports_every_declared_symbol(riftlib):
 def test_status_strings(riftlib):
     assert riftlib.status_string(0) == "ok"
     assert riftlib.status_string(riftlib.RIFT_ERR_CAPACITY) == "output capacity exceeded"
-    assert riftlib.abi_version() == 4
+    assert riftlib.abi_version() == 5
 
 
 FAKE = 0x10000  # a 16-byte aligned non-null address; validation rejects before using it
@@ -116,15 +116,32 @@ def test_pack_and_prefill_reject_bad_arguments(riftlib):
     m.head_dim = 96
     assert lib.rift_prefill_workspace_bytes(C.byref(m), 100, 2, 64) == 0
     m.head_dim, m.ffn = 64, 690
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, None, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, None, 10, FAKE, None, 1, 64, FAKE, None, None, FAKE, 1 << 30, 0) == INV
     m.ffn = 688
     # last-token logits need an output matrix; optional outputs must be 16-byte aligned
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, FAKE + 8, None, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, None, 10, FAKE, None, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, None, 10, FAKE, None, 1, 64, FAKE, FAKE + 8, None, FAKE, 1 << 30, 0) == INV
     m.vocab, m.lm_head = 1000, FAKE
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE + 4, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, None, 10, FAKE, None, 1, 64, FAKE, None, FAKE + 4, FAKE, 1 << 30, 0) == INV
     m.vocab = 1001  # not a multiple of 8
-    assert lib.rift_prefill_layers(C.byref(m), FAKE, 10, FAKE, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, None, 10, FAKE, None, 1, 64, FAKE, None, FAKE, FAKE, 1 << 30, 0) == INV
+    m.vocab = 1000
+    # rows without any sequence, negative capacities
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, FAKE, 10, FAKE, FAKE, 0, 64, FAKE, None, None, FAKE, 1 << 30, 0) == INV
+    assert lib.rift_prefill_layers(C.byref(m), FAKE, FAKE, -1, FAKE, FAKE, 1, 64, FAKE, None, None, FAKE, 1 << 30, 0) == INV
+
+
+def test_prefill_count_arguments(riftlib):
+    """Host counts are their own capacities; a device count needs one (marshalling only)."""
+    import torch
+    assert riftlib._count(7, None, "T") == (None, 7)
+    assert riftlib._count(7, 7, "T") == (None, 7)
+    with pytest.raises(ValueError):
+        riftlib._count(7, 9, "T")
+    with pytest.raises(ValueError):
+        riftlib._count(torch.zeros(1, dtype=torch.int32), None, "T")
+    t = torch.zeros(1, dtype=torch.int32)
+    assert riftlib._count(t, 9, "T") == (t.data_ptr(), 9)
 
 
 def test_decode_rejects_bad_arguments(riftlib):

@@ -46,7 +46,7 @@ def test_cache_logits_and_decode_match_oracle(dec, cuda, riftlib):
     packed = pipe.packed[:T].cpu().clone()
     kv = torch.full((dec.n_layers, 2, T, dec.d), float("nan"), dtype=torch.float16, device=cuda)
     last = torch.full((n, dec.vocab), float("nan"), dtype=torch.float32, device=cuda)
-    pipe.prefill(T, n, kv_out=kv, last_logits=last)
+    pipe.prefill(kv_out=kv, last_logits=last, counts=(n, T))
     ids = _token_ids(n, dec.vocab, 1)
     ids_d = torch.tensor(ids, dtype=torch.int32, device=cuda)
     hid = torch.empty(n, dec.d, dtype=torch.bfloat16, device=cuda)

@@ -235,3 +235,48 @@ def test_full_budget_equals_exhaustive_prefill_bit_for_bit(cases, cuda, riftlib)
     exh_out = _prefill_gpu(riftlib, dm, exh, cu, pos, L, cuda)
     assert n_kept == N and T == exh.shape[0]
     assert torch.equal(rift_out, exh_out)
+
+
+@pytest.mark.parametrize("name", [P.SMALL24.name, P.RAGGED.name])
+def test_device_counts_equal_host_counts(name, cases, cuda, riftlib):
+    """The query enqueued whole, the prefill reading n_kept and T on the device (no host
+    read-back), gives the same final hidden states bit for bit as the prefill run with the counts
+    read back to the host.  Both batches have more than 1024 rows, so both take the same GEMM
+    path (SM pairs)."""
+    wl, sc, sel = cases[name]
+    dm, layers, gf = _model(wl.decoder, cuda)
+    pipe, dv = P.gpu_pipeline(wl, sc, cuda, model=dm)
+    args = (dv["X"], dv["embed"], dv["q"], dv["bg"], dv["sys"], dv["q"])
+    assert pipe.run(*args, counts=False) is None
+    n_kept, T = pipe.counts()
+    riftlib.sync_status()
+    assert T >= 1024 and T == sum(wl.scene.S + b + wl.scene.Q for b in sel.budgets)
+    dev_out = pipe.packed[:T].cpu().clone()
+    pipe.run(*args, prefill=False)
+    pipe.prefill(counts=(n_kept, T))
+    riftlib.sync_status()
+    assert torch.equal(pipe.packed[:T].cpu(), dev_out)
+
+
+def test_device_sequence_count_above_capacity_is_reported(cuda, riftlib):
+    """A device sequence count above max_seqs: the first max_seqs sequences are prefilled and
+    the next rift_sync_status returns RIFT_ERR_CAPACITY; the context stays usable."""
+    dec = W.TINY_DECODER
+    dm, layers, gf = _model(dec, cuda)
+    lengths = [40, 24]
+    T = sum(lengths)
+    H0 = rng.normal_f32(11, rng.stream_id("count-cap"), T * dec.d, "cpu").view(T, dec.d).to(torch.bfloat16)
+    cu = torch.tensor([0, 40, 64], dtype=torch.int32, device=cuda)
+    pos = torch.tensor(list(range(40)) + list(range(24)), dtype=torch.int32, device=cuda)
+    i32 = dict(dtype=torch.int32, device=cuda)
+    need = riftlib.prefill_workspace_bytes(dm.struct, T, 1, 64)
+    ws = torch.empty(need, dtype=torch.uint8, device=cuda)
+    hid = H0.to(cuda)
+    riftlib.prefill_layers(dm.struct, hid, torch.tensor([T], **i32), cu, torch.tensor([2], **i32), 64, pos, ws,
+                           need, max_T=T, max_seqs=1)
+    with pytest.raises(riftlib.RiftError) as e:
+        riftlib.sync_status()
+    assert e.value.status == riftlib.RIFT_ERR_CAPACITY
+    ref = O.prefill_sequence(H0[:40], lambda l: layers[l], gf, dec)
+    assert P.max_abs_rel(hid[:40].cpu(), ref) < P.HIDDEN_TOL
+    riftlib.sync_status()  # cleared

@@ -71,6 +71,19 @@ def test_noalloc_scoring_matches_workspace_scoring_twice_in_a_row(cuda, riftlib)
         _check(ref, got)
 
 
+def test_noalloc_tensor_core_gram_branch_twice_in_a_row(cuda, riftlib):
+    # 1100 tiles: the kNN's Gram product over its largest scene that fits the array (at d = 256),
+    # with its split operands, tensor maps, split-K partials and the Gram matrix itself all inside
+    # the fixed array.
+    wl = W.Workload("noalloc_gram", W.SceneSpec(N=1100, d=256, x_dtype="bf16"), W.LLAVA7B, W.RIFT_POLICY)
+    s = wl.scene
+    assert riftlib.score_workspace_bytes(s.N, s.n_v, s.d, s.M) <= riftlib.NOALLOC_SCORE_SCRATCH_BYTES
+    sc = _scene(wl, cuda)
+    for _ in range(2):
+        ref, got = _score_both(riftlib, wl, sc, cuda)
+        _check(ref, got)
+
+
 def test_noalloc_rejects_scenes_larger_than_its_array(cuda, riftlib):
     N, n_v, d, M = 2000, 576, 4096, 8
     assert riftlib.score_workspace_bytes(N, n_v, d, M) > riftlib.NOALLOC_SCORE_SCRATCH_BYTES
