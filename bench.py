@@ -633,6 +633,9 @@ def main():
     prof = abi.profile_read()
     barrier(ws)
     value, ms_max = job_throughput(float(T * args.steps), ms, ws)
+    # the pre-prefill path alone (scoring, selection, packing), without the profiler's events
+    # between its classes
+    sel_ms = select_latency(pipe, sc, q, bg, sy, args.steps, stream)
 
     # ---- end to end: host buffers.  Every step copies its inputs (the scene's vision tokens and
     # the query's id lists) from pinned host memory and reads its result (the final hidden states)
@@ -719,8 +722,6 @@ def main():
     achieved = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
     traffic = gemm_traffic(wl.name)
     per_step = {k: round(v[0] / args.steps, 3) for k, v in prof.items()}
-    # the pre-prefill path alone, without the profiler's events between its classes
-    sel_ms = select_latency(pipe, sc, q, bg, sy, args.steps, stream)
     x_bytes = sc.X.numel() * sc.X.element_size()
 
     cpu = None

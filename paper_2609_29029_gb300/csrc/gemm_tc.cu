@@ -212,6 +212,17 @@ __device__ __forceinline__ void tile_coords(int tile, int mt, int nt, int group,
   n_blk = n_major ? a : b;
 }
 
+// Tile t of the upper triangle (bi <= bj) of an mt x mt tile grid, row by row.
+__device__ __forceinline__ void tri_coords(int t, int mt, int& bi, int& bj) {
+  int b = 0;
+  while (b < mt - 1 && t >= mt - b) {
+    t -= mt - b;
+    ++b;
+  }
+  bi = b;
+  bj = b + t;
+}
+
 __device__ __forceinline__ float silu(float g) { return g / (1.f + expf(-g)); }
 
 // Epilogue for one row of one 32-column chunk (columns n0 .. n0 + 31 of the tile).
@@ -378,7 +389,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int M = ep.m_dev ? max(0, min(M_cap, *ep.m_dev)) : M_cap;
 
   const int mt = (M + TM - 1) / TM, nt = (N + BN - 1) / BN, kt = (K + BK - 1) / BK;
-  const int n_tiles = mt * nt;
+  const int n_tiles = ep.symmetric ? mt * (mt + 1) / 2 : mt * nt;
+  auto coords = [&](int tile, int& m_blk, int& n_blk) {
+    if (ep.symmetric) tri_coords(tile, mt, m_blk, n_blk);
+    else tile_coords(tile, mt, nt, group_m, m_blk, n_blk);
+  };
   // unit u: tile u / splits, K-blocks [k0, k1) of slice u % splits (the host makes every slice
   // non-empty)
   const int n_units = n_tiles * splits, k_per = (kt + splits - 1) / splits;
@@ -400,7 +415,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int n_pre = 0;
       if (!PAIR && a_const && !ep.m_dev && u_first < n_units) {
         int m_blk, n_blk, k0, k1;
-        tile_coords(u_first / splits, mt, nt, group_m, m_blk, n_blk);
+        coords(u_first / splits, m_blk, n_blk);
         unit_k(u_first, k0, k1);
         n_pre = min(STAGES, k1 - k0);
         for (int j = 0; j < n_pre; ++j) {
@@ -413,7 +428,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (int u = u_first; u < n_units && ok; u += u_step) {
         int m_blk, n_blk, k0, k1;
-        tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
+        coords(u / splits, m_blk, n_blk);
         unit_k(u, k0, k1);
         for (int k = k0; k < k1; ++k, ++it) {
           const int s = it % STAGES;
@@ -497,7 +512,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     int tl = 0;
     for (int u = u_first; u < n_units; u += u_step, ++tl) {
       int m_blk, n_blk;
-      tile_coords(u / splits, mt, nt, group_m, m_blk, n_blk);
+      coords(u / splits, m_blk, n_blk);
       // split-K partials (EPI_STORE_F32 only): slice u % splits at C + slice * split_stride
       void* Cu = splits > 1 ? static_cast<void*>(static_cast<float*>(C) + (size_t)(u % splits) * split_stride) : C;
       const int b = tl & 1;
@@ -542,6 +557,18 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
           } else {
             if (row < M) epilogue_chunk<EPI>(r, row, n_blk * BN + c, N, Cu, ep.out_scale);
+            if constexpr (EPI == EPI_STORE_F32) {
+              // symmetric product: the off-diagonal tile also fills its mirror (a warp's lanes hold
+              // consecutive rows, so each transposed store is 32 consecutive floats)
+              if (ep.symmetric && m_blk != n_blk && row < M) {
+                float* out = static_cast<float*>(Cu);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                  const int col = n_blk * BN + c + e;
+                  if (col < M) out[(size_t)col * N + row] = __uint_as_float(r[e]) * ep.out_scale;
+                }
+              }
+            }
           }
         }
       }
@@ -1071,7 +1098,9 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits, pdl,
                                                   b_const ? 1 : 0))
       return 1;
-    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st, pdl);
+    EpiParams e = ep;
+    e.symmetric = 0;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, e, st, pdl);
   }
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
@@ -1082,7 +1111,9 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
   if (splits > 1 || fuse_norm) {
     if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits, pdl)) return 1;
-    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, ep, st, pdl);
+    EpiParams e = ep;
+    e.symmetric = 0;
+    return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, e, st, pdl);
   }
   // Many rows: 256 x 256 tiles on SM pairs.
   if (M >= 1024) {
@@ -1099,12 +1130,14 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
     }
     if (r >= 0) return r;
   }
+  EpiParams e1 = ep;  // one SM per tile: 128 x 256 tiles, every tile computed
+  e1.symmetric = 0;
   switch (epi) {
-    case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, ep, st);
-    case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, ep, st);
-    case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, ep, st);
-    case EPI_QKV_ROPE: return launch<EPI_QKV_ROPE>(ma, mb, M, N, K, C, ep, st);
-    case EPI_STORE_F32: return launch<EPI_STORE_F32>(ma, mb, M, N, K, C, ep, st);
+    case EPI_STORE_BF16: return launch<EPI_STORE_BF16>(ma, mb, M, N, K, C, e1, st);
+    case EPI_RESID_F32: return launch<EPI_RESID_F32>(ma, mb, M, N, K, C, e1, st);
+    case EPI_SWIGLU: return launch<EPI_SWIGLU>(ma, mb, M, N, K, C, e1, st);
+    case EPI_QKV_ROPE: return launch<EPI_QKV_ROPE>(ma, mb, M, N, K, C, e1, st);
+    case EPI_STORE_F32: return launch<EPI_STORE_F32>(ma, mb, M, N, K, C, e1, st);
     default: return 1;
   }
 }

@@ -146,6 +146,10 @@ struct EpiParams {
   // Device row count (nullable): the product covers rows min(M, *m_dev); M is then the capacity
   // the operands and the output are sized for.  Not used with split-K.
   const int* m_dev = nullptr;
+  // EPI_STORE_F32 of a symmetric product (A = B's first M rows, M <= N <= M + 7: a Gram matrix):
+  // only the tiles on and above the diagonal are computed, each off-diagonal one stored twice
+  // (as itself and transposed).  Honoured on the SM-pair path; the other paths compute every tile.
+  int symmetric = 0;
 };
 // split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
 // most SMs idle run as (tile, K-slice) units plus a reduction kernel.

@@ -78,46 +78,62 @@ __global__ void __launch_bounds__(256) query_prep_kernel(const uint16_t* __restr
   }
 }
 
-// One caption template: rows are plain means / copies, so every column is independent.  One
-// thread per column writes the unnormalised query row into t and the background rows into B;
-// normalize_rows_kernel then scales each row to unit length (one CTA per row).
-__global__ void query_rows_kernel(const uint16_t* __restrict__ embed, int vocab, int d,
-                                  const int* __restrict__ phrase_ids, int n_phrase,
-                                  const int* __restrict__ bg_ids, int M, float* __restrict__ t,
-                                  float* __restrict__ B) {
-  pdl_trigger();
-  pdl_wait();
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= d) return;
-  float s = 0.f;
-  for (int q = 0; q < n_phrase; ++q) {
-    const int id = phrase_ids[q];
-    if (id < 0 || id >= vocab) {
-      atomicOr(&g_err_score, RIFT_EBIT_BADID);
-      continue;
-    }
-    s += bf16_bits_to_float(embed[(size_t)id * d + c]);
-  }
-  t[c] = s / (float)n_phrase;
-  for (int j = 0; j < M; ++j) {
-    const int id = bg_ids[j];
-    const bool ok = id >= 0 && id < vocab;
-    if (!ok && c == 0) atomicOr(&g_err_score, RIFT_EBIT_BADID);
-    B[(size_t)j * d + c] = ok ? bf16_bits_to_float(embed[(size_t)id * d + c]) : 0.f;
-  }
-}
-
-// Row r of {t, B_0, ..., B_{M-1}} divided by its length (zero rows stay zero).
-__global__ void __launch_bounds__(256) normalize_rows_kernel(float* __restrict__ t, float* __restrict__ B, int d) {
+// One caption template: CTA 0 forms t = l2norm(mean_q embed[phrase_ids[q]]), CTA 1 + j forms
+// B_j = l2norm(embed[bg_ids[j]]); a thread owns 4 columns (VPT groups of them at d > 4096) and
+// issues the loads of all its rows before summing them, so a CTA waits on one round of loads.
+constexpr int QR_THREADS = 1024;
+__global__ void __launch_bounds__(QR_THREADS) query_rows_kernel(const uint16_t* __restrict__ embed, int vocab, int d,
+                                                                const int* __restrict__ phrase_ids, int n_phrase,
+                                                                const int* __restrict__ bg_ids, int M,
+                                                                float* __restrict__ t, float* __restrict__ B) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[32];
-  float* row = blockIdx.x == 0 ? t : B + (size_t)(blockIdx.x - 1) * d;
+  const bool is_t = blockIdx.x == 0;
+  float* out = is_t ? t : B + (size_t)(blockIdx.x - 1) * d;
+  const int n_ids = is_t ? n_phrase : 1;
+  const int* ids = is_t ? phrase_ids : bg_ids + (blockIdx.x - 1);
+  const int nv = d / 4;
+  float4 acc[2];
   float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += row[c] * row[c];
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int c = threadIdx.x + k * QR_THREADS;
+    acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c >= nv) continue;
+    for (int q0 = 0; q0 < n_ids; q0 += 8) {
+      uint2 raw[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {  // up to eight rows' loads in flight
+        const int q = q0 + u;
+        const int id = q < n_ids ? ids[q] : -1;
+        const bool ok = id >= 0 && id < vocab;
+        if (q < n_ids && !ok && c == 0) atomicOr(&g_err_score, RIFT_EBIT_BADID);
+        raw[u] = ok ? reinterpret_cast<const uint2*>(embed + (size_t)id * d)[c] : make_uint2(0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {  // ascending q, as the sum of the ids' rows is defined
+        if (q0 + u >= n_ids) break;
+        acc[k].x += __uint_as_float(raw[u].x << 16);
+        acc[k].y += __uint_as_float(raw[u].x & 0xffff0000u);
+        acc[k].z += __uint_as_float(raw[u].y << 16);
+        acc[k].w += __uint_as_float(raw[u].y & 0xffff0000u);
+      }
+    }
+    if (is_t) {
+      const float inv_n = 1.f / (float)n_phrase;
+      acc[k] = make_float4(acc[k].x * inv_n, acc[k].y * inv_n, acc[k].z * inv_n, acc[k].w * inv_n);
+    }
+    ss += acc[k].x * acc[k].x + acc[k].y * acc[k].y + acc[k].z * acc[k].z + acc[k].w * acc[k].w;
+  }
   const float tot = block_sum(ss, red);
   const float inv = tot > 0.f ? 1.f / sqrtf(tot) : 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) row[c] *= inv;
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int c = threadIdx.x + k * QR_THREADS;
+    if (c < nv)
+      reinterpret_cast<float4*>(out)[c] = make_float4(acc[k].x * inv, acc[k].y * inv, acc[k].z * inv, acc[k].w * inv);
+  }
 }
 
 // w = t - (1/M) sum_j B_j  (M = 0: w = t)
@@ -330,71 +346,109 @@ __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
 // K = 3 d gives hi.hi + hi.lo + lo.hi, i.e. V V^T to ~2^-22 relative (lo.lo is below that).
 constexpr float KNN_SPLIT_SCALE = 1024.f;
 // B holds every tile; A the rows row0 .. row1 - 1 (A row i - row0).  Rows N .. Np - 1 of B (the
-// padding of the Gram matrix's column count to a multiple of 8) are zero.
+// padding of the Gram matrix's column count to a multiple of 8) are zero.  A thread handles 8
+// consecutive elements of a row (two float4 loads, 16-byte stores into each of the row's parts).
 __global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, int row0, int row1,
                                  uint16_t* __restrict__ A, uint16_t* __restrict__ B) {
   pdl_trigger();
   pdl_wait();
+  const int n8 = d / 8;
   const size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (size_t)Np * d) return;
-  const size_t i = idx / d;
-  const int k = (int)(idx % d);
+  if (idx >= (size_t)Np * n8) return;
+  const size_t i = idx / n8;
+  const int k = (int)(idx % n8) * 8;
+  uint4* b = reinterpret_cast<uint4*>(B + i * 3 * d + k);
   if (i >= (size_t)N) {
-    uint16_t* b = B + i * 3 * d;
-    b[k] = 0; b[d + k] = 0; b[2 * d + k] = 0;
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    b[0] = z;
+    b[d / 8] = z;
+    b[d / 4] = z;
     return;
   }
-  const float v = V[idx] * KNN_SPLIT_SCALE;
-  const __half hi = __float2half_rn(v);
-  const __half lo = __float2half_rn(v - __half2float(hi));
-  const uint16_t h = *reinterpret_cast<const uint16_t*>(&hi), l = *reinterpret_cast<const uint16_t*>(&lo);
-  uint16_t* b = B + i * 3 * d;
-  b[k] = h; b[d + k] = l; b[2 * d + k] = h;
+  const float4 v0 = reinterpret_cast<const float4*>(V + i * d + k)[0];
+  const float4 v1 = reinterpret_cast<const float4*>(V + i * d + k)[1];
+  const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+  uint32_t h[4], l[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float a0 = v[2 * q] * KNN_SPLIT_SCALE, a1 = v[2 * q + 1] * KNN_SPLIT_SCALE;
+    const __half h0 = __float2half_rn(a0), h1 = __float2half_rn(a1);
+    h[q] = pack_half2(__half2float(h0), __half2float(h1));
+    l[q] = pack_half2(a0 - __half2float(h0), a1 - __half2float(h1));
+  }
+  const uint4 hv = make_uint4(h[0], h[1], h[2], h[3]), lv = make_uint4(l[0], l[1], l[2], l[3]);
+  b[0] = hv;
+  b[d / 8] = lv;
+  b[d / 4] = hv;
   if (i >= (size_t)row0 && i < (size_t)row1) {
-    uint16_t* a = A + (i - row0) * 3 * d;
-    a[k] = h; a[d + k] = h; a[2 * d + k] = l;
+    uint4* a = reinterpret_cast<uint4*>(A + (i - row0) * 3 * d + k);
+    a[0] = hv;
+    a[d / 8] = hv;
+    a[d / 4] = lv;
   }
 }
 
-// One warp per row of the materialised Gram matrix: each lane keeps a sorted top-C of its
-// columns, then C rounds of a warp-wide argmax (larger similarity, then lower index) merge them.
-// Row il of G is tile row0 + il.
+// One warp per row of the materialised Gram matrix: the row's 16 best columns (larger
+// similarity, then lower index) are kept sorted across lanes 0..15, one entry per lane.  The row
+// is read 32 columns at a time; a ballot picks the columns that beat the current 16th entry, and
+// each of them (in ascending column order) is inserted at the position the entries above it
+// give, the entries below moving down a lane.  Row il of G is tile row0 + il.
 __global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld, int row0, int n_rows, int C,
                                      int* __restrict__ top_j) {
   pdl_trigger();
   pdl_wait();
+  constexpr int K = RIFT_MAX_KNN;  // list length (C <= K)
   const int lane = threadIdx.x & 31;
   const int il = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (il >= n_rows) return;
   const int i = row0 + il;
-  float bg[RIFT_MAX_KNN];
-  int bj[RIFT_MAX_KNN];
-  for (int r = 0; r < C; ++r) { bg[r] = -INFINITY; bj[r] = 0x7fffffff; }
+  float lg = -INFINITY;  // this lane's entry (lanes >= K stay empty)
+  int lj = 0x7fffffff;
+  float tg = -INFINITY;  // the 16th entry: what a column must beat
+  int tj = 0x7fffffff;
   const float* row = G + (size_t)il * ld;
-  for (int j = lane; j < N; j += 32) {
-    if (j == i) continue;
-    const float g = row[j];
-    if (!(g == g)) { atomicOr(&g_err_score, RIFT_EBIT_NONFINITE); continue; }
-    if (!knn_better(g, j, bg[C - 1], bj[C - 1])) continue;
-    int p = C - 1;
-    while (p > 0 && knn_better(g, j, bg[p - 1], bj[p - 1])) { bg[p] = bg[p - 1]; bj[p] = bj[p - 1]; --p; }
-    bg[p] = g; bj[p] = j;
-  }
-  int head = 0;
-  for (int r = 0; r < C; ++r) {
-    float cg = head < C ? bg[head] : -INFINITY;
-    int cj = head < C ? bj[head] : 0x7fffffff;
-    int cl = lane;
+  bool bad = false;
+  for (int j0 = 0; j0 < N; j0 += 128) {
+    float gv[4];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float og = __shfl_xor_sync(0xffffffffu, cg, o);
-      const int oj = __shfl_xor_sync(0xffffffffu, cj, o);
-      const int ol = __shfl_xor_sync(0xffffffffu, cl, o);
-      if (knn_better(og, oj, cg, cj)) { cg = og; cj = oj; cl = ol; }
+    for (int q = 0; q < 4; ++q) {  // four loads in flight per lane
+      const int j = j0 + 32 * q + lane;
+      gv[q] = j < N ? row[j] : -INFINITY;
     }
-    if (cl == lane) ++head;
-    if (lane == 0) top_j[(size_t)il * C + r] = (cg == -INFINITY) ? 0x7fffffff : cj;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int j = j0 + 32 * q + lane;
+      float g = gv[q];
+      if (!(g == g)) {
+        bad = true;
+        g = -INFINITY;
+      }
+      if (j >= N || j == i) g = -INFINITY;
+      unsigned mask = __ballot_sync(0xffffffffu, g != -INFINITY && knn_better(g, j, tg, tj));
+      while (mask) {
+        const int src = __ffs(mask) - 1;
+        mask &= mask - 1;
+        const float cg = __shfl_sync(0xffffffffu, g, src);
+        const int cj = __shfl_sync(0xffffffffu, j, src);
+        if (!knn_better(cg, cj, tg, tj)) continue;  // the threshold rose meanwhile (uniform)
+        const int pos = __popc(__ballot_sync(0xffffffffu, lane < K && knn_better(lg, lj, cg, cj)));
+        const float ug = __shfl_up_sync(0xffffffffu, lg, 1);
+        const int uj = __shfl_up_sync(0xffffffffu, lj, 1);
+        if (lane > pos && lane < K) {
+          lg = ug;
+          lj = uj;
+        }
+        if (lane == pos) {
+          lg = cg;
+          lj = cj;
+        }
+        tg = __shfl_sync(0xffffffffu, lg, K - 1);
+        tj = __shfl_sync(0xffffffffu, lj, K - 1);
+      }
+    }
   }
+  if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&g_err_score, RIFT_EBIT_NONFINITE);
+  if (lane < C) top_j[(size_t)il * C + lane] = (lg == -INFINITY) ? 0x7fffffff : lj;
 }
 
 // One CTA per tile, one warp per candidate: recompute the C candidates' similarities to ~fp64
@@ -408,21 +462,19 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
     const float* __restrict__ s_raw, float* __restrict__ s_tilde, int* __restrict__ nbr) {
   pdl_trigger();
   pdl_wait();
-  extern __shared__ float4 vi_sm[];  // V_i, read by every candidate's warp
   __shared__ double g64[RIFT_MAX_KNN];
   __shared__ int jj[RIFT_MAX_KNN];
   const int il = blockIdx.x, i = row0 + il;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int k = threadIdx.x; k < d / 4; k += blockDim.x) vi_sm[k] = reinterpret_cast<const float4*>(V + (size_t)i * d)[k];
-  __syncthreads();
   if (w < C) {
     const int j = top_j[(size_t)il * C + w];
     // Each lane keeps its partial sum as an unevaluated pair hi + lo of floats: the product of
     // two floats is split exactly with an FMA (Dekker's TwoProduct as rewritten by Ogita, Rump
     // and Oishi) and added with Knuth's TwoSum, so the lane sum is good to ~2^-44 relative.
+    // V_i is read by all the CTA's warps (L1 serves all but the first).
     float hi = 0.f, lo = 0.f;
     if (j >= 0 && j < N) {
-      const float4* vi = vi_sm;
+      const float4* vi = reinterpret_cast<const float4*>(V + (size_t)i * d);
       const float4* vj = reinterpret_cast<const float4*>(V + (size_t)j * d);
       for (int k = lane; k < d / 4; k += 32) {
         const float4 a4 = vi[k], b4 = vj[k];
@@ -485,10 +537,9 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
 int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids, int n_tmpl,
                       int n_phrase, const int* bg_ids, int M, float* t, float* B, cudaStream_t st) {
   if (n_tmpl == 1) {
-    launch_ex(query_rows_kernel, dim3((d + 255) / 256), dim3(256), 0, st, true, static_cast<const uint16_t*>(embed),
-              vocab, d, phrase_ids, n_phrase, bg_ids, M, t, B);
-    launch_ex(normalize_rows_kernel, dim3(1 + M), dim3(256), 0, st, true, t, B, d);
-    return 2;
+    launch_ex(query_rows_kernel, dim3(1 + M), dim3(std::min(QR_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
+              static_cast<const uint16_t*>(embed), vocab, d, phrase_ids, n_phrase, bg_ids, M, t, B);
+    return 1;
   }
   // two fp32 rows of d in shared memory: 64 KB at the widest d (8192), past the 48 KB default
   static std::atomic<unsigned long long> smem_raised{0};
@@ -594,11 +645,14 @@ int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, in
     uint16_t* B16 = reinterpret_cast<uint16_t*>(ws + L.split_b_off);
     float* G = reinterpret_cast<float*>(ws + L.gram_off);
     const int Np = (N + 7) & ~7;
-    const size_t n = (size_t)Np * d;
+    const size_t n = (size_t)Np * (d / 8);
     launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, row0, row1,
               A16, B16);
     EpiParams ep;
     ep.out_scale = 1.f / (KNN_SPLIT_SCALE * KNN_SPLIT_SCALE);
+    // the whole scene's rows: G is symmetric (A holds the same rows as B, in the permuted parts
+    // [hi | hi | lo] against [hi | lo | hi], whose product is symmetric up to the order of its sums)
+    ep.symmetric = (row0 == 0 && n_rows == N) ? 1 : 0;
     // split-K partials for products with fewer tiles than SMs (a scene up to ~2000 tiles)
     void* part = L.splitk_bytes ? static_cast<void*>(ws + L.splitk_off) : nullptr;
     // B16 is the split kernel's output, not a constant operand
@@ -608,7 +662,7 @@ int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, in
               n_rows, C, topj);
     launched += 4;
   }
-  launch_ex(knn_rescore_smooth_kernel, dim3(n_rows), dim3(32 * RIFT_MAX_KNN), d * sizeof(float), st, true, V, d,
+  launch_ex(knn_rescore_smooth_kernel, dim3(n_rows), dim3(32 * RIFT_MAX_KNN), 0, st, true, V, d,
             (const int*)topj, N, row0, C, m, s_raw, s_tilde, nbr);
   return launched;
 }
