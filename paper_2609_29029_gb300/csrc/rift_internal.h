@@ -29,11 +29,12 @@ struct SmoothLayout {
   size_t top_off, split_a_off, split_b_off, gram_off, splitk_off, splitk_bytes, total;
 };
 SmoothLayout smooth_layout(int N, int n_rows, int d);
-// rift_score_tiles: the token pass, then V [N, d], then the smoothing of all N rows.
+// rift_score_tiles: V [N, d], then the token pass's scratch, which the smoothing of all N rows
+// reuses once V is formed.
 struct ScoreLayout {
   ShardLayout T;
   SmoothLayout S;
-  size_t V_off, smooth_off, total;
+  size_t V_off, tokens_off, smooth_off, total;
 };
 ScoreLayout score_layout(int N, int n_v, int d, int M);
 // The host-side argument checks shared by the scoring entry points (rift_score_tiles and
@@ -48,12 +49,16 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
                  int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
                  cudaStream_t st);
 // a2, a3 on N tiles: token scores, tile scores and the tile embeddings V [N, d] (ws: shard_layout).
+// A16, B16 (nullable): also write the whole scene's Gram operands (the layout of launch_smooth's
+// split_a / split_b), so that launch_smooth can skip its split.
 int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
-                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st);
+                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st,
+                        uint16_t* A16 = nullptr, uint16_t* B16 = nullptr);
 // a4 for tiles row0 .. row0 + n_rows - 1 of a scene of N tiles (V [N, d], s_raw [N]); s_tilde and
 // nbr are indexed by the local row (ws: smooth_layout).
+// split_done: the split operands in ws were written by launch_score_tokens (whole scene).
 int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, int n_rows, int m, float* s_tilde,
-                  int* nbr, char* ws, cudaStream_t st);
+                  int* nbr, char* ws, cudaStream_t st, bool split_done = false);
 // range = (min, max) of n scores.
 void launch_score_range(const float* s, int n, float* range, cudaStream_t st);
 

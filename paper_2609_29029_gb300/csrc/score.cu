@@ -281,15 +281,23 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
   }
 }
 
+// The fp16 hi/lo split of the Gram operands (see knn_split_kernel): rows of V scaled by 2^10 so
+// that the low parts stay normal in fp16.
+constexpr float KNN_SPLIT_SCALE = 1024.f;
+
 // a3: P_i = sum of the tile's partials (fixed order), V_i = P_i / ||P_i||, s_i = V_i . w.  One CTA
 // per tile, a float4 column per thread (two at d > 4096), so that each thread's partial loads all
-// issue together.
+// issue together.  With A16 and B16 (the whole scene's Gram operands, Np rows of B) it also writes
+// tile i's split rows, as knn_split_kernel would from V, and the zero padding rows of B.
 constexpr int TF_THREADS = 1024;
 __global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart,
                                                                   int n_chunks, int d,
                                                                   const float* __restrict__ w,
                                                                   float* __restrict__ V,
-                                                                  float* __restrict__ s_raw) {
+                                                                  float* __restrict__ s_raw,
+                                                                  uint16_t* __restrict__ A16,
+                                                                  uint16_t* __restrict__ B16, int N,
+                                                                  int Np) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[32];
@@ -320,12 +328,36 @@ __global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* 
     if (c < nv) {
       const float4 v = make_float4(p[k].x * inv, p[k].y * inv, p[k].z * inv, p[k].w * inv);
       reinterpret_cast<float4*>(V + (size_t)i * d)[c] = v;
+      if (B16) {
+        const float a[4] = {v.x * KNN_SPLIT_SCALE, v.y * KNN_SPLIT_SCALE, v.z * KNN_SPLIT_SCALE,
+                            v.w * KNN_SPLIT_SCALE};
+        uint32_t h[2], l[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const __half h0 = __float2half_rn(a[2 * q]), h1 = __float2half_rn(a[2 * q + 1]);
+          h[q] = pack_half2(__half2float(h0), __half2float(h1));
+          l[q] = pack_half2(a[2 * q] - __half2float(h0), a[2 * q + 1] - __half2float(h1));
+        }
+        const uint2 hv = make_uint2(h[0], h[1]), lv = make_uint2(l[0], l[1]);
+        uint2* b = reinterpret_cast<uint2*>(B16 + (size_t)i * 3 * d) + c;
+        uint2* a2 = reinterpret_cast<uint2*>(A16 + (size_t)i * 3 * d) + c;
+        b[0] = hv;
+        b[d / 4] = lv;
+        b[d / 2] = hv;
+        a2[0] = hv;
+        a2[d / 4] = hv;
+        a2[d / 2] = lv;
+      }
       const float4 wc = reinterpret_cast<const float4*>(w)[c];
       dt += v.x * wc.x + v.y * wc.y + v.z * wc.z + v.w * wc.w;
     }
   }
   dt = block_sum(dt, red);
   if (threadIdx.x == 0) s_raw[i] = dt;
+  if (B16)  // the padding rows N .. Np - 1 of B are zero
+    for (int r = N + i; r < Np; r += gridDim.x)
+      for (int c = threadIdx.x; c < 3 * d / 8; c += blockDim.x)
+        reinterpret_cast<uint4*>(B16 + (size_t)r * 3 * d)[c] = make_uint4(0, 0, 0, 0);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -344,7 +376,6 @@ __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
 // by 2^10, so that the low parts stay normal in fp16) is split into hi = fp16(v) and
 // lo = fp16(v - hi); A = [hi | hi | lo] and B = [hi | lo | hi] along K, so one fp16 GEMM with
 // K = 3 d gives hi.hi + hi.lo + lo.hi, i.e. V V^T to ~2^-22 relative (lo.lo is below that).
-constexpr float KNN_SPLIT_SCALE = 1024.f;
 // B holds every tile; A the rows row0 .. row1 - 1 (A row i - row0).  Rows N .. Np - 1 of B (the
 // padding of the Gram matrix's column count to a multiple of 8) are zero.  A thread handles 8
 // consecutive elements of a row (two float4 loads, 16-byte stores into each of the row's parts).
@@ -471,7 +502,9 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
     // Each lane keeps its partial sum as an unevaluated pair hi + lo of floats: the product of
     // two floats is split exactly with an FMA (Dekker's TwoProduct as rewritten by Ogita, Rump
     // and Oishi) and added with Knuth's TwoSum, so the lane sum is good to ~2^-44 relative.
-    // V_i is read by all the CTA's warps (L1 serves all but the first).
+    // V_i is read by all the CTA's warps (L1 serves all but the first).  The kernel moves 16 rows
+    // of V per tile from L2: its time follows those bytes, not the length of this chain (four
+    // independent chains with loads ahead measured slower, at fewer resident CTAs).
     float hi = 0.f, lo = 0.f;
     if (j >= 0 && j < N) {
       const float4* vi = reinterpret_cast<const float4*>(V + (size_t)i * d);
@@ -559,14 +592,14 @@ SmoothLayout smooth_layout(int N, int n_rows, int d) {
   auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
   const size_t Np = ((size_t)N + 7) & ~size_t(7);
   L.top_off = take(sizeof(int) * (size_t)n_rows * RIFT_MAX_KNN);
-  L.split_a_off = take(sizeof(uint16_t) * (size_t)n_rows * 3 * d);
-  L.split_b_off = take(sizeof(uint16_t) * Np * 3 * d);
   L.gram_off = take(sizeof(float) * (size_t)n_rows * Np);
   const size_t slice = sizeof(float) * (size_t)n_rows * Np;
   size_t part = ((size_t)16 << 20) / slice;
   part = part > 16 ? 16 : part;
   L.splitk_bytes = part >= 2 ? part * slice : 0;
   L.splitk_off = take(L.splitk_bytes);
+  L.split_a_off = take(sizeof(uint16_t) * (size_t)n_rows * 3 * d);  // the split operands last
+  L.split_b_off = take(sizeof(uint16_t) * Np * 3 * d);
   L.total = off;
   return L;
 }
@@ -574,7 +607,7 @@ SmoothLayout smooth_layout(int N, int n_rows, int d) {
 // Scratch of the token pass over N tiles: w and the partial pooled sums.
 ShardLayout shard_layout(int N, int n_v, int d) {
   ShardLayout L{};
-  L.chunk_tokens = 96;  // 6 CTAs per 576-token tile
+  L.chunk_tokens = 192;  // 3 CTAs per 576-token tile
   L.n_chunks = (n_v + L.chunk_tokens - 1) / L.chunk_tokens;
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
@@ -589,17 +622,14 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   ScoreLayout L{};
   L.T = shard_layout(N, n_v, d);
   L.S = smooth_layout(N, N, d);
-  // V after the token pass's scratch; the smoothing's scratch over the partial pooled sums, which
-  // are dead once V is formed (the smoothing runs after tile_finalize_kernel on the stream)
-  L.V_off = L.T.total;
-  const size_t v_end = L.V_off + ((sizeof(float) * (size_t)N * d + 255) & ~size_t(255));
-  L.smooth_off = L.T.ppart_off;
-  const size_t s_end = L.smooth_off + L.S.total;
-  L.total = s_end > v_end ? s_end : v_end;
-  if (s_end > L.V_off && L.smooth_off < v_end) {  // overlapping V: place the smoothing after V
-    L.smooth_off = v_end;
-    L.total = v_end + L.S.total;
-  }
+  // V first; after it the token pass's scratch (w, partial pooled sums).  The smoothing's scratch
+  // reuses the token scratch once V is formed (the smoothing runs after tile_finalize_kernel on
+  // the stream), except for its split operands, which tile_finalize_kernel writes while it reads
+  // the partial sums: they start past the token scratch.
+  L.V_off = 0;
+  L.tokens_off = (sizeof(float) * (size_t)N * d + 255) & ~size_t(255);
+  L.smooth_off = L.tokens_off + (L.T.total > L.S.split_a_off ? L.T.total - L.S.split_a_off : 0);
+  L.total = L.smooth_off + L.S.total;
   return L;
 }
 
@@ -611,7 +641,8 @@ static void launch_tokens(const void* X, int N, int n_v, int d, const ShardLayou
 }
 
 int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
-                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st) {
+                        int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st,
+                        uint16_t* A16, uint16_t* B16) {
   const ShardLayout L = shard_layout(N, n_v, d);
   float* w = reinterpret_cast<float*>(ws + L.w_off);
   float* Ppart = reinterpret_cast<float*>(ws + L.ppart_off);
@@ -628,12 +659,12 @@ int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, co
     else launch_tokens<float, 4>(X, N, n_v, d, L, w, token_scores, Ppart, st);
   }
   launch_ex(tile_finalize_kernel, dim3(N), dim3(std::min(TF_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
-            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw);
+            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw, A16, B16, N, (N + 7) & ~7);
   return 3;
 }
 
 int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, int n_rows, int m, float* s_tilde,
-                  int* nbr, char* ws, cudaStream_t st) {
+                  int* nbr, char* ws, cudaStream_t st, bool split_done) {
   const SmoothLayout L = smooth_layout(N, n_rows, d);
   const int row1 = row0 + n_rows;
   int* topj = reinterpret_cast<int*>(ws + L.top_off);
@@ -646,8 +677,9 @@ int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, in
     float* G = reinterpret_cast<float*>(ws + L.gram_off);
     const int Np = (N + 7) & ~7;
     const size_t n = (size_t)Np * (d / 8);
-    launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, row0, row1,
-              A16, B16);
+    if (!split_done)
+      launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, row0,
+                row1, A16, B16);
     EpiParams ep;
     ep.out_scale = 1.f / (KNN_SPLIT_SCALE * KNN_SPLIT_SCALE);
     // the whole scene's rows: G is symmetric (A holds the same rows as B, in the permuted parts
@@ -660,7 +692,7 @@ int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, in
       return -1;
     launch_ex(knn_gram_topc_kernel, dim3((n_rows + 3) / 4), dim3(128), 0, st, true, (const float*)G, N, Np, row0,
               n_rows, C, topj);
-    launched += 4;
+    launched += split_done ? 3 : 4;
   }
   launch_ex(knn_rescore_smooth_kernel, dim3(n_rows), dim3(32 * RIFT_MAX_KNN), 0, st, true, V, d,
             (const int*)topj, N, row0, C, m, s_raw, s_tilde, nbr);
@@ -672,8 +704,12 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
                  cudaStream_t st) {
   const ScoreLayout L = score_layout(N, n_v, d, M);
   float* V = reinterpret_cast<float*>(ws + L.V_off);
-  const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws, st);
-  const int b = launch_smooth(V, s_raw, N, d, 0, N, m, s_tilde, nbr, ws + L.smooth_off, st);
+  // with neighbours to find, tile_finalize_kernel also writes the Gram's split operands
+  uint16_t* A16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_a_off) : nullptr;
+  uint16_t* B16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_b_off) : nullptr;
+  const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws + L.tokens_off, st, A16,
+                                    B16);
+  const int b = launch_smooth(V, s_raw, N, d, 0, N, m, s_tilde, nbr, ws + L.smooth_off, st, m > 0);
   return b < 0 ? -1 : a + b;
 }
 
