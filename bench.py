@@ -46,11 +46,12 @@ def parse():
     ap.add_argument("--ncu-summary", metavar="CSV", help="summarise an ncu launch list (gpu__time_duration.sum) and exit")
     ap.add_argument("--sweep", action="store_true",
                     help="scoring/select/gather-only sweep over N in {100, 400, 1600, 6400} tiles (one JSON line per N)")
-    ap.add_argument("--kernel-case", choices=["prefill", "prefill_full", "score", "decode", "merge"],
+    ap.add_argument("--kernel-case", choices=["prefill", "prefill_full", "score", "decode", "merge", "attention"],
                     help="small profiling case: 'prefill' = one 7B-shaped layer over 12 sequences (T = 4092), "
                          "'prefill_full' = one 7B-shaped layer over the 400-tile query's retained length mix "
-                         "(73 sequences, T = 23,819), 'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens); "
-                         "each runs 3 times")
+                         "(73 sequences, T = 23,819), 'score' = Eq. 1 scoring of 64 tiles (302 MB of tokens), "
+                         "'attention' = the varlen attention alone over ~23.6K rows of sequences of one length, "
+                         "for lengths 131 to 4096 (CUDA events, one JSON line per length); the others run 3 times")
     return ap.parse_args()
 
 
@@ -510,6 +511,40 @@ def kernel_case(name: str):
         for _ in range(3):
             hid = H0.clone()
             abi.prefill_layers(dm.struct, hid, T, cu, len(lens), 635, pos, ws, need)
+        abi.sync_status()
+    elif name == "attention":
+        # the attention of one 7B-shaped layer over equal-length sequences: time per length
+        H, HD = 32, 128
+        d = H * HD
+        peaks = json.loads((ROOT / "MEASURED_PEAKS.json").read_text()) if (ROOT / "MEASURED_PEAKS.json").exists() else {}
+        hbm = peaks.get("hbm_gbs", 6796.5)
+        flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+        from synth import rng
+        for L in (131, 203, 256, 347, 512, 1024, 2048, 4096):
+            n = max(1, 23819 // L)
+            T = n * L
+            qkv = rng.normal_f32(0, rng.stream_id("case-attn", L), T * 3 * d, dev).view(T, 3 * d).to(torch.float16)
+            out = torch.empty(T, d, dtype=torch.float16, device=dev)
+            cu = torch.tensor([i * L for i in range(n + 1)], dtype=torch.int32, device=dev)
+            need = abi.attention_workspace_bytes(T, n)
+            ws = torch.empty(need, dtype=torch.uint8, device=dev)
+            for _ in range(3):
+                abi.attention_varlen(qkv, T, cu, n, H, HD, out, ws, need)
+            times = []
+            for _ in range(10):
+                flush.fill_(1)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                abi.attention_varlen(qkv, T, cu, n, H, HD, out, ws, need)
+                e1.record()
+                torch.cuda.synchronize()
+                times.append(e0.elapsed_time(e1))
+            ms = statistics.median(times)
+            blocks = n * H * sum(-(-min(L, 128 * b + 128) // 64) for b in range(-(-L // 128)))
+            print(json.dumps({"L": L, "sequences": n, "T": T, "us": round(1e3 * ms, 1), "kv_blocks": blocks,
+                              "us_per_block_per_cta_slot": round(1e3 * ms * 2 * 152 / blocks, 3),
+                              "of_hbm_floor": round(8 * d * T / (ms / 1e3) / (hbm * 1e9), 3)}), flush=True)
+            del qkv, out, ws
         abi.sync_status()
     elif name == "merge":
         # the 400-tile scene's selection with Stage 2's merge, three times
