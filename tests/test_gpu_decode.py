@@ -153,6 +153,13 @@ def test_split_k_decode_on_a_synthetic_batch(cuda, riftlib):
     riftlib.decode_step(dm.struct, kv, T, cu_d, n, max_len, torch.tensor(ids, dtype=torch.int32, device=cuda),
                         embed, 300, hid, kvn, lg, ws, need)
     riftlib.sync_status()
+    # the reductions inside the products and the attention leave their arrival counters zeroed:
+    # a second step on the same workspace gives the same bits
+    hid2, kvn2, lg2 = torch.empty_like(hid), torch.empty_like(kvn), torch.empty_like(lg)
+    riftlib.decode_step(dm.struct, kv, T, cu_d, n, max_len, torch.tensor(ids, dtype=torch.int32, device=cuda),
+                        embed, 300, hid2, kvn2, lg2, ws, need)
+    riftlib.sync_status()
+    assert torch.equal(hid, hid2) and torch.equal(kvn, kvn2) and torch.equal(lg, lg2)
     get = lambda l: layers[l]
     worst = {}
     for j in range(n):
