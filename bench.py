@@ -321,17 +321,28 @@ def gemm_traffic(workload: str):
     return int(b.group(1))
 
 
-def select_latency(pipe, sc, q, bg, sy, steps: int, stream=None) -> float:
-    """ms per query of scoring + selection + packing (the pre-prefill path), queries enqueued back
-    to back and timed by events around them only."""
+def select_latency(pipe, sc, q, bg, sy, steps: int, stream=None, batches: int = 5) -> float:
+    """ms per query of scoring + selection + packing (the pre-prefill path): `batches` batches of
+    `steps` queries enqueued back to back, each timed by events around it only, and the median
+    batch reported (the first batch after a long power-capped prefill loop can run at a lower
+    clock).  The stream is held by a short device-side sleep while the host enqueues a batch, so
+    that the events time the device's work and not the host's launch rate (a query is ~15
+    launches of well under a millisecond in all)."""
     st = stream if stream is not None else torch.cuda.current_stream()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(st)
-    for _ in range(steps):
-        pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False, counts=False, stream=st)
-    e1.record(st)
-    torch.cuda.synchronize()
-    return e0.elapsed_time(e1) / steps
+    times = []
+    for _ in range(batches):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if hasattr(torch.cuda, "_sleep"):
+            with torch.cuda.stream(st):
+                torch.cuda._sleep(int(2e6) * steps)  # ~1 ms of clock cycles per query at ~2 GHz
+        e0.record(st)
+        for _ in range(steps):
+            pipe.run(sc.X, sc.embed, q, bg, sy, q, prefill=False, counts=False, stream=st)
+        e1.record(st)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1) / steps)
+    print("select latency per batch (ms/query): " + " ".join(f"{t:.4f}" for t in times), file=sys.stderr)
+    return statistics.median(times)
 
 
 def sweep(steps: int, warmup: int):
@@ -423,6 +434,9 @@ def decode_measure(pipe, dm, sc, dec, n_kept, T, stream, steps):
         one()
     abi.sync_status(stream)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if hasattr(torch.cuda, "_sleep"):  # hold the stream while the host enqueues (see select_latency)
+        with torch.cuda.stream(stream):
+            torch.cuda._sleep(int(4e6) * steps)
     e0.record(stream)
     for _ in range(steps):
         one()
