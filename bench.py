@@ -345,6 +345,22 @@ def select_latency(pipe, sc, q, bg, sy, steps: int, stream=None, batches: int = 
     return statistics.median(times)
 
 
+def select_gather(n_kept: int, T: int, scene, x_elem: int, select_ms: float, pack_ms: float, hbm: float):
+    """HBM roofline of selection + gather (prune/budgets, top-b, sequence offsets, packing) for one
+    query: its algorithmic bytes -- the kept tiles' token scores r read, the selected token ids
+    written and read back, the selected vision tokens and the prompt rows of the embedding table
+    read, the packed rows written -- over the device time of the select and pack kernel classes."""
+    if not (select_ms + pack_ms) > 0:
+        return None
+    sigma_b = T - n_kept * (scene.S + scene.Q)
+    nbytes = (n_kept * scene.n_v * 4 + 2 * sigma_b * 4 + sigma_b * scene.d * x_elem
+              + n_kept * (scene.S + scene.Q) * scene.d * 2 + T * scene.d * 2)
+    ms = select_ms + pack_ms
+    gbs = nbytes / (ms / 1e3) / 1e9
+    return {"bytes_per_query": nbytes, "ms_per_query": ms, "achieved_gbs": gbs, "peak_gbs": hbm, "frac": gbs / hbm,
+            "kernels": "select and pack classes: prune/budgets, top-b, sequence offsets, packing"}
+
+
 def sweep(steps: int, warmup: int):
     """Scoring + selection + packing (no prefill) of the Rift policy over N tiles: per-step device
     time, per-kernel-class time, and the HBM rate of the token pass (N n_v d 2 bytes read)."""
@@ -377,7 +393,9 @@ def sweep(steps: int, warmup: int):
         line = {"sweep": f"select+gather N={N}", "ms_per_query": ms,
                 "kernels_ms": {k: round(v[0] / steps, 4) for k, v in prof.items() if v[1]},
                 "kept_tiles": n_kept, "packed_rows": T, "x_bytes": x_bytes,
-                "token_pass_lower_bound_ms": x_bytes / (hbm * 1e6)}
+                "token_pass_lower_bound_ms": x_bytes / (hbm * 1e6),
+                "select_gather": select_gather(n_kept, T, s, sc.X.element_size(), prof["select"][0] / steps,
+                                               prof["pack"][0] / steps, hbm)}
         print(json.dumps(line), flush=True)
         del sc, pipe
         torch.cuda.empty_cache()
@@ -770,8 +788,13 @@ def main():
     gemm_flops = args.steps * T * dec.linear_flops_per_token
     achieved = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
     traffic = gemm_traffic(wl.name)
+    peak_burst = peaks.get("bf16_tflops", 1887.6)
     per_step = {k: round(v[0] / args.steps, 3) for k, v in prof.items()}
     x_bytes = sc.X.numel() * sc.X.element_size()
+    hbm = peaks.get("hbm_gbs", 6796.5)
+    sigma_b = T - n_kept * (s.S + s.Q)
+    sel_gather = select_gather(n_kept, T, s, sc.X.element_size(), prof["select"][0] / args.steps,
+                               prof["pack"][0] / args.steps, hbm)
 
     cpu = None
     if not args.no_cpu_baseline and ws == 1:
@@ -792,12 +815,15 @@ def main():
                    "l2": l2_note(sc.X.numel() * sc.X.element_size(), dec.n_layers * dec.params_per_layer * 2,
                                  flush is not None)},
         "scene_queries_per_s": 1e3 * args.steps / ms_max,
+        "vision_tokens_per_s": value * sigma_b / max(T, 1),
         "select_latency_ms": sel_ms,
-        "select_latency_floor_ms": x_bytes / (peaks.get("hbm_gbs", 6796.5) * 1e6),
+        "select_latency_floor_ms": x_bytes / (hbm * 1e6),
+        "select_gather": sel_gather,
         "kernels_ms_per_step": per_step,
         "roofline": {"bound": "tensor", "kernel": "prefill GEMM", "achieved": achieved, "peak": peak,
                      "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None, "traffic": traffic,
                      "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained (of measured)",
+                     "peak_burst": peak_burst, "frac_burst": (achieved / peak_burst) if achieved else None,
                      "launches": gemm_n},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h,

@@ -84,3 +84,17 @@ def test_l2_note_and_traffic_belong_to_the_workload():
     assert bench.gemm_traffic("tiny") is None
     t = bench.gemm_traffic(bench.PROFILED_WORKLOAD)
     assert t is None or t > 0
+
+
+def test_select_gather_roofline_counts_the_algorithmic_bytes():
+    from types import SimpleNamespace
+    import bench
+    sc = SimpleNamespace(S=35, Q=24, n_v=576, d=4096)
+    n_kept, T = 3, 3 * (35 + 24) + 500  # 500 selected vision tokens
+    r = bench.select_gather(n_kept, T, sc, 2, 0.01, 0.03, 6796.5)
+    want = 3 * 576 * 4 + 2 * 500 * 4 + 500 * 4096 * 2 + 3 * 59 * 4096 * 2 + T * 4096 * 2
+    assert r["bytes_per_query"] == want
+    assert abs(r["ms_per_query"] - 0.04) < 1e-12
+    assert abs(r["achieved_gbs"] - want / 0.04e-3 / 1e9) < 1e-6
+    assert abs(r["frac"] - r["achieved_gbs"] / 6796.5) < 1e-12
+    assert bench.select_gather(n_kept, T, sc, 2, 0.0, 0.0, 6796.5) is None
