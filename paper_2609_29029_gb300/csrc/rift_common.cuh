@@ -30,19 +30,20 @@
 
 namespace rift {
 
-// Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current device, once per
-// device: a function's attributes belong to each device's context, so a process that drives
-// several GPUs needs the call on every one of them.  `done` is the call site's record of the
-// devices already raised (a device id of 64 or more is raised on every call).
+// The unique id of the calling thread's current CUDA context (cuCtxGetId: ids are never reused
+// within a process, unlike context handles), or 0 if it cannot be read.  (rift_abi.cu)
+unsigned long long current_context_id();
+
+// Raises `kernel`'s dynamic shared-memory limit to `bytes` in the current CUDA context.  A
+// function's attributes belong to a context (every device's primary context, and any context a
+// host creates with the driver API has its own), so `done`, the call site's record, holds the id
+// of the context last raised; a call from another context (or with an unreadable id) raises again.
 template <typename K>
 inline cudaError_t raise_smem_limit(std::atomic<unsigned long long>& done, K* kernel, int bytes) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  const unsigned long long bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0ull;
-  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
-  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+  const unsigned long long ctx = current_context_id();
+  if (ctx != 0 && done.load(std::memory_order_acquire) == ctx) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && ctx != 0) done.store(ctx, std::memory_order_release);
   return e;
 }
 

@@ -33,30 +33,6 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_score_scratch[RIFT_NOALLOC_SCORE_SCRATCH_BYTES];
 
-// The unique id of the calling thread's current CUDA context (cuCtxGetId: ids are never reused
-// within a process, unlike context handles), or 0 if it cannot be read.
-unsigned long long current_context_id() {
-  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
-  static PFN_cuCtxGetId_v12000 get_id = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
-    p = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
-  });
-  CUcontext ctx = nullptr;
-  unsigned long long id = 0;
-  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
-    return 0;
-  return id;
-}
-
 // The addresses recorded by uncaptured calls, one per context id (a small table: a process rarely
 // has more than one context per device).
 constexpr int kMaxContexts = 64;
@@ -69,7 +45,7 @@ int g_n_ctx = 0;
 rift_status scratch_address(cudaStream_t stream, void** out) {
   cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
   if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) return RIFT_ERR_CUDA;
-  const unsigned long long id = current_context_id();
+  const unsigned long long id = rift::current_context_id();
   std::lock_guard<std::mutex> lk(g_mu);
   int slot = -1;
   for (int i = 0; i < g_n_ctx; ++i)

@@ -84,6 +84,79 @@ def test_noalloc_tensor_core_gram_branch_twice_in_a_row(cuda, riftlib):
         _check(ref, got)
 
 
+class _Driver:
+    """The few CUDA driver calls the second-context test needs, through ctypes."""
+
+    def __init__(self):
+        import ctypes
+        self.C = ctypes
+        self.lib = ctypes.CDLL("libcuda.so.1")
+
+    def __call__(self, name, *args):
+        rc = getattr(self.lib, name)(*args)
+        assert rc == 0, f"{name} returned {rc}"
+
+    def alloc_copy(self, host_bytes):
+        C = self.C
+        p = C.c_uint64(0)
+        self("cuMemAlloc_v2", C.byref(p), C.c_size_t(max(len(host_bytes), 16)))
+        if host_bytes:
+            buf = C.create_string_buffer(host_bytes, len(host_bytes))
+            self("cuMemcpyHtoD_v2", p, buf, C.c_size_t(len(host_bytes)))
+        return p.value
+
+    def read(self, dptr, nbytes):
+        C = self.C
+        buf = C.create_string_buffer(nbytes)
+        self("cuMemcpyDtoH_v2", buf, C.c_uint64(dptr), C.c_size_t(nbytes))
+        return buf.raw
+
+
+def test_noalloc_in_a_second_context_of_the_device(cuda, riftlib):
+    # A host that drives the GPU through its own driver-API context (not the runtime's primary
+    # context) gets its own copy of the fixed array at another address: the call must look the
+    # address up in the context that is current, and the primary context must keep working after.
+    import numpy as np
+    wl = P.SMALL24
+    s = wl.scene
+    sc = _scene(wl, cuda)
+    xdt = riftlib.RIFT_BF16 if s.x_dtype == "bf16" else riftlib.RIFT_F32
+    ref, _ = _score_both(riftlib, wl, sc, cuda)
+    t, B = _query(riftlib, sc, wl, cuda)
+    host = {k: v.cpu().numpy() for k, v in dict(X=sc.X, t=t, B=B).items()}
+    want = {k: v.cpu().numpy() for k, v in ref.items()}
+    torch.cuda.synchronize()
+    drv = _Driver()
+    C = drv.C
+    drv("cuInit", 0)
+    dev, ctx = C.c_int(0), C.c_void_p(0)
+    drv("cuDeviceGet", C.byref(dev), 0)
+    drv("cuCtxCreate_v2", C.byref(ctx), 0, dev)  # created and made current on this thread
+    try:
+        d_in = {k: drv.alloc_copy(np.ascontiguousarray(v).tobytes()) for k, v in host.items()}
+        d_out = {k: drv.alloc_copy(bytes(v.nbytes)) for k, v in want.items()}
+        status = riftlib.lib.rift_score_tiles_noalloc(d_in["X"], xdt, s.N, s.n_v, s.d, d_in["t"], d_in["B"], s.M,
+                                                      wl.knn_m, d_out["r"], d_out["s0"], d_out["s1"], d_out["nbr"],
+                                                      None)
+        assert status == riftlib.RIFT_OK
+        drv("cuCtxSynchronize")
+        assert riftlib.lib.rift_sync_status(None) == riftlib.RIFT_OK
+        got = {k: np.frombuffer(drv.read(d_out[k], v.nbytes), dtype=v.dtype).reshape(v.shape) for k, v in want.items()}
+        for p in list(d_in.values()) + list(d_out.values()):
+            drv("cuMemFree_v2", C.c_uint64(p))
+    finally:
+        popped = C.c_void_p(0)
+        drv("cuCtxPopCurrent_v2", C.byref(popped))
+        drv("cuCtxDestroy_v2", ctx)
+    assert P.rel_err_rows(got["r"], want["r"]) < P.SCORE_RTOL
+    assert P.max_abs_rel(torch.from_numpy(got["s0"].copy()), torch.from_numpy(want["s0"])) < P.SCORE_RTOL
+    assert P.max_abs_rel(torch.from_numpy(got["s1"].copy()), torch.from_numpy(want["s1"])) < P.SCORE_RTOL
+    assert np.array_equal(got["nbr"], want["nbr"])
+    # back in the primary context: its own array, its own address
+    ref2, got2 = _score_both(riftlib, wl, sc, cuda)
+    _check(ref2, got2)
+
+
 def test_noalloc_rejects_scenes_larger_than_its_array(cuda, riftlib):
     N, n_v, d, M = 2000, 576, 4096, 8
     assert riftlib.score_workspace_bytes(N, n_v, d, M) > riftlib.NOALLOC_SCORE_SCRATCH_BYTES
