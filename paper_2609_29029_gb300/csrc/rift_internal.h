@@ -21,7 +21,7 @@ unsigned int read_clear_err_gemm();
 // The token pass over N tiles (Eq. 1 per token, pooled sums): w and the partial pooled sums.
 struct ShardLayout {
   int chunk_tokens, n_chunks;
-  size_t w_off, ppart_off, total;
+  size_t w_off, cnt_off, ppart_off, total;
 };
 ShardLayout shard_layout(int N, int n_v, int d);
 // The kNN smoothing of n_rows rows against all N tiles (Appendix B Step 2).

@@ -4,8 +4,8 @@
 // HBM-bound part: token_score_kernel makes the one pass over X [N, n_v, d].  Per token it
 // forms x.w and ||x||^2 (fp32), giving r = x.w / ||x|| with w = t - (1/M) sum_j B_j (Eq. 1
 // with the background mean folded into one vector), and it adds the token into the tile's
-// pooled sum P_i.  Several CTAs share a tile; each writes its partial P to the workspace and
-// tile_finalize_kernel adds them in a fixed order.
+// pooled sum P_i.  Several CTAs share a tile; each writes its partial P to the workspace, and
+// the one that writes the tile's last partial adds them in a fixed order and finalises the tile.
 #include <algorithm>
 
 #include "rift_internal.h"
@@ -136,16 +136,106 @@ __global__ void __launch_bounds__(QR_THREADS) query_rows_kernel(const uint16_t* 
   }
 }
 
-// w = t - (1/M) sum_j B_j  (M = 0: w = t)
+// w = t - (1/M) sum_j B_j  (M = 0: w = t).  Also zeroes the token pass's per-tile arrival
+// counters cnt[0 .. N) (every finalising CTA leaves its counter zeroed again).
 __global__ void fold_w_kernel(const float* __restrict__ t, const float* __restrict__ B, int M,
-                              int d, float* __restrict__ w) {
+                              int d, float* __restrict__ w, unsigned int* __restrict__ cnt, int N) {
   pdl_trigger();
   pdl_wait();
   int c = blockIdx.x * blockDim.x + threadIdx.x;
+  for (int k = c; k < N; k += gridDim.x * blockDim.x) cnt[k] = 0u;
   if (c >= d) return;
   float s = 0.f;
   for (int j = 0; j < M; ++j) s += B[(size_t)j * d + c];
   w[c] = M > 0 ? t[c] - s / (float)M : t[c];
+}
+
+// The fp16 hi/lo split of the Gram operands (see knn_split_kernel): rows of V scaled by 2^10 so
+// that the low parts stay normal in fp16.
+constexpr float KNN_SPLIT_SCALE = 1024.f;
+
+// a3 for tile i, by one CTA of any size (MAXC >= the float4 columns a thread holds): P_i = sum of
+// the tile's n_chunks partials (in chunk order), V_i = P_i / ||P_i||, s_i = V_i . w.  A thread
+// takes the float4 columns threadIdx.x + k blockDim.x, so that its partial loads all issue
+// together; the partials are read through L2 (other CTAs wrote them).  With A16 and B16 (the whole
+// scene's Gram operands, Np rows of B) it also writes tile i's split rows, as knn_split_kernel
+// would from V, and its share of the zero padding rows of B.
+template <int MAXC>
+__device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ Ppart, int n_chunks, int d,
+                                              const float* __restrict__ w, float* __restrict__ V,
+                                              float* __restrict__ s_raw, uint16_t* __restrict__ A16,
+                                              uint16_t* __restrict__ B16, int N, int Np, float* red) {
+  const int nv = d / 4;
+  float4 p[MAXC];
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < MAXC; ++k) {
+    const int c = threadIdx.x + k * blockDim.x;
+    p[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c < nv) {
+      const float4* src = reinterpret_cast<const float4*>(Ppart + (size_t)i * n_chunks * d) + c;
+      for (int q = 0; q < n_chunks; ++q) {
+        const float4 v = __ldcg(src + (size_t)q * nv);
+        p[k].x += v.x;
+        p[k].y += v.y;
+        p[k].z += v.z;
+        p[k].w += v.w;
+      }
+      ss += p[k].x * p[k].x + p[k].y * p[k].y + p[k].z * p[k].z + p[k].w * p[k].w;
+    }
+  }
+  const float inv = 1.f / sqrtf(block_sum(ss, red));
+  float dt = 0.f;
+#pragma unroll
+  for (int k = 0; k < MAXC; ++k) {
+    const int c = threadIdx.x + k * blockDim.x;
+    if (c < nv) {
+      const float4 v = make_float4(p[k].x * inv, p[k].y * inv, p[k].z * inv, p[k].w * inv);
+      reinterpret_cast<float4*>(V + (size_t)i * d)[c] = v;
+      if (B16) {
+        const float a[4] = {v.x * KNN_SPLIT_SCALE, v.y * KNN_SPLIT_SCALE, v.z * KNN_SPLIT_SCALE,
+                            v.w * KNN_SPLIT_SCALE};
+        uint32_t h[2], l[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const __half h0 = __float2half_rn(a[2 * q]), h1 = __float2half_rn(a[2 * q + 1]);
+          h[q] = pack_half2(__half2float(h0), __half2float(h1));
+          l[q] = pack_half2(a[2 * q] - __half2float(h0), a[2 * q + 1] - __half2float(h1));
+        }
+        const uint2 hv = make_uint2(h[0], h[1]), lv = make_uint2(l[0], l[1]);
+        uint2* b = reinterpret_cast<uint2*>(B16 + (size_t)i * 3 * d) + c;
+        uint2* a2 = reinterpret_cast<uint2*>(A16 + (size_t)i * 3 * d) + c;
+        b[0] = hv;
+        b[d / 4] = lv;
+        b[d / 2] = hv;
+        a2[0] = hv;
+        a2[d / 4] = hv;
+        a2[d / 2] = lv;
+      }
+      const float4 wc = reinterpret_cast<const float4*>(w)[c];
+      dt += v.x * wc.x + v.y * wc.y + v.z * wc.z + v.w * wc.w;
+    }
+  }
+  dt = block_sum(dt, red);
+  if (threadIdx.x == 0) s_raw[i] = dt;
+  if (B16)  // the padding rows N .. Np - 1 of B are zero: tile i takes rows N + i, N + i + N, ...
+    for (int r = N + i; r < Np; r += N)
+      for (int c = threadIdx.x; c < 3 * d / 8; c += blockDim.x)
+        reinterpret_cast<uint4*>(B16 + (size_t)r * 3 * d)[c] = make_uint4(0, 0, 0, 0);
+}
+
+// a3 after the token pass (small scenes): one CTA of up to 1024 threads per tile.
+constexpr int TF_THREADS = 1024;
+__global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart, int n_chunks,
+                                                                  int d, const float* __restrict__ w,
+                                                                  float* __restrict__ V, float* __restrict__ s_raw,
+                                                                  uint16_t* __restrict__ A16,
+                                                                  uint16_t* __restrict__ B16, int N, int Np) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[32];
+  finalize_tile<(8192 / 4 + TF_THREADS - 1) / TF_THREADS>(blockIdx.x, Ppart, n_chunks, d, w, V, s_raw, A16, B16, N,
+                                                          Np, red);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -195,7 +285,9 @@ template <typename XT, int NVEC>
 __global__ void __launch_bounds__(SC_THREADS, 2)
     token_score_kernel(const XT* __restrict__ X, int n_v, int d, int chunk_tokens, int n_chunks,
                        const float* __restrict__ w, float* __restrict__ token_scores,
-                       float* __restrict__ Ppart) {
+                       float* __restrict__ Ppart, unsigned int* __restrict__ cnt, float* __restrict__ V,
+                       float* __restrict__ s_raw, uint16_t* __restrict__ A16, uint16_t* __restrict__ B16, int N,
+                       int Np) {
   pdl_trigger();
   pdl_wait();
   using VT = VecTraits<XT>;
@@ -279,85 +371,24 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
         *reinterpret_cast<float4*>(out + v * VW + e) = make_float4(P[j][e], P[j][e + 1], P[j][e + 2], P[j][e + 3]);
     }
   }
-}
-
-// The fp16 hi/lo split of the Gram operands (see knn_split_kernel): rows of V scaled by 2^10 so
-// that the low parts stay normal in fp16.
-constexpr float KNN_SPLIT_SCALE = 1024.f;
-
-// a3: P_i = sum of the tile's partials (fixed order), V_i = P_i / ||P_i||, s_i = V_i . w.  One CTA
-// per tile, a float4 column per thread (two at d > 4096), so that each thread's partial loads all
-// issue together.  With A16 and B16 (the whole scene's Gram operands, Np rows of B) it also writes
-// tile i's split rows, as knn_split_kernel would from V, and the zero padding rows of B.
-constexpr int TF_THREADS = 1024;
-__global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart,
-                                                                  int n_chunks, int d,
-                                                                  const float* __restrict__ w,
-                                                                  float* __restrict__ V,
-                                                                  float* __restrict__ s_raw,
-                                                                  uint16_t* __restrict__ A16,
-                                                                  uint16_t* __restrict__ B16, int N,
-                                                                  int Np) {
-  pdl_trigger();
-  pdl_wait();
-  __shared__ float red[32];
-  const int i = blockIdx.x, nv = d / 4;
-  float4 p[2];
-  float ss = 0.f;
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const int c = threadIdx.x + k * TF_THREADS;
-    p[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (c < nv) {
-      const float4* src = reinterpret_cast<const float4*>(Ppart + (size_t)i * n_chunks * d) + c;
-      for (int q = 0; q < n_chunks; ++q) {
-        const float4 v = src[(size_t)q * nv];
-        p[k].x += v.x;
-        p[k].y += v.y;
-        p[k].z += v.z;
-        p[k].w += v.w;
-      }
-      ss += p[k].x * p[k].x + p[k].y * p[k].y + p[k].z * p[k].z + p[k].w * p[k].w;
-    }
+  // With cnt (large scenes), the CTA that stores the tile's last partial finalises the tile (the
+  // classic last-block reduction: every thread's stores are fenced before the count; the
+  // finalising CTA fences before it reads the other partials), so no finalisation kernel follows
+  // the pass.  Without it, tile_finalize_kernel does the same after the pass.
+  if (!cnt) return;
+  __shared__ unsigned int last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const bool l = atomicAdd(cnt + tile, 1u) == (unsigned)n_chunks - 1u;
+    if (l) atomicExch(cnt + tile, 0u);
+    last = l;
   }
-  const float inv = 1.f / sqrtf(block_sum(ss, red));
-  float dt = 0.f;
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const int c = threadIdx.x + k * TF_THREADS;
-    if (c < nv) {
-      const float4 v = make_float4(p[k].x * inv, p[k].y * inv, p[k].z * inv, p[k].w * inv);
-      reinterpret_cast<float4*>(V + (size_t)i * d)[c] = v;
-      if (B16) {
-        const float a[4] = {v.x * KNN_SPLIT_SCALE, v.y * KNN_SPLIT_SCALE, v.z * KNN_SPLIT_SCALE,
-                            v.w * KNN_SPLIT_SCALE};
-        uint32_t h[2], l[2];
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const __half h0 = __float2half_rn(a[2 * q]), h1 = __float2half_rn(a[2 * q + 1]);
-          h[q] = pack_half2(__half2float(h0), __half2float(h1));
-          l[q] = pack_half2(a[2 * q] - __half2float(h0), a[2 * q + 1] - __half2float(h1));
-        }
-        const uint2 hv = make_uint2(h[0], h[1]), lv = make_uint2(l[0], l[1]);
-        uint2* b = reinterpret_cast<uint2*>(B16 + (size_t)i * 3 * d) + c;
-        uint2* a2 = reinterpret_cast<uint2*>(A16 + (size_t)i * 3 * d) + c;
-        b[0] = hv;
-        b[d / 4] = lv;
-        b[d / 2] = hv;
-        a2[0] = hv;
-        a2[d / 4] = hv;
-        a2[d / 2] = lv;
-      }
-      const float4 wc = reinterpret_cast<const float4*>(w)[c];
-      dt += v.x * wc.x + v.y * wc.y + v.z * wc.z + v.w * wc.w;
-    }
-  }
-  dt = block_sum(dt, red);
-  if (threadIdx.x == 0) s_raw[i] = dt;
-  if (B16)  // the padding rows N .. Np - 1 of B are zero
-    for (int r = N + i; r < Np; r += gridDim.x)
-      for (int c = threadIdx.x; c < 3 * d / 8; c += blockDim.x)
-        reinterpret_cast<uint4*>(B16 + (size_t)r * 3 * d)[c] = make_uint4(0, 0, 0, 0);
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  finalize_tile<(8192 / 4 + SC_THREADS - 1) / SC_THREADS>(tile, Ppart, n_chunks, d, w, V, s_raw, A16, B16, N, Np,
+                                                          &red[0][0]);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -604,7 +635,8 @@ SmoothLayout smooth_layout(int N, int n_rows, int d) {
   return L;
 }
 
-// Scratch of the token pass over N tiles: w and the partial pooled sums.
+// Scratch of the token pass over N tiles: w, the per-tile arrival counters and the partial pooled
+// sums.
 ShardLayout shard_layout(int N, int n_v, int d) {
   ShardLayout L{};
   L.chunk_tokens = 192;  // 3 CTAs per 576-token tile
@@ -612,6 +644,7 @@ ShardLayout shard_layout(int N, int n_v, int d) {
   size_t off = 0;
   auto take = [&](size_t bytes) { size_t o = off; off += (bytes + 255) & ~size_t(255); return o; };
   L.w_off = take(sizeof(float) * d);
+  L.cnt_off = take(sizeof(unsigned int) * (size_t)N);
   L.ppart_off = take(sizeof(float) * (size_t)N * L.n_chunks * d);
   L.total = off;
   return L;
@@ -622,10 +655,10 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   ScoreLayout L{};
   L.T = shard_layout(N, n_v, d);
   L.S = smooth_layout(N, N, d);
-  // V first; after it the token pass's scratch (w, partial pooled sums).  The smoothing's scratch
-  // reuses the token scratch once V is formed (the smoothing runs after tile_finalize_kernel on
-  // the stream), except for its split operands, which tile_finalize_kernel writes while it reads
-  // the partial sums: they start past the token scratch.
+  // V first; after it the token pass's scratch (w, counters, partial pooled sums).  The
+  // smoothing's scratch reuses the token scratch once the pass is over (the smoothing runs after it
+  // on the stream), except for its split operands, which the pass's finalising CTAs write while
+  // other tiles' partial sums are still in use: they start past the token scratch.
   L.V_off = 0;
   L.tokens_off = (sizeof(float) * (size_t)N * d + 255) & ~size_t(255);
   L.smooth_off = L.tokens_off + (L.T.total > L.S.split_a_off ? L.T.total - L.S.split_a_off : 0);
@@ -635,9 +668,11 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
 
 template <typename XT, int NVEC>
 static void launch_tokens(const void* X, int N, int n_v, int d, const ShardLayout& L, const float* w,
-                          float* token_scores, float* Ppart, cudaStream_t st) {
+                          float* token_scores, float* Ppart, unsigned int* cnt, float* V, float* s_raw,
+                          uint16_t* A16, uint16_t* B16, cudaStream_t st) {
   launch_ex(token_score_kernel<XT, NVEC>, dim3(N * L.n_chunks), dim3(SC_THREADS), 0, st, true,
-            static_cast<const XT*>(X), n_v, d, L.chunk_tokens, L.n_chunks, (const float*)w, token_scores, Ppart);
+            static_cast<const XT*>(X), n_v, d, L.chunk_tokens, L.n_chunks, (const float*)w, token_scores, Ppart,
+            cnt, V, s_raw, A16, B16, N, (N + 7) & ~7);
 }
 
 int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
@@ -646,18 +681,33 @@ int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, co
   const ShardLayout L = shard_layout(N, n_v, d);
   float* w = reinterpret_cast<float*>(ws + L.w_off);
   float* Ppart = reinterpret_cast<float*>(ws + L.ppart_off);
-  launch_ex(fold_w_kernel, dim3((d + 255) / 256), dim3(256), 0, st, true, t, B, M, d, w);
+  // Large scenes finalise each tile inside the pass (no second read of the partial sums from
+  // HBM); below kFinalizeInPassTiles a separate kernel is faster (the pass is too short to hide
+  // the finalising CTAs' extra work: 0.458 against 0.441 ms per query at 400 tiles, 6.11 against
+  // 6.14 at 6400).
+  constexpr int kFinalizeInPassTiles = 3200;
+  const bool in_pass = N >= kFinalizeInPassTiles;
+  unsigned int* cnt = in_pass ? reinterpret_cast<unsigned int*>(ws + L.cnt_off) : nullptr;
+  launch_ex(fold_w_kernel, dim3((d + 255) / 256), dim3(256), 0, st, true, t, B, M, d, w, cnt, cnt ? N : 0);
   const int vw = (xdt == RIFT_BF16) ? 8 : 4;
   const int nvec_per_thread = (d / vw + SC_THREADS - 1) / SC_THREADS;
+  auto go = [&](auto xt, auto nvec) {
+    using XT = decltype(xt);
+    launch_tokens<XT, decltype(nvec)::value>(X, N, n_v, d, L, w, token_scores, Ppart, cnt, V, s_raw, A16, B16, st);
+  };
+  using I1 = std::integral_constant<int, 1>;
+  using I2 = std::integral_constant<int, 2>;
+  using I4 = std::integral_constant<int, 4>;
   if (xdt == RIFT_BF16) {
-    if (nvec_per_thread <= 1) launch_tokens<uint16_t, 1>(X, N, n_v, d, L, w, token_scores, Ppart, st);
-    else if (nvec_per_thread <= 2) launch_tokens<uint16_t, 2>(X, N, n_v, d, L, w, token_scores, Ppart, st);
-    else launch_tokens<uint16_t, 4>(X, N, n_v, d, L, w, token_scores, Ppart, st);
+    if (nvec_per_thread <= 1) go(uint16_t{}, I1{});
+    else if (nvec_per_thread <= 2) go(uint16_t{}, I2{});
+    else go(uint16_t{}, I4{});
   } else {
-    if (nvec_per_thread <= 1) launch_tokens<float, 1>(X, N, n_v, d, L, w, token_scores, Ppart, st);
-    else if (nvec_per_thread <= 2) launch_tokens<float, 2>(X, N, n_v, d, L, w, token_scores, Ppart, st);
-    else launch_tokens<float, 4>(X, N, n_v, d, L, w, token_scores, Ppart, st);
+    if (nvec_per_thread <= 1) go(float{}, I1{});
+    else if (nvec_per_thread <= 2) go(float{}, I2{});
+    else go(float{}, I4{});
   }
+  if (in_pass) return 2;
   launch_ex(tile_finalize_kernel, dim3(N), dim3(std::min(TF_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
             (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw, A16, B16, N, (N + 7) & ~7);
   return 3;
@@ -704,7 +754,7 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
                  cudaStream_t st) {
   const ScoreLayout L = score_layout(N, n_v, d, M);
   float* V = reinterpret_cast<float*>(ws + L.V_off);
-  // with neighbours to find, tile_finalize_kernel also writes the Gram's split operands
+  // with neighbours to find, the token pass's finalisation also writes the Gram's split operands
   uint16_t* A16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_a_off) : nullptr;
   uint16_t* B16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_b_off) : nullptr;
   const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws + L.tokens_off, st, A16,
