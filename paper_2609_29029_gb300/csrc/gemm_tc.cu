@@ -317,6 +317,12 @@ __device__ __forceinline__ void rope_chunk(const uint32_t (&r1)[32], const uint3
   }
 }
 
+// K-block k of an operand read through EpiParams' remap (mode 1: [hi | hi | lo], 2: [hi | lo | hi]
+// over a stored [hi | lo] row of D blocks each; 0: k).
+__device__ __forceinline__ int kblock(int mode, int D, int k) {
+  return mode == 1 ? (k < D ? k : k - D) : mode == 2 ? (k < 2 * D ? k : k - 2 * D) : k;
+}
+
 // BN_ x STAGES_: 256 x 4 for the prefill on one SM; 128 x 6 for few-row products with the
 // operands swapped (weights as the 128-row operand, the few activation rows as the N side;
 // EPI_STORE_F32_T).  PAIR: 2-CTA clusters on an SM pair, 256 x 256 tiles (cta_group::2): each SM
@@ -420,7 +426,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         n_pre = min(STAGES, k1 - k0);
         for (int j = 0; j < n_pre; ++j) {
           mbar_expect_tx(full_bar(j), STAGE_BYTES);
-          tma_load_2d(smem_u32(sA + j * A_BYTES), &tmA, (k0 + j) * BK, m_blk * BM, full_bar(j));
+          tma_load_2d(smem_u32(sA + j * A_BYTES), &tmA, kblock(ep.kmap_a, ep.kmap_d, k0 + j) * BK, m_blk * BM,
+                      full_bar(j));
         }
       }
       pdl_wait();
@@ -434,19 +441,22 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int s = it % STAGES;
           const uint32_t round = it / STAGES;
           if (it < n_pre) {  // A already requested (first round: the stage is free)
-            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, kblock(ep.kmap_b, ep.kmap_d, k) * BK, n_blk * BN,
+                        full_bar(s));
             continue;
           }
           if (!mbar_wait(empty_bar(s), (round & 1u) ^ 1u, abort_flag)) { ok = false; break; }
           if constexpr (PAIR) {
             const uint32_t fb = mapa_shared(full_bar(s), 0);
             if (rank == 0) mbar_expect_tx(full_bar(s), 2 * STAGE_BYTES);
-            tma_load_2d_pair(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * TM + (int)rank * BM, fb);
-            tma_load_2d_pair(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN + (int)rank * B_ROWS, fb);
+            tma_load_2d_pair(smem_u32(sA + s * A_BYTES), &tmA, kblock(ep.kmap_a, ep.kmap_d, k) * BK,
+                             m_blk * TM + (int)rank * BM, fb);
+            tma_load_2d_pair(smem_u32(sB + s * B_BYTES), &tmB, kblock(ep.kmap_b, ep.kmap_d, k) * BK,
+                             n_blk * BN + (int)rank * B_ROWS, fb);
           } else {
             mbar_expect_tx(full_bar(s), STAGE_BYTES);
-            tma_load_2d(smem_u32(sA + s * A_BYTES), &tmA, k * BK, m_blk * BM, full_bar(s));
-            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, k * BK, n_blk * BN, full_bar(s));
+            tma_load_2d(smem_u32(sA + s * A_BYTES), &tmA, kblock(ep.kmap_a, ep.kmap_d, k) * BK, m_blk * BM, full_bar(s));
+            tma_load_2d(smem_u32(sB + s * B_BYTES), &tmB, kblock(ep.kmap_b, ep.kmap_d, k) * BK, n_blk * BN, full_bar(s));
           }
         }
       }
@@ -1087,30 +1097,39 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   // Few rows (<= 128, with scratch: the decode step): the operands swapped so that the weights
   // stream as the 128-row operand in 128-row tiles and the rows sit on the N side (128 wide); the
   // slices' fp32 partials are stored transposed ([M, N] as the reductions below read them).
+  // The operands' stored row width: K, or 2 kmap_d blocks when read through the K-block remap.
+  if (ep.kmap_d && K != 3 * ep.kmap_d * BK) return 1;
+  const uint64_t Ks = ep.kmap_d ? (uint64_t)2 * ep.kmap_d * BK : (uint64_t)K;
+  EpiParams kp;  // the remap alone, for the partial products
+  kp.kmap_d = ep.kmap_d;
+  kp.kmap_a = ep.kmap_a;
+  kp.kmap_b = ep.kmap_b;
   if (split_ws && M <= 128 && (size_t)M * N * sizeof(float) <= split_ws_bytes) {
     constexpr int SW_BN = 128, SW_STAGES = 6;
     CUtensorMap mw, mx;
-    if (!make_map(&mw, B, (uint64_t)K, (uint64_t)N, BM) || !make_map(&mx, A, (uint64_t)K, (uint64_t)M, SW_BN)) return 1;
+    if (!make_map(&mw, B, Ks, (uint64_t)N, BM) || !make_map(&mx, A, Ks, (uint64_t)M, SW_BN)) return 1;
+    EpiParams ks = kp;  // the operands swapped: the kernel's A is B
+    ks.kmap_a = ep.kmap_b;
+    ks.kmap_b = ep.kmap_a;
     // a unit's partials (M x 128 fp32, written and read back) cost M / 16 K-blocks of weight
     // traffic; its fill and drain about 1.5 more
     const int splits = choose_splits(N, M, K, split_ws_bytes, SW_BN, M / 16.0 + 1.5);
     // constant weights (b_const) are requested before the wait on the kernel before this one
-    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, EpiParams(), st, splits, pdl,
-                                                  b_const ? 1 : 0))
+    if (launch<EPI_STORE_F32_T, SW_BN, SW_STAGES>(mw, mx, N, M, K, split_ws, ks, st, splits, pdl, b_const ? 1 : 0))
       return 1;
     EpiParams e = ep;
     e.symmetric = 0;
     return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, e, st, pdl);
   }
   CUtensorMap ma, mb;
-  if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) return 1;
+  if (!make_map(&ma, A, Ks, (uint64_t)M, BM) || !make_map(&mb, B, Ks, (uint64_t)N, BN)) return 1;
   // The residual product with a following RMSNorm (ep.norm_out) always goes through the
   // scratch, one slice or more, into the fused reduction + norm kernel.
   const bool fuse_norm = epi == EPI_RESID_F32 && ep.norm_out;
   if (fuse_norm && (!split_ws || N > 8192 || (size_t)M * N * sizeof(float) > split_ws_bytes)) return 1;
   const int splits = split_ws ? choose_splits(M, N, K, split_ws_bytes) : 1;
   if (splits > 1 || fuse_norm) {
-    if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, EpiParams(), st, splits, pdl)) return 1;
+    if (launch<EPI_STORE_F32>(ma, mb, M, N, K, split_ws, kp, st, splits, pdl)) return 1;
     EpiParams e = ep;
     e.symmetric = 0;
     return reduce_slices(static_cast<const float*>(split_ws), splits, M, N, epi, C, e, st, pdl);
@@ -1118,7 +1137,7 @@ int launch_gemm_tc(const void* A, const void* B, int M, int N, int K, int epi, v
   // Many rows: 256 x 256 tiles on SM pairs.
   if (M >= 1024) {
     CUtensorMap mb2;
-    if (!make_map(&mb2, B, (uint64_t)K, (uint64_t)N, BN / 2)) return 1;
+    if (!make_map(&mb2, B, Ks, (uint64_t)N, BN / 2)) return 1;
     int r = -1;
     switch (epi) {
       case EPI_STORE_BF16: r = launch_pair<EPI_STORE_BF16>(ma, mb2, M, N, K, C, ep, st); break;

@@ -26,7 +26,7 @@ struct ShardLayout {
 ShardLayout shard_layout(int N, int n_v, int d);
 // The kNN smoothing of n_rows rows against all N tiles (Appendix B Step 2).
 struct SmoothLayout {
-  size_t top_off, split_a_off, split_b_off, gram_off, splitk_off, splitk_bytes, total;
+  size_t top_off, split_off, gram_off, splitk_off, splitk_bytes, total;
 };
 SmoothLayout smooth_layout(int N, int n_rows, int d);
 // rift_score_tiles: V [N, d], then the token pass's scratch, which the smoothing of all N rows
@@ -49,11 +49,11 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
                  int M, int m, float* token_scores, float* s_raw, float* s_tilde, int* nbr, char* ws,
                  cudaStream_t st);
 // a2, a3 on N tiles: token scores, tile scores and the tile embeddings V [N, d] (ws: shard_layout).
-// A16, B16 (nullable): also write the whole scene's Gram operands (the layout of launch_smooth's
-// split_a / split_b), so that launch_smooth can skip its split.
+// S16 (nullable): also write the whole scene's Gram operand (the layout of launch_smooth's split
+// rows, [hi | lo] per tile), so that launch_smooth can skip its split.
 int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
                         int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st,
-                        uint16_t* A16 = nullptr, uint16_t* B16 = nullptr);
+                        uint16_t* S16 = nullptr);
 // a4 for tiles row0 .. row0 + n_rows - 1 of a scene of N tiles (V [N, d], s_raw [N]); s_tilde and
 // nbr are indexed by the local row (ws: smooth_layout).
 // split_done: the split operands in ws were written by launch_score_tokens (whole scene).
@@ -155,6 +155,11 @@ struct EpiParams {
   // only the tiles on and above the diagonal are computed, each off-diagonal one stored twice
   // (as itself and transposed).  Honoured on the SM-pair path; the other paths compute every tile.
   int symmetric = 0;
+  // K-block remap of the two operands (the kNN's split-operand Gram): with kmap_d > 0 each operand
+  // row is stored as [hi | lo], kmap_d K-blocks each (K = 3 kmap_d blocks of 64), and read as
+  // kmap_a / kmap_b: 1 = [hi | hi | lo], 2 = [hi | lo | hi] along K (0 = as stored).
+  int kmap_d = 0;
+  int kmap_a = 0, kmap_b = 0;
 };
 // split_ws (optional): scratch for split-K partial products; with it, products whose tiles leave
 // most SMs idle run as (tile, K-slice) units plus a reduction kernel.

@@ -157,14 +157,14 @@ constexpr float KNN_SPLIT_SCALE = 1024.f;
 // a3 for tile i, by one CTA of any size (MAXC >= the float4 columns a thread holds): P_i = sum of
 // the tile's n_chunks partials (in chunk order), V_i = P_i / ||P_i||, s_i = V_i . w.  A thread
 // takes the float4 columns threadIdx.x + k blockDim.x, so that its partial loads all issue
-// together; the partials are read through L2 (other CTAs wrote them).  With A16 and B16 (the whole
-// scene's Gram operands, Np rows of B) it also writes tile i's split rows, as knn_split_kernel
-// would from V, and its share of the zero padding rows of B.
+// together; the partials are read through L2 (other CTAs wrote them).  With S16 (the whole scene's
+// Gram operand, Np rows) it also writes tile i's split row, as knn_split_kernel would from V, and
+// its share of the zero padding rows.
 template <int MAXC>
 __device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ Ppart, int n_chunks, int d,
                                               const float* __restrict__ w, float* __restrict__ V,
-                                              float* __restrict__ s_raw, uint16_t* __restrict__ A16,
-                                              uint16_t* __restrict__ B16, int N, int Np, float* red) {
+                                              float* __restrict__ s_raw, uint16_t* __restrict__ S16, int N, int Np,
+                                              float* red) {
   const int nv = d / 4;
   float4 p[MAXC];
   float ss = 0.f;
@@ -192,7 +192,7 @@ __device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ P
     if (c < nv) {
       const float4 v = make_float4(p[k].x * inv, p[k].y * inv, p[k].z * inv, p[k].w * inv);
       reinterpret_cast<float4*>(V + (size_t)i * d)[c] = v;
-      if (B16) {
+      if (S16) {
         const float a[4] = {v.x * KNN_SPLIT_SCALE, v.y * KNN_SPLIT_SCALE, v.z * KNN_SPLIT_SCALE,
                             v.w * KNN_SPLIT_SCALE};
         uint32_t h[2], l[2];
@@ -202,15 +202,9 @@ __device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ P
           h[q] = pack_half2(__half2float(h0), __half2float(h1));
           l[q] = pack_half2(a[2 * q] - __half2float(h0), a[2 * q + 1] - __half2float(h1));
         }
-        const uint2 hv = make_uint2(h[0], h[1]), lv = make_uint2(l[0], l[1]);
-        uint2* b = reinterpret_cast<uint2*>(B16 + (size_t)i * 3 * d) + c;
-        uint2* a2 = reinterpret_cast<uint2*>(A16 + (size_t)i * 3 * d) + c;
-        b[0] = hv;
-        b[d / 4] = lv;
-        b[d / 2] = hv;
-        a2[0] = hv;
-        a2[d / 4] = hv;
-        a2[d / 2] = lv;
+        uint2* row = reinterpret_cast<uint2*>(S16 + (size_t)i * 2 * d) + c;  // [hi | lo]
+        row[0] = make_uint2(h[0], h[1]);
+        row[d / 4] = make_uint2(l[0], l[1]);
       }
       const float4 wc = reinterpret_cast<const float4*>(w)[c];
       dt += v.x * wc.x + v.y * wc.y + v.z * wc.z + v.w * wc.w;
@@ -218,10 +212,10 @@ __device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ P
   }
   dt = block_sum(dt, red);
   if (threadIdx.x == 0) s_raw[i] = dt;
-  if (B16)  // the padding rows N .. Np - 1 of B are zero: tile i takes rows N + i, N + i + N, ...
+  if (S16)  // the padding rows N .. Np - 1 are zero: tile i takes rows N + i, N + i + N, ...
     for (int r = N + i; r < Np; r += N)
-      for (int c = threadIdx.x; c < 3 * d / 8; c += blockDim.x)
-        reinterpret_cast<uint4*>(B16 + (size_t)r * 3 * d)[c] = make_uint4(0, 0, 0, 0);
+      for (int c = threadIdx.x; c < 2 * d / 8; c += blockDim.x)
+        reinterpret_cast<uint4*>(S16 + (size_t)r * 2 * d)[c] = make_uint4(0, 0, 0, 0);
 }
 
 // a3 after the token pass (small scenes): one CTA of up to 1024 threads per tile.
@@ -229,13 +223,12 @@ constexpr int TF_THREADS = 1024;
 __global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart, int n_chunks,
                                                                   int d, const float* __restrict__ w,
                                                                   float* __restrict__ V, float* __restrict__ s_raw,
-                                                                  uint16_t* __restrict__ A16,
-                                                                  uint16_t* __restrict__ B16, int N, int Np) {
+                                                                  uint16_t* __restrict__ S16, int N, int Np) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[32];
-  finalize_tile<(8192 / 4 + TF_THREADS - 1) / TF_THREADS>(blockIdx.x, Ppart, n_chunks, d, w, V, s_raw, A16, B16, N,
-                                                          Np, red);
+  finalize_tile<(8192 / 4 + TF_THREADS - 1) / TF_THREADS>(blockIdx.x, Ppart, n_chunks, d, w, V, s_raw, S16, N, Np,
+                                                          red);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -286,8 +279,7 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
     token_score_kernel(const XT* __restrict__ X, int n_v, int d, int chunk_tokens, int n_chunks,
                        const float* __restrict__ w, float* __restrict__ token_scores,
                        float* __restrict__ Ppart, unsigned int* __restrict__ cnt, float* __restrict__ V,
-                       float* __restrict__ s_raw, uint16_t* __restrict__ A16, uint16_t* __restrict__ B16, int N,
-                       int Np) {
+                       float* __restrict__ s_raw, uint16_t* __restrict__ S16, int N, int Np) {
   pdl_trigger();
   pdl_wait();
   using VT = VecTraits<XT>;
@@ -387,7 +379,7 @@ __global__ void __launch_bounds__(SC_THREADS, 2)
   __syncthreads();
   if (!last) return;
   __threadfence();
-  finalize_tile<(8192 / 4 + SC_THREADS - 1) / SC_THREADS>(tile, Ppart, n_chunks, d, w, V, s_raw, A16, B16, N, Np,
+  finalize_tile<(8192 / 4 + SC_THREADS - 1) / SC_THREADS>(tile, Ppart, n_chunks, d, w, V, s_raw, S16, N, Np,
                                                           &red[0][0]);
 }
 
@@ -403,15 +395,15 @@ __device__ __forceinline__ bool knn_better(float g, int j, float g2, int j2) {
   return g > g2 || (g == g2 && j < j2);
 }
 
-// The Gram matrix on the tensor cores.  Each fp32 row of V (scaled
-// by 2^10, so that the low parts stay normal in fp16) is split into hi = fp16(v) and
-// lo = fp16(v - hi); A = [hi | hi | lo] and B = [hi | lo | hi] along K, so one fp16 GEMM with
-// K = 3 d gives hi.hi + hi.lo + lo.hi, i.e. V V^T to ~2^-22 relative (lo.lo is below that).
-// B holds every tile; A the rows row0 .. row1 - 1 (A row i - row0).  Rows N .. Np - 1 of B (the
-// padding of the Gram matrix's column count to a multiple of 8) are zero.  A thread handles 8
-// consecutive elements of a row (two float4 loads, 16-byte stores into each of the row's parts).
-__global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, int row0, int row1,
-                                 uint16_t* __restrict__ A, uint16_t* __restrict__ B) {
+// The Gram matrix on the tensor cores.  Each fp32 row of V (scaled by 2^10, so that the low parts
+// stay normal in fp16) is split into hi = fp16(v) and lo = fp16(v - hi), stored once as the row
+// [hi | lo] of S (2 d fp16).  The product reads S twice through a K-block remap: A = [hi | hi | lo]
+// and B = [hi | lo | hi] along K, so one fp16 GEMM with K = 3 d gives hi.hi + hi.lo + lo.hi, i.e.
+// V V^T to ~2^-22 relative (lo.lo is below that).  S holds every tile; A is its rows row0 ..
+// row1 - 1.  Rows N .. Np - 1 of S (the padding of the Gram matrix's column count to a multiple of
+// 8) are zero.  A thread handles 8 consecutive elements of a row (two float4 loads, a 16-byte
+// store into each half of the row).
+__global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int d, uint16_t* __restrict__ S) {
   pdl_trigger();
   pdl_wait();
   const int n8 = d / 8;
@@ -419,12 +411,11 @@ __global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int
   if (idx >= (size_t)Np * n8) return;
   const size_t i = idx / n8;
   const int k = (int)(idx % n8) * 8;
-  uint4* b = reinterpret_cast<uint4*>(B + i * 3 * d + k);
+  uint4* row = reinterpret_cast<uint4*>(S + i * 2 * d + k);
   if (i >= (size_t)N) {
     const uint4 z = make_uint4(0, 0, 0, 0);
-    b[0] = z;
-    b[d / 8] = z;
-    b[d / 4] = z;
+    row[0] = z;
+    row[d / 8] = z;
     return;
   }
   const float4 v0 = reinterpret_cast<const float4*>(V + i * d + k)[0];
@@ -438,16 +429,8 @@ __global__ void knn_split_kernel(const float* __restrict__ V, int N, int Np, int
     h[q] = pack_half2(__half2float(h0), __half2float(h1));
     l[q] = pack_half2(a0 - __half2float(h0), a1 - __half2float(h1));
   }
-  const uint4 hv = make_uint4(h[0], h[1], h[2], h[3]), lv = make_uint4(l[0], l[1], l[2], l[3]);
-  b[0] = hv;
-  b[d / 8] = lv;
-  b[d / 4] = hv;
-  if (i >= (size_t)row0 && i < (size_t)row1) {
-    uint4* a = reinterpret_cast<uint4*>(A + (i - row0) * 3 * d + k);
-    a[0] = hv;
-    a[d / 8] = hv;
-    a[d / 4] = lv;
-  }
+  row[0] = make_uint4(h[0], h[1], h[2], h[3]);
+  row[d / 8] = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
 // One warp per row of the materialised Gram matrix: the row's 16 best columns (larger
@@ -615,7 +598,7 @@ int launch_query_prep(const void* embed, int vocab, int d, const int* phrase_ids
 }
 
 // Scratch of the kNN smoothing of rows row0 .. row0 + n_rows - 1 against all N tiles: the split
-// operands, the Gram rows, split-K partials when the product has fewer tiles than SMs (at most 16
+// rows of every tile, the Gram rows, split-K partials when the product has fewer tiles than SMs (at most 16
 // slices within 16 MB), the candidate lists.
 SmoothLayout smooth_layout(int N, int n_rows, int d) {
   SmoothLayout L{};
@@ -629,8 +612,7 @@ SmoothLayout smooth_layout(int N, int n_rows, int d) {
   part = part > 16 ? 16 : part;
   L.splitk_bytes = part >= 2 ? part * slice : 0;
   L.splitk_off = take(L.splitk_bytes);
-  L.split_a_off = take(sizeof(uint16_t) * (size_t)n_rows * 3 * d);  // the split operands last
-  L.split_b_off = take(sizeof(uint16_t) * Np * 3 * d);
+  L.split_off = take(sizeof(uint16_t) * Np * 2 * d);  // the split rows last
   L.total = off;
   return L;
 }
@@ -657,11 +639,11 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
   L.S = smooth_layout(N, N, d);
   // V first; after it the token pass's scratch (w, counters, partial pooled sums).  The
   // smoothing's scratch reuses the token scratch once the pass is over (the smoothing runs after it
-  // on the stream), except for its split operands, which the pass's finalising CTAs write while
-  // other tiles' partial sums are still in use: they start past the token scratch.
+  // on the stream), except for its split rows, which the pass's finalising CTAs write while other
+  // tiles' partial sums are still in use: they start past the token scratch.
   L.V_off = 0;
   L.tokens_off = (sizeof(float) * (size_t)N * d + 255) & ~size_t(255);
-  L.smooth_off = L.tokens_off + (L.T.total > L.S.split_a_off ? L.T.total - L.S.split_a_off : 0);
+  L.smooth_off = L.tokens_off + (L.T.total > L.S.split_off ? L.T.total - L.S.split_off : 0);
   L.total = L.smooth_off + L.S.total;
   return L;
 }
@@ -669,15 +651,15 @@ ScoreLayout score_layout(int N, int n_v, int d, int M) {
 template <typename XT, int NVEC>
 static void launch_tokens(const void* X, int N, int n_v, int d, const ShardLayout& L, const float* w,
                           float* token_scores, float* Ppart, unsigned int* cnt, float* V, float* s_raw,
-                          uint16_t* A16, uint16_t* B16, cudaStream_t st) {
+                          uint16_t* S16, cudaStream_t st) {
   launch_ex(token_score_kernel<XT, NVEC>, dim3(N * L.n_chunks), dim3(SC_THREADS), 0, st, true,
             static_cast<const XT*>(X), n_v, d, L.chunk_tokens, L.n_chunks, (const float*)w, token_scores, Ppart,
-            cnt, V, s_raw, A16, B16, N, (N + 7) & ~7);
+            cnt, V, s_raw, S16, N, (N + 7) & ~7);
 }
 
 int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, const float* t, const float* B,
                         int M, float* token_scores, float* s_raw, float* V, char* ws, cudaStream_t st,
-                        uint16_t* A16, uint16_t* B16) {
+                        uint16_t* S16) {
   const ShardLayout L = shard_layout(N, n_v, d);
   float* w = reinterpret_cast<float*>(ws + L.w_off);
   float* Ppart = reinterpret_cast<float*>(ws + L.ppart_off);
@@ -693,7 +675,7 @@ int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, co
   const int nvec_per_thread = (d / vw + SC_THREADS - 1) / SC_THREADS;
   auto go = [&](auto xt, auto nvec) {
     using XT = decltype(xt);
-    launch_tokens<XT, decltype(nvec)::value>(X, N, n_v, d, L, w, token_scores, Ppart, cnt, V, s_raw, A16, B16, st);
+    launch_tokens<XT, decltype(nvec)::value>(X, N, n_v, d, L, w, token_scores, Ppart, cnt, V, s_raw, S16, st);
   };
   using I1 = std::integral_constant<int, 1>;
   using I2 = std::integral_constant<int, 2>;
@@ -709,36 +691,38 @@ int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, co
   }
   if (in_pass) return 2;
   launch_ex(tile_finalize_kernel, dim3(N), dim3(std::min(TF_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
-            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw, A16, B16, N, (N + 7) & ~7);
+            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw, S16, N, (N + 7) & ~7);
   return 3;
 }
 
 int launch_smooth(const float* V, const float* s_raw, int N, int d, int row0, int n_rows, int m, float* s_tilde,
                   int* nbr, char* ws, cudaStream_t st, bool split_done) {
   const SmoothLayout L = smooth_layout(N, n_rows, d);
-  const int row1 = row0 + n_rows;
   int* topj = reinterpret_cast<int*>(ws + L.top_off);
   // candidates per row: m plus spares for the fp64 rescoring, at most the N - 1 other tiles
   const int C = m > 0 ? std::min(std::min(m + KNN_SPARE, RIFT_MAX_KNN), N - 1) : 0;
   int launched = 1;
   if (m > 0) {
-    uint16_t* A16 = reinterpret_cast<uint16_t*>(ws + L.split_a_off);
-    uint16_t* B16 = reinterpret_cast<uint16_t*>(ws + L.split_b_off);
+    uint16_t* S16 = reinterpret_cast<uint16_t*>(ws + L.split_off);
     float* G = reinterpret_cast<float*>(ws + L.gram_off);
     const int Np = (N + 7) & ~7;
     const size_t n = (size_t)Np * (d / 8);
     if (!split_done)
-      launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, row0,
-                row1, A16, B16);
+      launch_ex(knn_split_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, true, V, N, Np, d, S16);
     EpiParams ep;
     ep.out_scale = 1.f / (KNN_SPLIT_SCALE * KNN_SPLIT_SCALE);
+    // A = rows row0 .. row0 + n_rows - 1 of S read as [hi | hi | lo], B = all of S as [hi | lo | hi]
+    ep.kmap_d = d / 64;
+    ep.kmap_a = 1;
+    ep.kmap_b = 2;
     // the whole scene's rows: G is symmetric (A holds the same rows as B, in the permuted parts
     // [hi | hi | lo] against [hi | lo | hi], whose product is symmetric up to the order of its sums)
     ep.symmetric = (row0 == 0 && n_rows == N) ? 1 : 0;
     // split-K partials for products with fewer tiles than SMs (a scene up to ~2000 tiles)
     void* part = L.splitk_bytes ? static_cast<void*>(ws + L.splitk_off) : nullptr;
-    // B16 is the split kernel's output, not a constant operand
-    if (launch_gemm_tc(A16, B16, n_rows, Np, 3 * d, EPI_STORE_F32, G, ep, st, part, L.splitk_bytes, true, false))
+    // S is written by an earlier kernel of the chain, not a constant operand
+    if (launch_gemm_tc(S16 + (size_t)row0 * 2 * d, S16, n_rows, Np, 3 * d, EPI_STORE_F32, G, ep, st, part,
+                       L.splitk_bytes, true, false))
       return -1;
     launch_ex(knn_gram_topc_kernel, dim3((n_rows + 3) / 4), dim3(128), 0, st, true, (const float*)G, N, Np, row0,
               n_rows, C, topj);
@@ -754,11 +738,9 @@ int launch_score(const void* X, rift_dtype xdt, int N, int n_v, int d, const flo
                  cudaStream_t st) {
   const ScoreLayout L = score_layout(N, n_v, d, M);
   float* V = reinterpret_cast<float*>(ws + L.V_off);
-  // with neighbours to find, the token pass's finalisation also writes the Gram's split operands
-  uint16_t* A16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_a_off) : nullptr;
-  uint16_t* B16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_b_off) : nullptr;
-  const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws + L.tokens_off, st, A16,
-                                    B16);
+  // with neighbours to find, the token pass's finalisation also writes the Gram's split rows
+  uint16_t* S16 = m > 0 ? reinterpret_cast<uint16_t*>(ws + L.smooth_off + L.S.split_off) : nullptr;
+  const int a = launch_score_tokens(X, xdt, N, n_v, d, t, B, M, token_scores, s_raw, V, ws + L.tokens_off, st, S16);
   const int b = launch_smooth(V, s_raw, N, d, 0, N, m, s_tilde, nbr, ws + L.smooth_off, st, m > 0);
   return b < 0 ? -1 : a + b;
 }
