@@ -23,22 +23,21 @@ unsigned int read_clear_err_pack() {
 constexpr int PK_ROWS = 32;
 constexpr int PK_THREADS = 256;
 
-// cu_seqlens[j] = row_base + min(j, n) (S + Q) + sel_off[min(j, n)] + ctx_off[min(j, n)],
-// T = cu_seqlens[n] - row_base (row_base: rows of the queries packed before this one).
-__global__ void seqlens_kernel(const int* __restrict__ n_kept, const int* __restrict__ sel_off,
-                               const int* __restrict__ ctx_off, int N, int S, int Q, int max_T, int row_base,
-                               int* __restrict__ cu, int* __restrict__ T) {
-  pdl_trigger();
-  pdl_wait();
-  const int n = *n_kept;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= N; j += gridDim.x * blockDim.x) {
-    const int jj = min(j, n);
-    const int v = jj * (S + Q) + sel_off[jj] + (ctx_off ? ctx_off[jj] : 0);
-    cu[j] = row_base + v;
-    if (j == N) {
-      *T = v;
-      if (v > max_T) atomicOr(&g_err_pack, RIFT_EBIT_CAPACITY);
-    }
+// The sequence offsets of the prefill, written by thread 0 of CTA (j, 0) of the packing kernels:
+// cu_seqlens[j] = row_base + min(j, n) (S + Q) + sel_off[min(j, n)] + ctx_off[min(j, n)], and CTA
+// (N - 1, 0) also writes cu_seqlens[N] and T = cu_seqlens[N] - row_base (row_base: rows of the
+// queries packed before this one); T over max_T sets RIFT_EBIT_CAPACITY.  (The packing itself
+// computes each sequence's first row the same way.)
+__device__ __forceinline__ void write_offsets(int j, int n, int N, const int* __restrict__ sel_off,
+                                              const int* __restrict__ ctx_off, int S, int Q, int max_T, int row_base,
+                                              int* __restrict__ cu, int* __restrict__ T) {
+  auto off = [&](int jj) { return jj * (S + Q) + sel_off[jj] + (ctx_off ? ctx_off[jj] : 0); };
+  cu[j] = row_base + off(min(j, n));
+  if (j == N - 1) {
+    const int v = off(min(N, n));
+    cu[N] = row_base + v;
+    *T = v;
+    if (v > max_T) atomicOr(&g_err_pack, RIFT_EBIT_CAPACITY);
   }
 }
 
@@ -48,11 +47,14 @@ __global__ void __launch_bounds__(PK_THREADS) pack_kernel(
     const int* __restrict__ n_kept, const int* __restrict__ sel, const int* __restrict__ sel_off,
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
     const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
-    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
+    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions,
+    int row_base, int* __restrict__ cu, int* __restrict__ T) {
   pdl_trigger();
   pdl_wait();
   const int j = blockIdx.x;
-  if (j >= *n_kept) return;
+  const int nk = *n_kept;
+  if (blockIdx.y == 0 && threadIdx.x == 0) write_offsets(j, nk, N, sel_off, ctx_off, S, Q, max_T, row_base, cu, T);
+  if (j >= nk) return;
   const int so = sel_off[j];
   const int dom = sel_off[j + 1] - so;  // selected tokens, then m contextual ones
   const int co = ctx_off ? ctx_off[j] : 0, m = ctx_off ? ctx_off[j + 1] - co : 0;
@@ -137,13 +139,16 @@ __global__ void __launch_bounds__(64) pack_bulk_kernel(
     const int* __restrict__ n_kept, const int* __restrict__ sel, const int* __restrict__ sel_off,
     const int* __restrict__ sys_ids, int S, const int* __restrict__ query_ids, int Q,
     const uint16_t* __restrict__ embed, int vocab, const uint16_t* __restrict__ ctx,
-    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions) {
+    const int* __restrict__ ctx_off, uint16_t* __restrict__ packed, int max_T, int* __restrict__ positions,
+    int row_base, int* __restrict__ cu, int* __restrict__ T) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(128) uint8_t ring[];
   __shared__ __align__(8) uint64_t bars[PKB_SLOTS];
   const int j = blockIdx.x;
-  if (j >= *n_kept) return;
+  const int nk = *n_kept;
+  if (blockIdx.y == 0 && threadIdx.x == 0) write_offsets(j, nk, N, sel_off, ctx_off, S, Q, max_T, row_base, cu, T);
+  if (j >= nk) return;
   const int so = sel_off[j];
   const int dom = sel_off[j + 1] - so;  // selected tokens, then m contextual ones
   const int co = ctx_off ? ctx_off[j] : 0, m = ctx_off ? ctx_off[j + 1] - co : 0;
@@ -227,8 +232,6 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
                  const int* query_ids, int Q, const void* embed, int vocab, const void* ctx, const int* ctx_off,
                  void* packed, int max_T, int* cu_seqlens, int* positions, int* T, int row_base,
                  cudaStream_t st) {
-  launch_ex(seqlens_kernel, dim3((N + 1 + 255) / 256), dim3(256), 0, st, true, n_kept, sel_off, ctx_off, N, S, Q,
-            max_T, row_base, cu_seqlens, T);
   const uint16_t* cx = static_cast<const uint16_t*>(ctx);
   const int max_L = S + n_v + Q;
   dim3 grid(N, (max_L + PK_ROWS - 1) / PK_ROWS);
@@ -240,11 +243,11 @@ void launch_pack(const void* X, rift_dtype xdt, int N, int n_v, int d, const int
     dim3 gb(N, (max_L + PKB_ROWS - 1) / PKB_ROWS);
     launch_ex(pack_bulk_kernel, gb, dim3(64), smem, st, true, static_cast<const uint16_t*>(X), N, n_v, d, kept,
               n_kept, sel, sel_off, sys_ids, S, query_ids, Q, static_cast<const uint16_t*>(embed), vocab, cx, ctx_off,
-              static_cast<uint16_t*>(packed), max_T, positions);
+              static_cast<uint16_t*>(packed), max_T, positions, row_base, cu_seqlens, T);
   } else
     launch_ex(pack_kernel<float>, grid, dim3(PK_THREADS), 0, st, true, static_cast<const float*>(X), N, n_v, d, kept,
               n_kept, sel, sel_off, sys_ids, S, query_ids, Q, static_cast<const uint16_t*>(embed), vocab, cx, ctx_off,
-              static_cast<uint16_t*>(packed), max_T, positions);
+              static_cast<uint16_t*>(packed), max_T, positions, row_base, cu_seqlens, T);
 }
 
 }  // namespace rift
