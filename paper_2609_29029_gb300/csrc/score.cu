@@ -453,15 +453,18 @@ __global__ void knn_gram_topc_kernel(const float* __restrict__ G, int N, int ld,
   int tj = 0x7fffffff;
   const float* row = G + (size_t)il * ld;
   bool bad = false;
-  for (int j0 = 0; j0 < N; j0 += 128) {
-    float gv[4];
+  // 16 loads in flight per lane (512 columns per step): a step is bounded by the loads' latency,
+  // not by the insertions, so fewer and wider steps finish a row sooner
+  constexpr int NL = 16;
+  for (int j0 = 0; j0 < N; j0 += 32 * NL) {
+    float gv[NL];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {  // four loads in flight per lane
+    for (int q = 0; q < NL; ++q) {
       const int j = j0 + 32 * q + lane;
       gv[q] = j < N ? row[j] : -INFINITY;
     }
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < NL; ++q) {
       const int j = j0 + 32 * q + lane;
       float g = gv[q];
       if (!(g == g)) {
@@ -523,6 +526,7 @@ __global__ void __launch_bounds__(32 * RIFT_MAX_KNN) knn_rescore_smooth_kernel(
     if (j >= 0 && j < N) {
       const float4* vi = reinterpret_cast<const float4*>(V + (size_t)i * d);
       const float4* vj = reinterpret_cast<const float4*>(V + (size_t)j * d);
+#pragma unroll 4
       for (int k = lane; k < d / 4; k += 32) {
         const float4 a4 = vi[k], b4 = vj[k];
         const float av[4] = {a4.x, a4.y, a4.z, a4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
