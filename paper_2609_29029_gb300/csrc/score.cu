@@ -218,17 +218,18 @@ __device__ __forceinline__ void finalize_tile(int i, const float* __restrict__ P
         reinterpret_cast<uint4*>(S16 + (size_t)r * 2 * d)[c] = make_uint4(0, 0, 0, 0);
 }
 
-// a3 after the token pass (small scenes): one CTA of up to 1024 threads per tile.
-constexpr int TF_THREADS = 1024;
-__global__ void __launch_bounds__(TF_THREADS) tile_finalize_kernel(const float* __restrict__ Ppart, int n_chunks,
-                                                                  int d, const float* __restrict__ w,
-                                                                  float* __restrict__ V, float* __restrict__ s_raw,
-                                                                  uint16_t* __restrict__ S16, int N, int Np) {
+// a3 after the token pass (scenes below the in-pass size): one CTA per tile of the token pass's
+// width, SC_THREADS, so that the finalisation's sums (and V, bit for bit) are the same whichever
+// kernel runs it and whatever the scene's or shard's size; each thread has four float4 columns of
+// loads in flight (d = 4096).
+__global__ void __launch_bounds__(256) tile_finalize_kernel(const float* __restrict__ Ppart, int n_chunks, int d,
+                                                           const float* __restrict__ w, float* __restrict__ V,
+                                                           float* __restrict__ s_raw, uint16_t* __restrict__ S16,
+                                                           int N, int Np) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[32];
-  finalize_tile<(8192 / 4 + TF_THREADS - 1) / TF_THREADS>(blockIdx.x, Ppart, n_chunks, d, w, V, s_raw, S16, N, Np,
-                                                          red);
+  finalize_tile<8192 / 4 / 256>(blockIdx.x, Ppart, n_chunks, d, w, V, s_raw, S16, N, Np, red);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -694,8 +695,9 @@ int launch_score_tokens(const void* X, rift_dtype xdt, int N, int n_v, int d, co
     else go(float{}, I4{});
   }
   if (in_pass) return 2;
-  launch_ex(tile_finalize_kernel, dim3(N), dim3(std::min(TF_THREADS, (d / 4 + 31) / 32 * 32)), 0, st, true,
-            (const float*)Ppart, L.n_chunks, d, (const float*)w, V, s_raw, S16, N, (N + 7) & ~7);
+  static_assert(SC_THREADS == 256, "the separate finalisation has the token pass's width");
+  launch_ex(tile_finalize_kernel, dim3(N), dim3(SC_THREADS), 0, st, true, (const float*)Ppart, L.n_chunks, d,
+            (const float*)w, V, s_raw, S16, N, (N + 7) & ~7);
   return 3;
 }
 

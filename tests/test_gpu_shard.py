@@ -33,10 +33,13 @@ def _sharded(wl, sc, dv, R, cuda, model=None):
     return shard.run_inprocess([shard.sharded_query(e, r, R, s.N, dec=dec) for r, e in enumerate(engines)])
 
 
-@pytest.mark.parametrize("name,R", [("small24_f32", 2), ("ragged40_bf16", 3), ("sweep400", 4), ("sweep1600", 3)])
+# sweep6400 over 3 ranks: the whole scene finalises its tiles inside the token pass, the shards of
+# 2133 tiles in the separate kernel; both must give the same bits
+@pytest.mark.parametrize("name,R", [("small24_f32", 2), ("ragged40_bf16", 3), ("sweep400", 4), ("sweep1600", 3),
+                                    ("sweep6400", 3)])
 def test_sharded_selection_equals_single_rank(name, R, cuda, riftlib):
     wl = {"small24_f32": P.SMALL24, "ragged40_bf16": P.RAGGED, "sweep400": W.sweep_workload(400),
-          "sweep1600": W.sweep_workload(1600)}[name]
+          "sweep1600": W.sweep_workload(1600), "sweep6400": W.sweep_workload(6400)}[name]
     sc = W.make_scene(wl.scene, wl.decoder.vocab, cuda)
     r1, dv = _single(wl, sc, cuda)
     res = _sharded(wl, sc, dv, R, cuda)
